@@ -1,0 +1,512 @@
+"""Benchmark of the verify step on GB300: prints ONE JSON line.
+
+Workload: the 8B-class target verify step of the paper's speculative-decoding
+loop (Sec. 2.2 Eq. verify; target shape from Sec. 4 "Targets and drafts":
+Qwen3-VL-8B backbone, 36 layers). Per scene and step, every one of the 36
+layers runs, on its own KV cache (L = 4096 prefix = 4 cameras x 896 patches +
+512 text tokens, 32 query / 8 KV heads x 128, bf16):
+    M-RoPE of the K + 1 = 8 new Q/K rows (sections [16,24,24], base 1e6)
+    KV append of the 8 rows
+    verify attention of the 8 causal rows over 4104 keys
+then one greedy acceptance over bf16 logits [8, 151936] and the KV rollback
+of all 36 layers to the committed length. After the timed work of a step the
+lengths are put back to L (one 144-byte device copy) so that every step
+processes the same L = 4096 workload.
+
+The 36 caches (605 MB) exceed the 129 MB L2, so every step streams its KV
+from HBM: "inputs larger than L2". The whole step is captured once in a CUDA
+graph and replayed. Multi-GPU: one independent replica per rank (scenes are
+independent: weak scaling, no data-path collective).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+"""
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "verify-step µs & HBM GB/s vs ~8 TB/s at L=4096,K=7,32q/8kv; accept µs"
+LAYERS = 36
+L, K, HQ, HKV, D, V = 4096, 7, 32, 8, 128, 151936
+R = K + 1
+SECTIONS = (16, 24, 24)
+BASE = 1e6
+
+
+# ------------------------------------------------------------ byte accounting
+def attention_bytes(B=1):
+    """Algorithmic bytes of one verify-attention launch: K and V of L + R keys
+    for every KV head, plus the Q rows read and the O rows written."""
+    kv = B * (L + R) * HKV * D * 2 * 2
+    qo = 2 * B * R * HQ * D * 2
+    return kv + qo
+
+
+def layer_bytes(B=1):
+    rope = 2 * B * R * (HQ + HKV) * D * 2          # read + write Q and K rows
+    append = 2 * 2 * B * R * HKV * D * 2           # read K/V rows, write them
+    return attention_bytes(B) + rope + append
+
+
+def step_bytes(B=1):
+    accept = B * R * V * 2 + B * K * 4 + B * (2 * R + 1) * 4
+    rollback = 2 * LAYERS * B * 4 + B * 4
+    return LAYERS * layer_bytes(B) + accept + rollback
+
+
+# ------------------------------------------------------------------ helpers
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+def kernel_source_hash():
+    path = os.path.join(ROOT, "paper_2606_31160_gb300", "csrc", "attention.cu")
+    with open(path, "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()
+
+
+def ncu_traffic():
+    """DRAM bytes per verify-attention launch from the committed ncu summary,
+    or None when the kernel source changed since the counters were taken."""
+    path = os.path.join(ROOT, "profiles", "ncu_traffic.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)["verify_attention"]
+        if d.get("src_sha256") == kernel_source_hash():
+            return float(d["dram_bytes_per_launch"])
+    except Exception:
+        pass
+    return None
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled during the timed region."""
+    FIELDS = ["clocks.sm", "clocks.max.sm", "clocks_event_reasons.hw_slowdown",
+              "clocks_event_reasons.hw_thermal_slowdown", "clocks_event_reasons.sw_thermal_slowdown",
+              "clocks_event_reasons.sw_power_cap"]
+    NAMES = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+
+    def __init__(self, index):
+        self.index = index
+        self.samples = []
+        self._stop = threading.Event()
+        self._thread = None
+
+    def _one(self):
+        try:
+            out = subprocess.run(["nvidia-smi", "-i", str(self.index), "--query-gpu=" + ",".join(self.FIELDS),
+                                  "--format=csv,noheader,nounits"], capture_output=True, text=True, timeout=5)
+            parts = [p.strip() for p in out.stdout.strip().split(",")]
+            if len(parts) == len(self.FIELDS):
+                self.samples.append(parts)
+        except Exception:
+            pass
+
+    def _run(self):
+        while not self._stop.is_set():
+            self._one()
+            self._stop.wait(0.1)
+
+    def __enter__(self):
+        self._thread = threading.Thread(target=self._run, daemon=True)
+        self._thread.start()
+        return self
+
+    def __exit__(self, *exc):
+        self._stop.set()
+        self._thread.join(timeout=10)
+        if not self.samples:
+            self._one()
+
+    def summary(self):
+        if not self.samples:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        sm = [float(s[0]) for s in self.samples if s[0].replace(".", "").isdigit()]
+        mx = [float(s[1]) for s in self.samples if s[1].replace(".", "").isdigit()]
+        reasons = set()
+        for s in self.samples:
+            for name, val in zip(self.NAMES, s[2:]):
+                if val.strip().lower() == "active":
+                    reasons.add(name)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": sorted(reasons), "samples": len(self.samples)}
+
+
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+# ------------------------------------------------------------- workload
+class Step:
+    """Device-resident inputs and outputs of one verify step (one scene)."""
+
+    def __init__(self, device):
+        from paper_2606_31160_gb300 import sd, workloads
+        self.sd = sd
+        self.device = device
+        gen_t0 = time.time()
+        self.cases = [workloads.target_layer(B=1, layer=l, ell=[3]) for l in range(LAYERS)]
+        self.gen_s = time.time() - gen_t0
+        c0 = self.cases[0]
+        # host copies (pinned) of the per-step inputs, for the end-to-end leg
+        self.h_q = torch.stack([c.q for c in self.cases]).pin_memory()          # [36,1,R,HQ,D]
+        self.h_k = torch.stack([c.k_new for c in self.cases]).pin_memory()
+        self.h_v = torch.stack([c.v_new for c in self.cases]).pin_memory()
+        self.h_pos = c0.pos.clone().pin_memory()
+        self.h_logits = c0.extra["logits"].clone().pin_memory()
+        self.h_draft = c0.extra["draft"].clone().pin_memory()
+        # device buffers
+        self.q = self.h_q.to(device)
+        self.k = self.h_k.to(device)
+        self.v = self.h_v.to(device)
+        self.pos = self.h_pos.to(device)
+        self.logits = self.h_logits.to(device)
+        self.draft = self.h_draft.to(device)
+        self.lens = torch.full((LAYERS, 1), L, dtype=torch.int32, device=device)
+        self.lens0 = self.lens.clone()
+        self.caches = [sd.KVCache(c.k_cache.to(device), c.v_cache.to(device), self.lens[l])
+                       for l, c in enumerate(self.cases)]
+        self.out = torch.empty_like(self.q)
+        self.ws = sd.workspace(sd.greedy_workspace_bytes(1, K, V), device)
+        self.n_emit = torch.zeros(1, dtype=torch.int32, device=device)
+        self.tokens = torch.zeros((1, R), dtype=torch.int32, device=device)
+        self.argmax = torch.zeros((1, R), dtype=torch.int32, device=device)
+        self.h_out = torch.zeros((1 + R,), dtype=torch.int32).pin_memory()
+        for c in self.cases:  # free host copies of the caches
+            c.k_cache = c.v_cache = None
+
+    def run(self):
+        sd = self.sd
+        for l in range(LAYERS):
+            sd.rope_apply(self.q[l], self.k[l], self.pos, SECTIONS, 0, BASE)
+            sd.kv_append(self.caches[l], self.k[l], self.v[l])
+            sd.verify_attention(self.q[l], self.caches[l], out=self.out[l])
+        sd.accept_greedy(self.logits, self.draft, ws=self.ws, n_emit=self.n_emit, tokens=self.tokens,
+                         argmax=self.argmax)
+        sd.kv_rollback(self.lens, self.n_emit, R)
+        self.lens.copy_(self.lens0, non_blocking=True)
+
+    def attention_only(self):
+        for l in range(LAYERS):
+            self.sd.verify_attention(self.q[l], self.caches[l], out=self.out[l])
+
+    def accept_only(self):
+        self.sd.accept_greedy(self.logits, self.draft, ws=self.ws, n_emit=self.n_emit, tokens=self.tokens,
+                              argmax=self.argmax)
+
+    def h2d(self):
+        self.q.copy_(self.h_q, non_blocking=True)
+        self.k.copy_(self.h_k, non_blocking=True)
+        self.v.copy_(self.h_v, non_blocking=True)
+        self.pos.copy_(self.h_pos, non_blocking=True)
+        self.logits.copy_(self.h_logits, non_blocking=True)
+        self.draft.copy_(self.h_draft, non_blocking=True)
+
+    def d2h(self):
+        self.h_out[:1].copy_(self.n_emit, non_blocking=True)
+        self.h_out[1:].copy_(self.tokens[0], non_blocking=True)
+
+    @property
+    def h2d_bytes(self):
+        return sum(t.numel() * t.element_size() for t in (self.h_q, self.h_k, self.h_v, self.h_pos,
+                                                          self.h_logits, self.h_draft))
+
+    @property
+    def d2h_bytes(self):
+        return (1 + R) * 4
+
+
+def capture(fn):
+    g = torch.cuda.CUDAGraph()
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(s):
+        fn()  # warm once on the capture stream
+    torch.cuda.current_stream().wait_stream(s)
+    torch.cuda.synchronize()
+    with torch.cuda.graph(g):
+        fn()
+    torch.cuda.synchronize()
+    return g
+
+
+def time_graph(g, reps, warm=3):
+    for _ in range(warm):
+        g.replay()
+    torch.cuda.synchronize()
+    st = torch.cuda.current_stream()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(st)
+    for _ in range(reps):
+        g.replay()
+    e1.record(st)
+    e1.synchronize()
+    return e0.elapsed_time(e1) / reps  # ms
+
+
+# ------------------------------------------------------------- CPU oracle
+def oracle_layer_sample(case, logits, draft):
+    """The float64 oracle on one layer of the step plus the acceptance:
+    returns bytes of the workload it covered (same accounting as the GPU)."""
+    import oracle
+    f64 = lambda t: t.float().numpy().astype(np.float64)
+    pos = case.pos.numpy()[:, :, None, :]
+    q = oracle.mrope_apply(f64(case.q), pos, SECTIONS, 0, BASE)
+    k = oracle.mrope_apply(f64(case.k_new), pos, SECTIONS, 0, BASE)
+    kc, vc, lens = oracle.kv_append(f64(case.k_cache), f64(case.v_cache), case.prefix, k, f64(case.v_new))
+    oracle.verify_attention(q, kc, vc, lens)
+    n_emit, _, _ = oracle.accept_greedy(f64(logits), draft.numpy())
+    oracle.kv_rollback(lens, n_emit, R)
+    return layer_bytes(1) + (step_bytes(1) - LAYERS * layer_bytes(1))
+
+
+def cpu_threads():
+    try:
+        from threadpoolctl import threadpool_info
+        n = max((i.get("num_threads", 1) for i in threadpool_info()), default=1)
+        return int(n)
+    except Exception:
+        return len(os.sched_getaffinity(0))
+
+
+def time_oracle(budget_s, max_layers=None):
+    """Oracle leg: whole layers of the step (rope, append, attention) plus the
+    acceptance and rollback, repeated until budget_s is spent."""
+    from paper_2606_31160_gb300 import workloads
+    case = workloads.target_layer(B=1, layer=0, ell=[3])
+    logits, draft = case.extra["logits"], case.extra["draft"]
+    done_bytes, t0, n = 0, time.perf_counter(), 0
+    while True:
+        done_bytes += oracle_layer_sample(case, logits, draft)
+        n += 1
+        el = time.perf_counter() - t0
+        if el >= budget_s or (max_layers and n >= max_layers):
+            break
+    return done_bytes / el / 1e9, n, el
+
+
+# ------------------------------------------------------------------ main
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--cpu-budget", type=float, default=12.0, help="seconds of oracle time (rank 0)")
+    args = ap.parse_args()
+    world, rank, local = dist_env()
+    if args.warmup < 3:
+        args.warmup = 3
+
+    if args.impl == "reference":
+        return reference_arm(args, world, rank)
+
+    import torch.distributed as dist
+    torch.cuda.set_device(local)
+    device = torch.device("cuda", local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=device)
+
+    from paper_2606_31160_gb300 import build, sd
+    build.build()
+    sd.lib()
+
+    st = Step(device)
+    # eager warm-up (sets kernel attributes before any capture), then graphs
+    for _ in range(2):
+        st.run()
+    torch.cuda.synchronize()
+    g_step = capture(st.run)
+    g_attn = capture(st.attention_only)
+    g_acc = capture(st.accept_only)
+    for _ in range(args.warmup):
+        g_step.replay()
+    torch.cuda.synchronize()
+    assert sd.get_device_error() == 0
+
+    # ---- timed region: K whole steps
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    stream = torch.cuda.current_stream()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(local) as clocks:
+        e0.record(stream)
+        for _ in range(args.steps):
+            g_step.replay()
+        e1.record(stream)
+        e1.synchronize()
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    ms_total = e0.elapsed_time(e1)
+    t = torch.tensor([ms_total], dtype=torch.float64, device=device)
+    if world > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    ms_total = float(t.item())
+    ms_step = ms_total / args.steps
+
+    # ---- dominant kernel: verify attention alone (36 distinct caches per replay)
+    reps = max(20, min(2000, args.steps))
+    ms_attn_launch = time_graph(g_attn, reps) / LAYERS
+    ms_accept = time_graph(g_acc, reps)
+
+    # ---- end to end: pinned host inputs -> device, step, result -> host
+    e2e_steps = max(10, min(500, args.steps))
+    for _ in range(3):
+        st.h2d(); g_step.replay(); st.d2h()
+    torch.cuda.synchronize()
+    a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a0.record(stream)
+    for _ in range(e2e_steps):
+        st.h2d()
+        g_step.replay()
+        st.d2h()
+    a1.record(stream)
+    a1.synchronize()
+    ms_e2e = a0.elapsed_time(a1) / e2e_steps
+    te = torch.tensor([ms_e2e], dtype=torch.float64, device=device)
+    if world > 1:
+        dist.all_reduce(te, op=dist.ReduceOp.MAX)
+    ms_e2e = float(te.item())
+    assert sd.get_device_error() == 0
+
+    if rank != 0:
+        if world > 1:
+            dist.barrier()
+            dist.destroy_process_group()
+        return
+
+    peak, peak_kind = measured_peaks()
+    bytes_step = step_bytes(1) * world
+    value = bytes_step / (ms_step * 1e-3) / 1e9
+    achieved = attention_bytes(1) / (ms_attn_launch * 1e-3) / 1e9
+    traffic = ncu_traffic()
+    cpu_gbs, cpu_layers, cpu_s = time_oracle(args.cpu_budget)
+    line = {
+        "metric": METRIC,
+        "value": round(value, 2),
+        "unit": "GB/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(ms_step, 5),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic (seeded Philox; no clips or weights exist here)",
+        "config": {
+            "workload": "8B-class target verify step: 36 layers x (M-RoPE + KV append + verify attention, "
+                        "L=4096, K=7, 32q/8kv x 128, bf16) + greedy accept over bf16 logits V=151936 + rollback",
+            "batch_per_gpu": 1, "layers": LAYERS, "prefix_len": L, "K": K, "q_heads": HQ, "kv_heads": HKV,
+            "head_dim": D, "vocab": V, "mrope_section": list(SECTIONS), "rope_base": BASE,
+            "parallelism": "replicas" if world > 1 else "single-gpu",
+            "l2": "inputs larger than L2: 36 distinct KV caches (605 MB) streamed per step",
+            "timing": "CUDA graph of one step, replayed; CUDA events on the launching stream",
+        },
+        "verify_step_us": round(ms_step * 1e3, 3),
+        "per_layer_us": round(ms_step * 1e3 / LAYERS, 3),
+        "attention_us": round(ms_attn_launch * 1e3, 3),
+        "accept_us": round(ms_accept * 1e3, 3),
+        "bytes_per_step": step_bytes(1),
+        "roofline": {
+            "kernel": "sd_verify_attention (verify_attn_kernel<128,2,1>)",
+            "bound": "hbm",
+            "achieved": round(achieved, 1),
+            "peak": peak,
+            "peak_kind": peak_kind,
+            "unit": "GB/s",
+            "frac": round(achieved / peak, 4),
+            "traffic": traffic,
+            "algorithmic_bytes_per_launch": attention_bytes(1),
+        },
+        "cpu_baseline": {
+            "value": round(cpu_gbs, 4),
+            "unit": "GB/s",
+            "cores": cpu_threads(),
+            "kind": "oracle",
+            "sample": "%d full target layers (M-RoPE, append, attention over 4104 keys, all 32 heads) each "
+                      "with the greedy accept over 8 x 151936 and the rollback, float64 numpy, %.1f s"
+                      % (cpu_layers, cpu_s),
+        },
+        "e2e": {
+            "value": round(bytes_step / (ms_e2e * 1e-3) / 1e9, 2),
+            "unit": "GB/s",
+            "ms_per_step": round(ms_e2e, 5),
+            "h2d_bytes_per_step": st.h2d_bytes,
+            "d2h_bytes_per_step": st.d2h_bytes,
+        },
+        "gpu_launches": args.steps * (3 * LAYERS + 2),
+        "clocks": clocks.summary(),
+    }
+    print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.barrier()
+        dist.destroy_process_group()
+
+
+def reference_arm(args, world, rank):
+    """The float64 oracle run as the reference arm on the host cores: each
+    step is one full layer of the workload plus the acceptance and rollback."""
+    if rank != 0:
+        return
+    from paper_2606_31160_gb300 import workloads
+    case = workloads.target_layer(B=1, layer=0, ell=[3])
+    logits, draft = case.extra["logits"], case.extra["draft"]
+    for _ in range(args.warmup):
+        oracle_layer_sample(case, logits, draft)
+    steps = min(args.steps, 50)
+    t0 = time.perf_counter()
+    done = 0
+    for _ in range(steps):
+        done += oracle_layer_sample(case, logits, draft)
+    el = time.perf_counter() - t0
+    value = done / el / 1e9
+    line = {
+        "impl": "reference",
+        "metric": METRIC,
+        "value": round(value, 4),
+        "unit": "GB/s",
+        "n_gpus": world,
+        "steps": steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(el / steps * 1e3, 3),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "f64",
+        "data": "synthetic (seeded Philox)",
+        "config": {"workload": "8B-class target verify step, one layer per step (sample): M-RoPE + append + "
+                               "attention L=4096 K=7 32q/8kv x 128 + greedy accept V=151936 + rollback",
+                   "parallelism": "host cores"},
+        "cpu_baseline": {"value": round(value, 4), "unit": "GB/s", "cores": cpu_threads(), "kind": "oracle",
+                         "sample": "one target layer + acceptance per step, %d steps" % steps},
+        "e2e": {"value": round(value, 4), "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+if __name__ == "__main__":
+    main()

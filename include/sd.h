@@ -1,0 +1,215 @@
+/*
+ * sd.h -- C ABI of libsd.so, the GB300 (sm_103a) verify step of two-reasoner
+ * speculative decoding ("Reasoning-aware Speculative Decoding for Efficient
+ * VLA Models in Autonomous Driving", arxiv 2606.31160).
+ *
+ * In the paper's propose / verify / commit loop (Sec. 2.2) a small draft
+ * proposes K tokens and the unmodified multimodal target scores them in one
+ * pass. This library is the data-parallel hot path of that pass: the rotary
+ * position encoding of the new rows (Sec. 2.3, Sec. 3.2), the KV-cache append
+ * and rollback (Eq. commit), the causally masked GQA attention of the K + 1
+ * verify rows (Eq. verify), and the two acceptance rules (Eqs. accept,
+ * commit; Leviathan/Chen rejection sampling, cited in Sec. 1-2).
+ *
+ * Conventions shared by every entry point:
+ *   - All tensor pointers are DEVICE pointers owned by the caller, row-major
+ *     with the innermost index last, 16-byte aligned. The library never
+ *     allocates device memory and never synchronises, except
+ *     sd_get_device_error(), which synchronises the stream it is given.
+ *   - Every call is asynchronous on `stream` (NULL = legacy default stream).
+ *   - Problems visible on the host (bad sizes, NULL pointers, unsupported
+ *     shapes, short workspace) return a status before anything is launched.
+ *     Problems only visible on the device (a length past the capacity, a
+ *     rollback past the appended rows, a token id outside the vocabulary)
+ *     set bits of a per-device error word, read with sd_get_device_error();
+ *     the affected scene is skipped and no kernel traps.
+ *   - bf16 is IEEE-754 binary32 truncated to its upper 16 bits (bfloat16),
+ *     stored as uint16.
+ *   - B = scenes, R = K + 1 verify rows, Hq / Hkv = query / KV heads with
+ *     G = Hq / Hkv, D = head dim, V = vocabulary size.
+ */
+#ifndef SD_H_
+#define SD_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* cudaStream_t without pulling in the CUDA headers. */
+typedef struct CUstream_st* sd_stream_t;
+
+typedef enum {
+  SD_OK = 0,
+  SD_ERR_INVALID_ARG = 1,  /* NULL pointer, non-positive size, misalignment   */
+  SD_ERR_UNSUPPORTED = 2,  /* valid but not built: D not in {64,128}, ...      */
+  SD_ERR_WORKSPACE = 3,    /* workspace NULL or smaller than the size query    */
+  SD_ERR_CUDA = 4,         /* a CUDA runtime call failed (launch, attribute)   */
+  SD_ERR_DEVICE = 5,       /* sd_get_device_error found device-side error bits */
+  SD_ERR_TIMEOUT = 6       /* a bounded device wait gave up (see error bits)   */
+} sd_status;
+
+typedef enum { SD_BF16 = 0, SD_F32 = 1 } sd_dtype;
+
+/* Device error bits (sd_get_device_error). */
+#define SD_DEVERR_KV_OVERFLOW   0x1u  /* append would pass the capacity        */
+#define SD_DEVERR_ROLLBACK      0x2u  /* committed outside [0, n_appended]     */
+#define SD_DEVERR_TOKEN_RANGE   0x4u  /* a draft token outside [0, V)          */
+#define SD_DEVERR_LENGTH        0x8u  /* len[b] < R or len[b] > capacity       */
+#define SD_DEVERR_TIMEOUT       0x10u /* a bounded mbarrier wait ran out       */
+
+/*
+ * KV cache of one attention layer. k and v are [B][Hkv][capacity][D] bf16;
+ * len is a device int32[B]: the number of valid rows of each scene. Rows at
+ * or past len[b] are never read by the attention (their contents may be
+ * anything, NaN included).
+ */
+typedef struct {
+  void* k;
+  void* v;
+  int32_t* len;
+  int32_t batch;
+  int32_t n_kv_heads;
+  int32_t capacity;
+  int32_t head_dim;
+} sd_kv_cache;
+
+/* Name of a status code; a static string, never NULL. */
+const char* sd_status_str(sd_status s);
+
+/* Library version string, e.g. "sd 0.1 sm_103a". */
+const char* sd_version(void);
+
+/*
+ * M-RoPE rotation of the new Q and K rows, in place (Sec. 2.3 Eq. rope-3d;
+ * Sec. 3.2 Eqs. axis-assign, mrope-phase).
+ *   q:   [B][R][Hq][D] bf16, k: [B][R][Hkv][D] bf16 (either may be NULL when
+ *        its head count is 0).
+ *   pos: [B][R][3] int32 (t, h, w) coordinates of each row, device memory.
+ *   sections: HOST int32[3] = (s_T, s_H, s_W), summing to D / 2.
+ *   interleaved: 0 = blocked axis assignment, 1 = a(d) = (T,H,W)[d mod 3].
+ *   base: theta_d = base^(-2d/D).
+ * Pair d is the adjacent dimensions (2d, 2d+1): x' = x cos(phi) - y sin(phi),
+ * y' = x sin(phi) + y cos(phi), phi = theta_d * pos[a(d)]. Arithmetic is fp32
+ * with an extended-precision angle; results round to bf16.
+ * D must be 64 or 128 (SD_ERR_UNSUPPORTED otherwise).
+ */
+sd_status sd_rope_apply(void* q, void* k, int B, int R, int Hq, int Hkv, int D,
+                        const int32_t* pos, const int32_t sections[3],
+                        int interleaved, float base, sd_stream_t stream);
+
+/*
+ * FlatRoPE / plain 1D RoPE (Sec. 2.3 Eq. rope-1d; Sec. 3.2 Eq. flatrope-proj):
+ * the same rotation with every axis at the sequence index pos1d[b][r]
+ * (device int32[B][R]). Equal, bit for bit, to sd_rope_apply with
+ * pos = (m, m, m) under any section layout.
+ */
+sd_status sd_rope_apply_1d(void* q, void* k, int B, int R, int Hq, int Hkv, int D,
+                           const int32_t* pos1d, float base, sd_stream_t stream);
+
+/*
+ * Append R new rows per scene (Eq. commit: the verify pass writes the keys and
+ * values of all K + 1 rows before the acceptance is known).
+ *   k_new, v_new: [B][R][Hkv][D] bf16 (rotated keys; values).
+ * Writes row i of scene b at cache position len[b] + i, then len[b] += R.
+ * A scene with len[b] + R > capacity is left untouched and sets
+ * SD_DEVERR_KV_OVERFLOW.
+ */
+sd_status sd_kv_append(const sd_kv_cache* cache, const void* k_new,
+                       const void* v_new, int R, sd_stream_t stream);
+
+/*
+ * Roll the lengths back to the committed rows (Eq. commit: t <- t + l + 1).
+ *   len:       device int32[count], count a multiple of B (one length array
+ *              per layer, all layers' arrays contiguous: [n_layers][B]).
+ *   committed: device int32[B], rows kept of the n_appended just appended
+ *              (n_emit of sd_accept_greedy / sd_accept_sample).
+ * len[l*B + b] <- len[l*B + b] - n_appended + committed[b]. A committed value
+ * outside [0, n_appended] (or a length that would drop below 0) leaves that
+ * entry untouched and sets SD_DEVERR_ROLLBACK.
+ */
+sd_status sd_kv_rollback(int32_t* len, int count, int B, const int32_t* committed,
+                         int n_appended, sd_stream_t stream);
+
+/*
+ * Verify attention (Eq. verify, Sec. 2.2): for scene b, query head h (KV head
+ * g = h / G) and row i < R,
+ *   o[b][i][h] = softmax_n( q[b][i][h] . k[b][g][n] * scale ) v[b][g][n],
+ *   n = 0 .. len[b] - R + i
+ * i.e. row i is the token at position L_b + i (L_b = len[b] - R, the prefix
+ * before the append) and sees the prefix plus the new rows up to itself.
+ *   q:   [B][R][Hq][D] bf16 (rotated), cache: keys/values already appended,
+ *   out: [B][R][Hq][D] bf16.
+ *   scale: 0 selects 1/sqrt(D).
+ * The G*R query rows that share a KV head are packed into one tile, so each
+ * K/V row is read from HBM once. Requires D in {64, 128}, Hq % Hkv == 0 and
+ * G*R <= 128. A scene with len[b] < R or len[b] > capacity sets
+ * SD_DEVERR_LENGTH and its output is left unwritten. No workspace.
+ */
+sd_status sd_verify_attention(const void* q, const sd_kv_cache* cache, void* out,
+                              int R, int Hq, float scale, sd_stream_t stream);
+
+/*
+ * Workspace bytes sd_accept_greedy needs for (B, R = K + 1, V).
+ */
+size_t sd_accept_greedy_workspace(int B, int K, int V);
+
+/*
+ * Greedy acceptance (Eqs. verify, accept, commit; Sec. 3.3 Eq. accept-length).
+ *   logits: [B][K+1][V] of `dtype` (SD_BF16 or SD_F32).
+ *   draft:  [B][K] int32 draft tokens.
+ * Outputs (device): argmax [B][K+1] int32, the lowest index among equal
+ * maxima (values compare numerically, +0 == -0; NaN is outside the
+ * contract); n_emit [B] int32 = l + 1, l = the number of leading drafts equal
+ * to argmax; tokens [B][K+1] int32 = draft[0..l-1], argmax[l], then -1.
+ * ws: caller-owned device scratch of sd_accept_greedy_workspace() bytes,
+ * zero-filled before its first use; every call leaves it zero-filled again.
+ * Calls that share a workspace must not overlap on the device.
+ * argmax may be NULL. K = 0 is plain argmax.
+ */
+sd_status sd_accept_greedy(const void* logits, sd_dtype dtype, int B, int K, int V,
+                           const int32_t* draft, int32_t* n_emit, int32_t* tokens,
+                           int32_t* argmax, void* ws, size_t ws_bytes,
+                           sd_stream_t stream);
+
+/*
+ * Workspace bytes sd_accept_sample needs for (B, K, V).
+ */
+size_t sd_accept_sample_workspace(int B, int K, int V);
+
+/*
+ * Rejection-sampling acceptance (Leviathan et al. / Chen et al., cited in
+ * Sec. 1-2) at temperature T > 0, driven by caller-supplied uniforms.
+ *   z_target: [B][K+1][V] fp32, z_draft: [B][K][V] fp32, draft: [B][K] int32,
+ *   u: [B][K+1] fp32 uniforms in [0, 1).
+ * With p_j = softmax(z_target[j] / T), q_j = softmax(z_draft[j] / T):
+ * draft j is accepted iff u[j] * q_j(x) <= p_j(x); at the first rejection j
+ * the token is drawn from (p_j - q_j)+ with u[K], and when all K are
+ * accepted the bonus is drawn from p_K with u[K]; a draw from weights w takes
+ * the smallest v with sum_{v' <= v} w(v') > u[K] * sum(w).
+ * Outputs: n_emit [B] = l + 1 and tokens [B][K+1] (draft[0..l-1], the drawn
+ * token, then -1). fp32 arithmetic with fixed-order reductions: the result is
+ * a deterministic function of the inputs.
+ * ws: as for sd_accept_greedy (zero-filled before first use, left zeroed).
+ */
+sd_status sd_accept_sample(const float* z_target, const float* z_draft, int B, int K,
+                           int V, float temperature, const int32_t* draft,
+                           const float* u, int32_t* n_emit, int32_t* tokens,
+                           void* ws, size_t ws_bytes, sd_stream_t stream);
+
+/*
+ * Synchronise `stream`, return the device error bits accumulated on the
+ * current device since the last call in *bits, and clear them.
+ * Returns SD_OK when no bit is set, SD_ERR_DEVICE when some bit is set
+ * (SD_ERR_TIMEOUT when SD_DEVERR_TIMEOUT is among them), SD_ERR_CUDA when the
+ * synchronisation itself failed.
+ */
+sd_status sd_get_device_error(sd_stream_t stream, uint32_t* bits);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SD_H_ */

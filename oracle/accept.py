@@ -80,14 +80,15 @@ def _softmax_t(z, temperature):
 
 def _inverse_cdf(w, u):
     """Smallest v with sum_{v' <= v} w(v') > u * sum(w); also the distance of
-    u * sum(w) to the nearest step of that cumulative sum, relative to sum(w)."""
+    u * sum(w) to the nearest step of that cumulative sum, in the units of w
+    (probability units: w is p - q clipped, or p)."""
     c = np.cumsum(w)
     total = c[-1]
     target = np.float64(u) * total
     v = int(np.searchsorted(c, target, side="right"))
     v = min(v, len(w) - 1)
     lo = c[v - 1] if v > 0 else 0.0
-    margin = min(abs(c[v] - target), abs(target - lo)) / total
+    margin = min(abs(c[v] - target), abs(target - lo))
     return v, float(margin)
 
 
@@ -97,9 +98,9 @@ def accept_sample(z_target, z_draft, draft, u, temperature):
     z_target: [B, K+1, V], z_draft: [B, K, V], draft: [B, K] ints,
     u: [B, K+1] uniforms in [0, 1), temperature T > 0.
     returns (n_emit [B], tokens [B, K+1] with -1 after n_emit, margins), where
-    margins[b] lists the relative distance of every decision taken to its
-    boundary: |u q - p| / max(p, u q) for each acceptance test, and the
-    inverse-CDF distance for the final draw.
+    margins[b] lists the distance of every decision taken to its boundary:
+    |u q - p| / max(p, u q) (relative) for each acceptance test, then the
+    inverse-CDF distance of the final draw in probability units.
     """
     z_target = np.asarray(z_target, dtype=np.float64)
     z_draft = np.asarray(z_draft, dtype=np.float64)

@@ -1,0 +1,236 @@
+// K4: greedy acceptance (Eqs. verify, accept, commit, Sec. 2.2; Eq.
+// accept-length, Sec. 3.3).
+//
+//   r*_j = argmax_v logits[b][j][v]   (lowest index among equal maxima)
+//   l    = number of leading drafts equal to r*   (draft[j] vs r*_j, j < K)
+//   emit draft[0..l-1], r*_l            n_emit = l + 1
+//
+// One launch. The vocabulary of every row is split into chunks; a CTA scans
+// one (scene, row, chunk) with 16-byte vector loads, reduces (value, index)
+// pairs with warp shuffles and shared memory, and writes one partial. The
+// last CTA of each scene (atomic ticket, no spin) reduces the partials of all
+// K + 1 rows, compares with the drafts and writes the outputs, then re-arms
+// its ticket. The (value desc, index asc) order is total, so the result does
+// not depend on the order partials are combined in: bit-exact and
+// deterministic.
+#include "common.cuh"
+
+SD_DEFINE_ERROR_ACCESSOR(sd_take_error_greedy)
+
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kMaxChunks = 1024;
+
+struct Best {
+  float v;
+  int i;
+};
+
+// a beats b: larger value, or equal value (numerically: +0 == -0) and lower index.
+__device__ __forceinline__ bool beats(float av, int ai, float bv, int bi) {
+  return av > bv || (av == bv && ai < bi);
+}
+
+__device__ __forceinline__ void take(Best& best, float v, int i) {
+  if (beats(v, i, best.v, best.i)) {
+    best.v = v;
+    best.i = i;
+  }
+}
+
+__device__ __forceinline__ Best warp_best(Best b) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float ov = __shfl_xor_sync(0xffffffffu, b.v, o);
+    const int oi = __shfl_xor_sync(0xffffffffu, b.i, o);
+    take(b, ov, oi);
+  }
+  return b;
+}
+
+template <typename T>
+__device__ __forceinline__ float load_one(const T* p, long long i);
+template <>
+__device__ __forceinline__ float load_one<float>(const float* p, long long i) { return p[i]; }
+template <>
+__device__ __forceinline__ float load_one<__nv_bfloat16>(const __nv_bfloat16* p, long long i) {
+  return __bfloat162float(p[i]);
+}
+
+// Scan [lo, hi) of one row. Each thread keeps the first maximum of its own
+// ascending subsequence; the cross-thread combine uses the full order.
+template <typename T>
+__device__ Best scan_chunk(const T* row, int lo, int hi, bool vec_ok) {
+  Best best{-INFINITY, 0x7fffffff};
+  constexpr int kPer = 16 / sizeof(T);  // elements per 16-byte vector
+  int start = lo;
+  if (vec_ok) {
+    const int vlo = (lo + kPer - 1) / kPer * kPer;
+    const int vhi = hi / kPer * kPer;
+    // head and tail elements outside the aligned body
+    for (int i = lo + threadIdx.x; i < min(vlo, hi); i += blockDim.x) take(best, load_one(row, i), i);
+    for (int i = max(vhi, vlo) + threadIdx.x; i < hi; i += blockDim.x) take(best, load_one(row, i), i);
+    for (int v = vlo / kPer + threadIdx.x; v < vhi / kPer; v += blockDim.x) {
+      const uint4 w = __ldg(reinterpret_cast<const uint4*>(row) + v);
+      const int base = v * kPer;
+      if (sizeof(T) == 4) {
+        take(best, __uint_as_float(w.x), base + 0);
+        take(best, __uint_as_float(w.y), base + 1);
+        take(best, __uint_as_float(w.z), base + 2);
+        take(best, __uint_as_float(w.w), base + 3);
+      } else {
+        const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          take(best, sd_bf16_lo(ws[j]), base + 2 * j);
+          take(best, sd_bf16_hi(ws[j]), base + 2 * j + 1);
+        }
+      }
+    }
+    start = hi;  // everything covered
+  }
+  for (int i = start + threadIdx.x; i < hi; i += blockDim.x) take(best, load_one(row, i), i);
+  return best;
+}
+
+__device__ Best block_best(Best b) {
+  __shared__ float sv[kThreads / 32];
+  __shared__ int si[kThreads / 32];
+  b = warp_best(b);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (lane == 0) {
+    sv[warp] = b.v;
+    si[warp] = b.i;
+  }
+  __syncthreads();
+  if (warp == 0) {
+    Best c{-INFINITY, 0x7fffffff};
+    if (lane < kThreads / 32) c = Best{sv[lane], si[lane]};
+    b = warp_best(c);
+  }
+  return b;  // valid in warp 0
+}
+
+template <typename T>
+__global__ void __launch_bounds__(kThreads) greedy_kernel(const T* __restrict__ logits, int R, int V,
+                                                          int chunk, int n_chunks,
+                                                          const int32_t* __restrict__ draft,
+                                                          int32_t* __restrict__ n_emit,
+                                                          int32_t* __restrict__ tokens,
+                                                          int32_t* __restrict__ argmax_out,
+                                                          float2* __restrict__ part,
+                                                          uint32_t* __restrict__ ticket) {
+  const int c = blockIdx.x, r = blockIdx.y, b = blockIdx.z;
+  const T* row = logits + (static_cast<long long>(b) * R + r) * V;
+  const bool vec_ok = ((static_cast<long long>(V) * sizeof(T)) % 16 == 0) &&
+                      ((reinterpret_cast<uintptr_t>(logits) & 15) == 0);
+  const int lo = c * chunk, hi = min(V, lo + chunk);
+  Best best = block_best(scan_chunk(row, lo, hi, vec_ok));
+  __shared__ bool s_last;
+  if (threadIdx.x == 0) {
+    part[(static_cast<long long>(b) * R + r) * n_chunks + c] = make_float2(best.v, __int_as_float(best.i));
+    __threadfence();
+    const uint32_t prev = atomicAdd(&ticket[b], 1u);
+    s_last = prev == static_cast<uint32_t>(R * n_chunks - 1);
+  }
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  // ---- last CTA of scene b: reduce every row's partials, then accept
+  __shared__ int s_star[32 * 4];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (int rr = warp; rr < R; rr += kThreads / 32) {
+    Best w{-INFINITY, 0x7fffffff};
+    const float2* pr = part + (static_cast<long long>(b) * R + rr) * n_chunks;
+    for (int k = lane; k < n_chunks; k += 32) {
+      const float2 e = __ldcg(pr + k);
+      take(w, e.x, __float_as_int(e.y));
+    }
+    w = warp_best(w);
+    if (lane == 0) {
+      const int star = w.i == 0x7fffffff ? 0 : w.i;
+      s_star[rr] = star;
+      if (argmax_out) argmax_out[static_cast<long long>(b) * R + rr] = star;
+    }
+  }
+  const int K = R - 1;
+  __shared__ int s_draft[128];
+  for (int j = threadIdx.x; j < K; j += kThreads) s_draft[j] = draft[static_cast<long long>(b) * K + j];
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int ell = K;
+    bool range_ok = true;
+    for (int j = 0; j < K; ++j) {
+      const int d = s_draft[j];
+      if (d < 0 || d >= V) range_ok = false;
+      if (ell == K && d != s_star[j]) ell = j;
+    }
+    if (!range_ok) sd_set_error(SD_DEVERR_TOKEN_RANGE);
+    int32_t* tk = tokens + static_cast<long long>(b) * R;
+    for (int j = 0; j < R; ++j) {
+      int v = -1;
+      if (j < ell) v = s_draft[j];
+      else if (j == ell) v = s_star[ell];
+      tk[j] = v;
+    }
+    n_emit[b] = ell + 1;
+    ticket[b] = 0;  // re-arm for the next call
+  }
+}
+
+// Chunking depends on V only (never on the device), so the workspace size
+// is the same wherever it is queried: 4096 elements per CTA, more when the
+// row would need over kMaxChunks chunks.
+void plan(int B, int R, int V, int* chunk, int* n_chunks) {
+  (void)B;
+  (void)R;
+  long long ch = 4096;
+  while ((V + ch - 1) / ch > kMaxChunks) ch *= 2;
+  *chunk = static_cast<int>(ch);
+  *n_chunks = static_cast<int>((V + ch - 1) / ch);
+}
+
+size_t ws_bytes_for(int B, int R, int n_chunks) {
+  return static_cast<size_t>(B) * R * n_chunks * sizeof(float2) + static_cast<size_t>(B) * 4 + 256;
+}
+
+}  // namespace
+
+extern "C" size_t sd_accept_greedy_workspace(int B, int K, int V) {
+  if (B <= 0 || K < 0 || V <= 0) return 0;
+  int chunk, n_chunks;
+  plan(B, K + 1, V, &chunk, &n_chunks);
+  return ws_bytes_for(B, K + 1, n_chunks);
+}
+
+extern "C" sd_status sd_accept_greedy(const void* logits, sd_dtype dtype, int B, int K, int V,
+                                      const int32_t* draft, int32_t* n_emit, int32_t* tokens,
+                                      int32_t* argmax, void* ws, size_t ws_bytes,
+                                      sd_stream_t stream) {
+  if (B < 0 || K < 0 || V <= 0) return SD_ERR_INVALID_ARG;
+  if (dtype != SD_BF16 && dtype != SD_F32) return SD_ERR_INVALID_ARG;
+  if (K + 1 > 128 || B > 65535) return SD_ERR_UNSUPPORTED;
+  if (B == 0) return SD_OK;
+  if (!logits || !n_emit || !tokens || (K > 0 && !draft)) return SD_ERR_INVALID_ARG;
+  const int R = K + 1;
+  int chunk, n_chunks;
+  plan(B, R, V, &chunk, &n_chunks);
+  const size_t need = ws_bytes_for(B, R, n_chunks);
+  if (!ws || ws_bytes < need || !sd_aligned16(ws)) return SD_ERR_WORKSPACE;
+  auto* part = static_cast<float2*>(ws);
+  auto* ticket = reinterpret_cast<uint32_t*>(static_cast<char*>(ws) +
+                                             static_cast<size_t>(B) * R * n_chunks * sizeof(float2));
+  const dim3 grid(n_chunks, R, B);
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  if (dtype == SD_BF16)
+    greedy_kernel<__nv_bfloat16><<<grid, kThreads, 0, st>>>(
+        static_cast<const __nv_bfloat16*>(logits), R, V, chunk, n_chunks, draft, n_emit, tokens,
+        argmax, part, ticket);
+  else
+    greedy_kernel<float><<<grid, kThreads, 0, st>>>(static_cast<const float*>(logits), R, V, chunk,
+                                                    n_chunks, draft, n_emit, tokens, argmax, part,
+                                                    ticket);
+  SD_CHECK_LAUNCH();
+  return SD_OK;
+}

@@ -1,0 +1,435 @@
+// K5: rejection-sampling acceptance (Leviathan et al. / Chen et al., cited
+// in Sec. 1-2 of the paper, which evaluates the greedy rule only).
+//
+//   p_j = softmax(z_T[j] / T), q_j = softmax(z_D[j] / T)
+//   draft j (token x) accepted iff u_j * q_j(x) <= p_j(x)
+//   first rejection at j: draw from (p_j - q_j)+ with u_K
+//   all K accepted:       draw the bonus from p_K with u_K
+//   draw from w with u:   smallest v with sum_{v' <= v} w(v') > u * sum(w)
+//
+// Two launches:
+//   stats:  grid (chunk, row, scene) over the 2K + 1 rows; each CTA writes
+//           (max, sum exp2((z - max) * log2e / T)) of one chunk. The last CTA
+//           of a scene (atomic ticket, no spin) merges the chunks of every
+//           row in a fixed order, runs the K acceptance tests and records l
+//           and the normalisers of the row to draw from.
+//   draw:   grid (chunk, scene) over that one row; each CTA writes the
+//           chunk sums of the residual weights and of the target weights; the
+//           last CTA of a scene finds the chunk where the running sum passes
+//           u_K * S and scans inside it.
+// All reductions run in a fixed order (deterministic), the weight formula
+// uses non-contractible intrinsics so both passes of the draw evaluate
+// identical values, and every spin-free ticket is re-armed after use.
+#include "common.cuh"
+
+SD_DEFINE_ERROR_ACCESSOR(sd_take_error_sample)
+
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kMaxChunks = 1024;
+constexpr float kLog2e = 1.4426950408889634f;
+
+struct DrawInfo {
+  int ell;
+  float mt, inv_zt;  // target row l (or K): max and 1 / sum
+  float md, inv_zd;  // draft row l (when l < K)
+  float pad[3];
+};
+
+// exp2((z - m) * c2) with a fixed rounding sequence
+__device__ __forceinline__ float wexp(float z, float m, float c2) {
+  return exp2f(__fmul_rn(__fsub_rn(z, m), c2));
+}
+
+// (max, sum) pair merge: sum rescaled to the larger max
+__device__ __forceinline__ void merge_ms(float& m, float& s, float m2, float s2, float c2) {
+  if (m2 == -INFINITY) return;
+  if (m == -INFINITY) {
+    m = m2;
+    s = s2;
+    return;
+  }
+  if (m2 > m) {
+    s = __fadd_rn(__fmul_rn(s, wexp(m, m2, c2)), s2);
+    m = m2;
+  } else {
+    s = __fadd_rn(s, __fmul_rn(s2, wexp(m2, m, c2)));
+  }
+}
+
+__device__ __forceinline__ const float* row_ptr(const float* zt, const float* zd, int b, int rr,
+                                                int K, int V) {
+  if (rr <= K) return zt + (static_cast<long long>(b) * (K + 1) + rr) * V;
+  return zd + (static_cast<long long>(b) * K + (rr - K - 1)) * V;
+}
+
+// ------------------------------------------------------------------ stats
+__global__ void __launch_bounds__(kThreads)
+    sample_stats_kernel(const float* __restrict__ zt, const float* __restrict__ zd, int K, int V,
+                        float c2, int chunk, int n_chunks, const int32_t* __restrict__ draft,
+                        const float* __restrict__ u, int32_t* __restrict__ n_emit,
+                        int32_t* __restrict__ tokens, float2* __restrict__ part,
+                        uint32_t* __restrict__ ticket, DrawInfo* __restrict__ info) {
+  const int c = blockIdx.x, rr = blockIdx.y, b = blockIdx.z;
+  const int rows = 2 * K + 1;
+  const float* row = row_ptr(zt, zd, b, rr, K, V);
+  const int lo = c * chunk, hi = min(V, lo + chunk);
+  // thread max, then thread sum, over a fixed strided subset of the chunk
+  float m = -INFINITY;
+  for (int i = lo + threadIdx.x; i < hi; i += kThreads) m = fmaxf(m, __ldg(row + i));
+  float s = 0.f;
+  if (m != -INFINITY)
+    for (int i = lo + threadIdx.x; i < hi; i += kThreads) s = __fadd_rn(s, wexp(__ldg(row + i), m, c2));
+  // warp then block merge, fixed tree
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float m2 = __shfl_xor_sync(0xffffffffu, m, o);
+    const float s2 = __shfl_xor_sync(0xffffffffu, s, o);
+    merge_ms(m, s, m2, s2, c2);
+  }
+  __shared__ float sm[kThreads / 32], ss[kThreads / 32];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (lane == 0) {
+    sm[warp] = m;
+    ss[warp] = s;
+  }
+  __syncthreads();
+  __shared__ bool s_last;
+  if (threadIdx.x == 0) {
+    float bm = sm[0], bs = ss[0];
+    for (int w = 1; w < kThreads / 32; ++w) merge_ms(bm, bs, sm[w], ss[w], c2);
+    part[(static_cast<long long>(b) * rows + rr) * n_chunks + c] = make_float2(bm, bs);
+    __threadfence();
+    s_last = atomicAdd(&ticket[b], 1u) == static_cast<uint32_t>(rows * n_chunks - 1);
+  }
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  // ---- last CTA of scene b: merge chunks per row, then the acceptance tests
+  __shared__ float row_m[2 * 128 + 1], row_s[2 * 128 + 1];
+  for (int r = warp; r < rows; r += kThreads / 32) {
+    float rm = -INFINITY, rs = 0.f;
+    const float2* pr = part + (static_cast<long long>(b) * rows + r) * n_chunks;
+    for (int k = lane; k < n_chunks; k += 32) {
+      const float2 e = __ldcg(pr + k);
+      merge_ms(rm, rs, e.x, e.y, c2);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const float m2 = __shfl_xor_sync(0xffffffffu, rm, o);
+      const float s2 = __shfl_xor_sync(0xffffffffu, rs, o);
+      merge_ms(rm, rs, m2, s2, c2);
+    }
+    if (lane == 0) {
+      row_m[r] = rm;
+      row_s[r] = rs;
+    }
+  }
+  __syncthreads();
+  // the K draft tokens and their two logits, fetched in parallel
+  __shared__ int s_x[128];
+  __shared__ float s_zt[128], s_zd[128];
+  for (int j = threadIdx.x; j < K; j += kThreads) {
+    const int x = draft[static_cast<long long>(b) * K + j];
+    s_x[j] = x;
+    const bool ok = x >= 0 && x < V;
+    s_zt[j] = ok ? row_ptr(zt, zd, b, j, K, V)[x] : 0.f;
+    s_zd[j] = ok ? row_ptr(zt, zd, b, K + 1 + j, K, V)[x] : 0.f;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int ell = K;
+    bool range_ok = true;
+    for (int j = 0; j < K; ++j) {
+      const int x = s_x[j];
+      if (x < 0 || x >= V) {
+        range_ok = false;
+        ell = j;
+        break;
+      }
+      const float p = __fdiv_rn(wexp(s_zt[j], row_m[j], c2), row_s[j]);
+      const float q = __fdiv_rn(wexp(s_zd[j], row_m[K + 1 + j], c2), row_s[K + 1 + j]);
+      if (!(__fmul_rn(u[static_cast<long long>(b) * (K + 1) + j], q) <= p)) {
+        ell = j;
+        break;
+      }
+    }
+    if (!range_ok) sd_set_error(SD_DEVERR_TOKEN_RANGE);
+    DrawInfo di;
+    di.ell = ell;
+    di.mt = row_m[ell];
+    di.inv_zt = __fdiv_rn(1.f, row_s[ell]);
+    di.md = ell < K ? row_m[K + 1 + ell] : 0.f;
+    di.inv_zd = ell < K ? __fdiv_rn(1.f, row_s[K + 1 + ell]) : 0.f;
+    di.pad[0] = di.pad[1] = di.pad[2] = 0.f;
+    info[b] = di;
+    int32_t* tk = tokens + static_cast<long long>(b) * (K + 1);
+    for (int j = 0; j <= K; ++j) tk[j] = j < ell ? s_x[j] : -1;
+    n_emit[b] = ell + 1;
+    ticket[b] = 0;
+  }
+}
+
+// ------------------------------------------------------------------ draw
+// Weights of element v of the draw row: residual (p - q)+ (l < K) and the
+// unnormalised target weight exp2((z_T - m_T) * c2).
+__device__ __forceinline__ void weights(const float* rt, const float* rd, const DrawInfo& di, int K,
+                                        float c2, int v, float& w_res, float& w_tgt) {
+  const float et = wexp(rt[v], di.mt, c2);
+  w_tgt = et;
+  if (di.ell < K) {
+    const float p = __fmul_rn(et, di.inv_zt);
+    const float q = __fmul_rn(wexp(rd[v], di.md, c2), di.inv_zd);
+    w_res = fmaxf(__fsub_rn(p, q), 0.f);
+  } else {
+    w_res = 0.f;
+  }
+}
+
+__device__ float block_sum(float x, float* red) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) x = __fadd_rn(x, __shfl_xor_sync(0xffffffffu, x, o));
+  __syncthreads();
+  if (lane == 0) red[warp] = x;
+  __syncthreads();
+  float t = 0.f;
+  if (threadIdx.x == 0)
+    for (int w = 0; w < kThreads / 32; ++w) t = __fadd_rn(t, red[w]);
+  return t;  // valid in thread 0
+}
+
+__global__ void __launch_bounds__(kThreads)
+    sample_draw_kernel(const float* __restrict__ zt, const float* __restrict__ zd, int K, int V,
+                       float c2, int chunk, int n_chunks, const float* __restrict__ u,
+                       int32_t* __restrict__ tokens, const DrawInfo* __restrict__ info,
+                       float2* __restrict__ sums, uint32_t* __restrict__ ticket) {
+  const int c = blockIdx.x, b = blockIdx.y;
+  const DrawInfo di = info[b];
+  const float* rt = zt + (static_cast<long long>(b) * (K + 1) + di.ell) * V;
+  const float* rd = di.ell < K ? zd + (static_cast<long long>(b) * K + di.ell) * V : nullptr;
+  const int lo = c * chunk, hi = min(V, lo + chunk);
+  float sr = 0.f, sp = 0.f;
+  for (int v = lo + threadIdx.x; v < hi; v += kThreads) {
+    float wr, wt;
+    weights(rt, rd, di, K, c2, v, wr, wt);
+    sr = __fadd_rn(sr, wr);
+    sp = __fadd_rn(sp, wt);
+  }
+  __shared__ float red[kThreads / 32];
+  const float tr = block_sum(sr, red);
+  const float tp = block_sum(sp, red);
+  __shared__ bool s_last;
+  if (threadIdx.x == 0) {
+    sums[static_cast<long long>(b) * n_chunks + c] = make_float2(tr, tp);
+    __threadfence();
+    s_last = atomicAdd(&ticket[b], 1u) == static_cast<uint32_t>(n_chunks - 1);
+  }
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  // ---- last CTA of scene b: choose the weights, locate the chunk, scan it
+  __shared__ float s_sr[kMaxChunks], s_sp[kMaxChunks];
+  for (int k = threadIdx.x; k < n_chunks; k += kThreads) {
+    const float2 e = __ldcg(sums + static_cast<long long>(b) * n_chunks + k);
+    s_sr[k] = e.x;
+    s_sp[k] = e.y;
+  }
+  __syncthreads();
+  __shared__ int s_chunk, s_use_res;
+  __shared__ float s_base, s_target;
+  if (threadIdx.x < 32) {
+    const int lane = threadIdx.x;
+    // lane l owns chunks [l*per, (l+1)*per): sequential lane sums, warp scan
+    const int per = (n_chunks + 31) / 32;
+    const int k0 = min(n_chunks, lane * per), k1 = min(n_chunks, k0 + per);
+    float lr = 0.f, lp = 0.f;
+    for (int k = k0; k < k1; ++k) {
+      lr = __fadd_rn(lr, s_sr[k]);
+      lp = __fadd_rn(lp, s_sp[k]);
+    }
+    float ir = lr, ip = lp;  // inclusive warp scan
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const float xr = __shfl_up_sync(0xffffffffu, ir, o);
+      const float xp = __shfl_up_sync(0xffffffffu, ip, o);
+      if (lane >= o) {
+        ir = __fadd_rn(xr, ir);
+        ip = __fadd_rn(xp, ip);
+      }
+    }
+    const float tot_r = __shfl_sync(0xffffffffu, ir, 31);
+    const float tot_p = __shfl_sync(0xffffffffu, ip, 31);
+    const int use_res = (di.ell < K && tot_r > 0.f) ? 1 : 0;
+    const float total = use_res ? tot_r : tot_p;
+    const float target = __fmul_rn(u[static_cast<long long>(b) * (K + 1) + K], total);
+    const float incl = use_res ? ir : ip;
+    float run = __shfl_up_sync(0xffffffffu, incl, 1);
+    if (lane == 0) run = 0.f;
+    int found = -1, last_nz = -1;
+    float base = 0.f;
+    for (int k = k0; k < k1; ++k) {
+      const float w = use_res ? s_sr[k] : s_sp[k];
+      if (w > 0.f) last_nz = k;
+      const float nxt = __fadd_rn(run, w);
+      if (found < 0 && nxt > target) {
+        found = k;
+        base = run;
+      }
+      run = nxt;
+    }
+    const unsigned hit = __ballot_sync(0xffffffffu, found >= 0);
+    int lnz = last_nz;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) lnz = max(lnz, __shfl_xor_sync(0xffffffffu, lnz, o));
+    if (hit) {
+      const int src = __ffs(hit) - 1;
+      found = __shfl_sync(0xffffffffu, found, src);
+      base = __shfl_sync(0xffffffffu, base, src);
+    } else {
+      // u * S at or above the rounded total: the draw is the last positive
+      // weight, found by the in-chunk fallback below
+      found = lnz >= 0 ? lnz : 0;
+      base = -INFINITY;
+    }
+    if (lane == 0) {
+      s_chunk = found;
+      s_base = base;
+      s_target = target;
+      s_use_res = use_res;
+    }
+  }
+  __syncthreads();
+  // in-chunk scan: each thread owns a run of consecutive elements
+  const int clo = s_chunk * chunk, chi = min(V, clo + chunk);
+  const int per = (chunk + kThreads - 1) / kThreads;
+  const int my_lo = min(chi, clo + threadIdx.x * per), my_hi = min(chi, my_lo + per);
+  const bool use_res = s_use_res != 0;
+  float tsum = 0.f;
+  for (int v = my_lo; v < my_hi; ++v) {
+    float wr, wt;
+    weights(rt, rd, di, K, c2, v, wr, wt);
+    tsum = __fadd_rn(tsum, use_res ? wr : wt);
+  }
+  // exclusive prefix of the thread sums: warp scan + warp offsets (fixed)
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  float incl = tsum;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const float x = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl = __fadd_rn(x, incl);
+  }
+  float excl = __shfl_up_sync(0xffffffffu, incl, 1);
+  if (lane == 0) excl = 0.f;
+  __shared__ float s_wtot[kThreads / 32];
+  if (lane == 31) s_wtot[warp] = incl;
+  __syncthreads();
+  float woff = 0.f;
+  for (int w = 0; w < warp; ++w) woff = __fadd_rn(woff, s_wtot[w]);
+  float run = __fadd_rn(s_base, __fadd_rn(woff, excl));
+  int cand = 0x7fffffff, last_pos = -1;
+  for (int v = my_lo; v < my_hi; ++v) {
+    float wr, wt;
+    weights(rt, rd, di, K, c2, v, wr, wt);
+    const float w = use_res ? wr : wt;
+    if (w > 0.f) last_pos = v;
+    run = __fadd_rn(run, w);
+    if (cand == 0x7fffffff && run > s_target) cand = v;
+  }
+  // block min of candidates, block max of the last positive weight
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    cand = min(cand, __shfl_xor_sync(0xffffffffu, cand, o));
+    last_pos = max(last_pos, __shfl_xor_sync(0xffffffffu, last_pos, o));
+  }
+  __shared__ int s_cand[kThreads / 32], s_lastp[kThreads / 32];
+  if (lane == 0) {
+    s_cand[warp] = cand;
+    s_lastp[warp] = last_pos;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int best = 0x7fffffff, lp = -1;
+    for (int w = 0; w < kThreads / 32; ++w) {
+      best = min(best, s_cand[w]);
+      lp = max(lp, s_lastp[w]);
+    }
+    const int tok = best != 0x7fffffff ? best : (lp >= 0 ? lp : clo);
+    tokens[static_cast<long long>(b) * (K + 1) + di.ell] = tok;
+    ticket[b] = 0;
+  }
+}
+
+struct Plan {
+  int chunk1, n1, chunk2, n2;
+};
+
+Plan plan(int V) {
+  Plan p;
+  p.chunk1 = 4096;
+  while ((V + p.chunk1 - 1) / p.chunk1 > kMaxChunks) p.chunk1 *= 2;
+  p.n1 = (V + p.chunk1 - 1) / p.chunk1;
+  p.chunk2 = 2048;
+  while ((V + p.chunk2 - 1) / p.chunk2 > kMaxChunks) p.chunk2 *= 2;
+  p.n2 = (V + p.chunk2 - 1) / p.chunk2;
+  return p;
+}
+
+struct Layout {
+  size_t part, ticket1, info, sums, ticket2, total;
+};
+
+Layout layout(int B, int K, const Plan& p) {
+  Layout l;
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    const size_t at = off;
+    off += (bytes + 255) / 256 * 256;
+    return at;
+  };
+  l.part = take(static_cast<size_t>(B) * (2 * K + 1) * p.n1 * sizeof(float2));
+  l.ticket1 = take(static_cast<size_t>(B) * 4);
+  l.info = take(static_cast<size_t>(B) * sizeof(DrawInfo));
+  l.sums = take(static_cast<size_t>(B) * p.n2 * sizeof(float2));
+  l.ticket2 = take(static_cast<size_t>(B) * 4);
+  l.total = off;
+  return l;
+}
+
+}  // namespace
+
+extern "C" size_t sd_accept_sample_workspace(int B, int K, int V) {
+  if (B <= 0 || K < 0 || V <= 0) return 0;
+  return layout(B, K, plan(V)).total;
+}
+
+extern "C" sd_status sd_accept_sample(const float* z_target, const float* z_draft, int B, int K,
+                                      int V, float temperature, const int32_t* draft,
+                                      const float* u, int32_t* n_emit, int32_t* tokens, void* ws,
+                                      size_t ws_bytes, sd_stream_t stream) {
+  if (B < 0 || K < 0 || V <= 0) return SD_ERR_INVALID_ARG;
+  if (!(temperature > 0.f) || !isfinite(temperature)) return SD_ERR_INVALID_ARG;
+  if (K > 128 || B > 65535) return SD_ERR_UNSUPPORTED;
+  if (B == 0) return SD_OK;
+  if (!z_target || !u || !n_emit || !tokens || (K > 0 && (!z_draft || !draft)))
+    return SD_ERR_INVALID_ARG;
+  const Plan p = plan(V);
+  const Layout l = layout(B, K, p);
+  if (!ws || ws_bytes < l.total || !sd_aligned16(ws)) return SD_ERR_WORKSPACE;
+  char* w = static_cast<char*>(ws);
+  auto* part = reinterpret_cast<float2*>(w + l.part);
+  auto* ticket1 = reinterpret_cast<uint32_t*>(w + l.ticket1);
+  auto* info = reinterpret_cast<DrawInfo*>(w + l.info);
+  auto* sums = reinterpret_cast<float2*>(w + l.sums);
+  auto* ticket2 = reinterpret_cast<uint32_t*>(w + l.ticket2);
+  const float c2 = static_cast<float>(kLog2e / static_cast<double>(temperature));
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  sample_stats_kernel<<<dim3(p.n1, 2 * K + 1, B), kThreads, 0, st>>>(
+      z_target, z_draft, K, V, c2, p.chunk1, p.n1, draft, u, n_emit, tokens, part, ticket1, info);
+  SD_CHECK_LAUNCH();
+  sample_draw_kernel<<<dim3(p.n2, B), kThreads, 0, st>>>(z_target, z_draft, K, V, c2, p.chunk2,
+                                                          p.n2, u, tokens, info, sums, ticket2);
+  SD_CHECK_LAUNCH();
+  return SD_OK;
+}

@@ -1,0 +1,163 @@
+// K1: rotary position encoding of the new verify rows (sm_103a).
+//
+// Sec. 2.3 Eq. rope-1d: each adjacent pair (2d, 2d+1) of a head vector
+// rotates by phi_d; Sec. 2.3 Eq. rope-3d with Sec. 3.2 Eqs. axis-assign and
+// mrope-phase: phi_d = theta_d * p_{a(d)}, theta_d = base^(-2d/D), a(d)
+// blocked over (s_T, s_H, s_W) or (T,H,W)[d mod 3]; Sec. 3.2 Eq.
+// flatrope-proj: FlatRoPE puts every axis at the sequence index.
+//
+// Layout: one thread rotates 4 pairs (8 bf16 = one 16-byte load/store) of
+// one head row; the whole launch is a few thousand threads and is bound by
+// launch latency, not bandwidth.
+//
+// Angle precision. theta_d * p reaches ~1.6e4 rad at the positions of the
+// longest workloads, where an fp32 product alone is off by ~1e-3 rad. The
+// angle is instead carried in TURNS: the host gives tau_d = theta_d / (2 pi)
+// as an fp32 hi/lo pair; the device forms p * tau_d with an exact fma split,
+// drops the whole turns (an exact subtraction) and evaluates
+// sincospif(2 * frac), so the reduced angle is accurate to ~1e-7 rad for any
+// |p| < 2^24.
+#include "common.cuh"
+
+#include <math.h>
+
+SD_DEFINE_ERROR_ACCESSOR(sd_take_error_rope)
+
+namespace {
+
+constexpr int kMaxPairs = 64;  // D <= 128
+
+struct RopeTable {
+  float tau_hi[kMaxPairs];   // fp32 part of theta_d / (2 pi)
+  float tau_lo[kMaxPairs];   // remainder theta_d / (2 pi) - tau_hi
+  int8_t axis[kMaxPairs];    // a(d) in {0 = T, 1 = H, 2 = W}
+};
+
+// Fractional turns of p * tau, in [-0.5, 0.5] up to rounding.
+__device__ __forceinline__ float frac_turns(float p, float hi, float lo) {
+  float a = p * hi;                 // rounded product
+  float e = fmaf(p, hi, -a);        // its exact rounding error
+  float f = a - rintf(a);           // exact: whole turns removed
+  return f + fmaf(p, lo, e);
+}
+
+// One thread: 8 consecutive elements (4 pairs) of one head row.
+template <int D, bool kFlat>
+__global__ void __launch_bounds__(256) rope_kernel(__nv_bfloat16* __restrict__ q,
+                                                   __nv_bfloat16* __restrict__ k,
+                                                   int rows, int hq, int hkv,
+                                                   const int32_t* __restrict__ pos,
+                                                   RopeTable tab) {
+  constexpr int kVecPerHead = D / 8;
+  const int heads = hq + hkv;
+  const long long total = (long long)rows * heads * kVecPerHead;
+  for (long long idx = blockIdx.x * (long long)blockDim.x + threadIdx.x; idx < total;
+       idx += (long long)gridDim.x * blockDim.x) {
+    const int vec = (int)(idx % kVecPerHead);
+    const long long t = idx / kVecPerHead;
+    const int head = (int)(t % heads);
+    const long long row = t / heads;  // flattened (b, r)
+    __nv_bfloat16* base = head < hq ? q + ((row * hq + head) * D)
+                                    : k + ((row * hkv + (head - hq)) * D);
+    uint4* ptr = reinterpret_cast<uint4*>(base) + vec;
+    uint4 w = *ptr;
+    uint32_t words[4] = {w.x, w.y, w.z, w.w};
+    int p3[3];
+    if (kFlat) {
+      p3[0] = p3[1] = p3[2] = pos[row];
+    } else {
+      p3[0] = pos[row * 3 + 0];
+      p3[1] = pos[row * 3 + 1];
+      p3[2] = pos[row * 3 + 2];
+    }
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int d = vec * 4 + j;
+      const float p = (float)p3[tab.axis[d]];
+      float s, c;
+      sincospif(2.0f * frac_turns(p, tab.tau_hi[d], tab.tau_lo[d]), &s, &c);
+      const float x = sd_bf16_lo(words[j]);
+      const float y = sd_bf16_hi(words[j]);
+      const float xr = fmaf(x, c, -y * s);
+      const float yr = fmaf(x, s, y * c);
+      words[j] = sd_pack_bf16x2(xr, yr);
+    }
+    *ptr = make_uint4(words[0], words[1], words[2], words[3]);
+  }
+}
+
+bool build_table(int D, const int32_t* sections, int interleaved, float base, RopeTable* tab) {
+  const int pairs = D / 2;
+  if (sections) {
+    if (sections[0] < 0 || sections[1] < 0 || sections[2] < 0) return false;
+    if (sections[0] + sections[1] + sections[2] != pairs) return false;
+  }
+  const double two_pi = 6.283185307179586476925286766559;
+  for (int d = 0; d < pairs; ++d) {
+    const double theta = pow((double)base, -2.0 * d / (double)D);
+    const double tau = theta / two_pi;
+    tab->tau_hi[d] = (float)tau;
+    tab->tau_lo[d] = (float)(tau - (double)tab->tau_hi[d]);
+    int a = 0;
+    if (sections) {
+      if (interleaved) a = d % 3;
+      else if (d < sections[0]) a = 0;
+      else if (d < sections[0] + sections[1]) a = 1;
+      else a = 2;
+    }
+    tab->axis[d] = (int8_t)a;
+  }
+  for (int d = pairs; d < kMaxPairs; ++d) {
+    tab->tau_hi[d] = tab->tau_lo[d] = 0.f;
+    tab->axis[d] = 0;
+  }
+  return true;
+}
+
+sd_status launch(void* q, void* k, int B, int R, int Hq, int Hkv, int D, const int32_t* pos,
+                 const int32_t* sections, int interleaved, float base, bool flat,
+                 cudaStream_t stream) {
+  if (B < 0 || R < 0 || Hq < 0 || Hkv < 0) return SD_ERR_INVALID_ARG;
+  if (D != 64 && D != 128) return SD_ERR_UNSUPPORTED;
+  if (!(base > 1.0f) || !isfinite(base)) return SD_ERR_INVALID_ARG;
+  if ((Hq > 0 && (!q || !sd_aligned16(q))) || (Hkv > 0 && (!k || !sd_aligned16(k))))
+    return SD_ERR_INVALID_ARG;
+  const long long rows = (long long)B * R;
+  if (rows == 0 || Hq + Hkv == 0) return SD_OK;
+  if (!pos) return SD_ERR_INVALID_ARG;
+  if (!flat && !sections) return SD_ERR_INVALID_ARG;
+  RopeTable tab;
+  if (!build_table(D, flat ? nullptr : sections, interleaved, base, &tab)) return SD_ERR_INVALID_ARG;
+  const long long total = rows * (Hq + Hkv) * (D / 8);
+  const int threads = 256;
+  long long blocks = (total + threads - 1) / threads;
+  const long long cap = (long long)sd_num_sms() * 8;
+  if (blocks > cap) blocks = cap;
+  auto* qp = static_cast<__nv_bfloat16*>(q);
+  auto* kp = static_cast<__nv_bfloat16*>(k);
+  if (D == 64) {
+    if (flat) rope_kernel<64, true><<<(int)blocks, threads, 0, stream>>>(qp, kp, (int)rows, Hq, Hkv, pos, tab);
+    else rope_kernel<64, false><<<(int)blocks, threads, 0, stream>>>(qp, kp, (int)rows, Hq, Hkv, pos, tab);
+  } else {
+    if (flat) rope_kernel<128, true><<<(int)blocks, threads, 0, stream>>>(qp, kp, (int)rows, Hq, Hkv, pos, tab);
+    else rope_kernel<128, false><<<(int)blocks, threads, 0, stream>>>(qp, kp, (int)rows, Hq, Hkv, pos, tab);
+  }
+  SD_CHECK_LAUNCH();
+  return SD_OK;
+}
+
+}  // namespace
+
+extern "C" sd_status sd_rope_apply(void* q, void* k, int B, int R, int Hq, int Hkv, int D,
+                                   const int32_t* pos, const int32_t sections[3],
+                                   int interleaved, float base, sd_stream_t stream) {
+  if (interleaved != 0 && interleaved != 1) return SD_ERR_INVALID_ARG;
+  return launch(q, k, B, R, Hq, Hkv, D, pos, sections, interleaved, base, false,
+                reinterpret_cast<cudaStream_t>(stream));
+}
+
+extern "C" sd_status sd_rope_apply_1d(void* q, void* k, int B, int R, int Hq, int Hkv, int D,
+                                      const int32_t* pos1d, float base, sd_stream_t stream) {
+  return launch(q, k, B, R, Hq, Hkv, D, pos1d, nullptr, 0, base, true,
+                reinterpret_cast<cudaStream_t>(stream));
+}

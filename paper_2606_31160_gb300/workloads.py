@@ -111,7 +111,7 @@ def verify_case(workload, *, B, Hq, Hkv, D, prefix, K, sections, base,
     q = to_bf16(rng.standard_normal((B, R, Hq, D), dtype=np.float32))
     k_new = to_bf16(rng.standard_normal((B, R, Hkv, D), dtype=np.float32))
     v_new = to_bf16(rng.standard_normal((B, R, Hkv, D), dtype=np.float32))
-    pos = torch.from_numpy(np.ascontiguousarray(query_pos, dtype=np.int32))
+    pos = torch.from_numpy(np.array(query_pos, dtype=np.int32, copy=True))
     return VerifyCase(B, R, Hq, Hkv, D, cap, prefix, tuple(sections), interleaved,
                       float(base), k_cache, v_cache, q, k_new, v_new, pos)
 

@@ -1,0 +1,89 @@
+"""C ABI checks that need no GPU: libsd.so builds for sm_103a, loads, exports
+every function include/sd.h declares, and rejects bad host arguments before
+launching anything."""
+import ctypes
+import subprocess
+
+import pytest
+
+from paper_2606_31160_gb300 import build, sd
+
+
+@pytest.fixture(scope="module")
+def lib():
+    build.build()
+    return sd.lib()
+
+
+def test_every_header_symbol_is_exported(lib):
+    names = sd.header_symbols()
+    assert len(names) >= 12
+    for name in names:
+        assert hasattr(lib, name), name
+    out = subprocess.run(["nm", "-D", "--defined-only", sd.LIB_PATH], capture_output=True, text=True).stdout
+    exported = {line.split()[-1] for line in out.splitlines() if " T " in line}
+    assert set(names) <= exported
+    # nothing else leaks out under the sd_ prefix
+    assert {n for n in exported if n.startswith("sd_")} == set(names)
+
+
+def test_built_for_sm103a_only():
+    out = subprocess.run(["cuobjdump", "--list-elf", sd.LIB_PATH], capture_output=True, text=True)
+    if out.returncode != 0:
+        pytest.skip("cuobjdump unavailable")
+    assert "sm_103a" in out.stdout
+
+
+def test_status_strings(lib):
+    assert sd.status_str(0) == "SD_OK"
+    assert sd.status_str(1) == "SD_ERR_INVALID_ARG"
+    assert sd.status_str(3) == "SD_ERR_WORKSPACE"
+    assert sd.status_str(6) == "SD_ERR_TIMEOUT"
+    assert sd.status_str(99) == "SD_ERR_UNKNOWN"
+    assert "sm_103a" in sd.version()
+
+
+def test_workspace_queries_are_host_arithmetic(lib):
+    g = sd.greedy_workspace_bytes(1, 7, 151936)
+    assert g >= 8 * 38 * 8
+    assert sd.greedy_workspace_bytes(32, 16, 151936) > g
+    assert sd.greedy_workspace_bytes(0, 7, 10) == 0
+    s = sd.sample_workspace_bytes(8, 7, 151936)
+    assert s >= 8 * 15 * 38 * 8
+    assert sd.sample_workspace_bytes(8, 7, 0) == 0
+
+
+def test_bad_arguments_return_status_before_launch(lib):
+    null = ctypes.c_void_p(0)
+    # NULL cache / unsupported head dim / bad GQA ratio
+    assert lib.sd_verify_attention(null, None, null, 8, 32, 0.0, null) == 1
+    cache = sd.KVCacheStruct(16, 16, 16, 1, 8, 64, 96)
+    assert lib.sd_verify_attention(ctypes.c_void_p(16), ctypes.byref(cache), ctypes.c_void_p(16), 8, 32, 0.0, null) == 2
+    cache = sd.KVCacheStruct(16, 16, 16, 1, 3, 64, 128)
+    assert lib.sd_verify_attention(ctypes.c_void_p(16), ctypes.byref(cache), ctypes.c_void_p(16), 8, 32, 0.0, null) == 1
+    # G * R beyond the packed-tile limit
+    cache = sd.KVCacheStruct(16, 16, 16, 1, 1, 64, 128)
+    assert lib.sd_verify_attention(ctypes.c_void_p(16), ctypes.byref(cache), ctypes.c_void_p(16), 17, 8, 0.0, null) == 2
+    # misaligned pointer
+    cache = sd.KVCacheStruct(18, 16, 16, 1, 8, 64, 128)
+    assert lib.sd_verify_attention(ctypes.c_void_p(16), ctypes.byref(cache), ctypes.c_void_p(16), 8, 32, 0.0, null) == 1
+    # rope: unsupported head dim, bad sections
+    sec = (ctypes.c_int32 * 3)(16, 24, 24)
+    assert lib.sd_rope_apply(ctypes.c_void_p(16), ctypes.c_void_p(16), 1, 8, 32, 8, 96, ctypes.c_void_p(16), sec, 0, 1e6, null) == 2
+    bad = (ctypes.c_int32 * 3)(16, 24, 23)
+    assert lib.sd_rope_apply(ctypes.c_void_p(16), ctypes.c_void_p(16), 1, 8, 32, 8, 128, ctypes.c_void_p(16), bad, 0, 1e6, null) == 1
+    assert lib.sd_rope_apply(ctypes.c_void_p(16), ctypes.c_void_p(16), 1, 8, 32, 8, 128, ctypes.c_void_p(16), sec, 2, 1e6, null) == 1
+    # kv: NULL cache, rollback with count not a multiple of B
+    assert lib.sd_kv_append(None, null, null, 8, null) == 1
+    assert lib.sd_kv_rollback(ctypes.c_void_p(16), 5, 2, ctypes.c_void_p(16), 8, null) == 1
+    # acceptance: short workspace, bad dtype, bad temperature
+    assert lib.sd_accept_greedy(ctypes.c_void_p(16), 0, 1, 7, 151936, ctypes.c_void_p(16), ctypes.c_void_p(16),
+                                ctypes.c_void_p(16), null, ctypes.c_void_p(16), 8, null) == 3
+    assert lib.sd_accept_greedy(ctypes.c_void_p(16), 7, 1, 7, 100, ctypes.c_void_p(16), ctypes.c_void_p(16),
+                                ctypes.c_void_p(16), null, ctypes.c_void_p(16), 1 << 20, null) == 1
+    assert lib.sd_accept_sample(ctypes.c_void_p(16), ctypes.c_void_p(16), 1, 7, 100, 0.0, ctypes.c_void_p(16),
+                                ctypes.c_void_p(16), ctypes.c_void_p(16), ctypes.c_void_p(16),
+                                ctypes.c_void_p(16), 1 << 20, null) == 1
+    # empty batches are a no-op success
+    cache = sd.KVCacheStruct(0, 0, 0, 0, 8, 64, 128)
+    assert lib.sd_verify_attention(null, ctypes.byref(cache), null, 8, 32, 0.0, null) == 0

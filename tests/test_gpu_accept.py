@@ -1,0 +1,161 @@
+"""GPU parity of sd_accept_greedy and sd_accept_sample against the float64 oracle.
+
+Greedy: n_emit, tokens and argmax bit-exact. Sampling: bit-exact on every
+scene whose decisions all sit clear of their boundary in the oracle's float64
+arithmetic -- acceptance tests farther than ACCEPT_MARGIN (relative) and the
+final draw farther than DRAW_MARGIN (probability units) from a step of the
+cumulative sum; these bounds sit well above the fp32 error of the kernel's
+normalisers (~1e-6 relative) and running sums (~1e-6 absolute).
+Near-boundary scenes are counted and must be rare.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2606_31160_gb300 import sd, workloads
+from tests.helpers import ensure_lib
+
+pytestmark = pytest.mark.gpu
+
+ACCEPT_MARGIN = 1e-5
+DRAW_MARGIN = 2e-6
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    ensure_lib()
+
+
+def _greedy_both(logits, draft):
+    n, t, a = sd.accept_greedy(logits.cuda(), draft.cuda())
+    rn, rt, ra = oracle.accept_greedy(logits.float().numpy(), draft.numpy())
+    assert n.cpu().numpy().tolist() == rn.tolist()
+    assert t.cpu().numpy().tolist() == rt.tolist()
+    assert a.cpu().numpy().tolist() == ra.tolist()
+    return rn
+
+
+@pytest.mark.parametrize("make", [workloads.tiny, workloads.target_layer])
+def test_greedy_workloads(make):
+    case = make()
+    rn = _greedy_both(case.extra["logits"], case.extra["draft"])
+    assert rn.tolist() == (case.extra["ell"] + 1).tolist()
+
+
+@pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
+@pytest.mark.parametrize("B,K,V", [(1, 0, 5), (3, 1, 4097), (8, 7, 151936), (2, 16, 32000), (5, 3, 123457)])
+def test_greedy_random(dtype, B, K, V):
+    rng = np.random.default_rng(B * 1000 + K + V)
+    z = rng.standard_normal((B, K + 1, V)).astype(np.float32) * 2
+    logits = torch.from_numpy(z).to(dtype)
+    star = logits.float().argmax(-1).numpy()
+    draft = np.where(rng.random((B, K)) < 0.7, star[:, :K], rng.integers(0, V, (B, K)))
+    _greedy_both(logits, torch.from_numpy(draft.astype(np.int32)))
+
+
+def test_greedy_all_match_and_planted_ties():
+    B, K, V = 4, 7, 151936
+    rng = np.random.default_rng(70)
+    z = rng.standard_normal((B, K + 1, V)).astype(np.float32)
+    # ties of the maximum in different chunks of the vocabulary, +0 / -0 ties,
+    # and a row whose every entry is equal
+    z[0, 0, [5, 70000, 151935]] = 9.0
+    z[0, 1, [151935, 4096, 4095]] = 9.0
+    z[1, 2, :] = -1.0
+    z[1, 3, :] = 0.0
+    z[1, 3, [100, 7]] = -0.0
+    z[2, 0, [60000, 60001]] = np.float32(8.5)
+    logits = torch.from_numpy(z).to(torch.bfloat16)
+    star = oracle.accept_greedy(logits.float().numpy(), np.zeros((B, K), np.int64))[2]
+    assert star[0, 0] == 5 and star[0, 1] == 4095 and star[1, 2] == 0 and star[1, 3] == 0
+    draft = torch.from_numpy(star[:, :K].astype(np.int32))   # all drafts match
+    rn = _greedy_both(logits, draft)
+    assert rn.tolist() == [K + 1] * B
+
+
+def test_greedy_workspace_reuse_and_counters_rearm():
+    case = workloads.target_layer()
+    logits, draft = case.extra["logits"].cuda(), case.extra["draft"].cuda()
+    ws = sd.workspace(sd.greedy_workspace_bytes(1, 7, logits.shape[-1]))
+    first = [x.clone() for x in sd.accept_greedy(logits, draft, ws=ws)]
+    for _ in range(3):
+        again = sd.accept_greedy(logits, draft, ws=ws)
+        assert all(torch.equal(a, b) for a, b in zip(first, again))
+    assert sd.get_device_error() == 0
+
+
+def test_greedy_draft_out_of_range_sets_error():
+    logits = torch.zeros((1, 3, 10), dtype=torch.float32, device="cuda")
+    draft = torch.tensor([[0, 12]], dtype=torch.int32, device="cuda")
+    sd.get_device_error()
+    n, t, _ = sd.accept_greedy(logits, draft)
+    assert sd.get_device_error() & sd.SD_DEVERR_TOKEN_RANGE
+    assert n.item() == 2   # draft 0 matches argmax 0; draft 1 never can
+
+
+# ------------------------------------------------------------------ sampling
+
+def _sample_both(z_t, z_d, draft, u, T):
+    n, t = sd.accept_sample(z_t.cuda(), z_d.cuda(), draft.cuda(), u.cuda(), T)
+    rn, rt, margins = oracle.accept_sample(z_t.numpy(), z_d.numpy(), draft.numpy(), u.numpy(), T)
+    n, t = n.cpu().numpy(), t.cpu().numpy()
+    near = [b for b in range(len(rn))
+            if min(margins[b][:-1], default=1.0) < ACCEPT_MARGIN or margins[b][-1] < DRAW_MARGIN]
+    for b in range(len(rn)):
+        if b in near:
+            continue
+        assert n[b] == rn[b], (b, n[b], rn[b])
+        assert t[b].tolist() == rt[b].tolist(), (b, t[b], rt[b])
+    return rn, near
+
+
+def test_sample_stochastic_workload():
+    w = workloads.stochastic()
+    rn, near = _sample_both(w["z_target"], w["z_draft"], w["draft"], w["u"], w["temperature"])
+    assert len(near) == 0
+    assert rn.min() >= 1 and rn.max() <= w["K"] + 1
+
+
+@pytest.mark.parametrize("seed", range(4))
+def test_sample_more_seeds(seed):
+    w = workloads.stochastic(B=16, K=5, V=50000, temperature=0.8, seed_layer=10 + seed)
+    rn, near = _sample_both(w["z_target"], w["z_draft"], w["draft"], w["u"], w["temperature"])
+    assert len(near) <= 4   # flatter T = 0.8 rows over 50k tokens have small CDF steps
+
+
+def test_sample_equal_distributions_always_accept():
+    rng = np.random.default_rng(80)
+    B, K, V = 8, 7, 20000
+    z = torch.from_numpy(rng.standard_normal((B, K + 1, V)).astype(np.float32))
+    draft = torch.from_numpy(rng.integers(0, V, (B, K)).astype(np.int32))
+    u = torch.from_numpy(workloads.uniforms24(rng, (B, K + 1)))
+    n, t = sd.accept_sample(z.cuda(), z[:, :K].contiguous().cuda(), draft.cuda(), u.cuda(), 0.7)
+    assert n.cpu().tolist() == [K + 1] * B
+    assert torch.equal(t[:, :K].cpu(), draft)
+
+
+def test_sample_output_law_by_enumeration_on_gpu():
+    # Leviathan/Chen on a 5-token vocabulary through the kernel: every draft
+    # token x (weight q(x)) times an N x N grid of uniforms, in one batch.
+    rng = np.random.default_rng(81)
+    V, T, N = 5, 0.8, 64
+    z_t = (rng.standard_normal((2, V)) * 1.5).astype(np.float32)
+    z_d = (rng.standard_normal((1, V)) * 1.5).astype(np.float32)
+    grid = (np.arange(N) + 0.5) / N
+    u0, u1 = np.meshgrid(grid, grid, indexing="ij")
+    u = np.stack([u0.ravel(), u1.ravel()], 1).astype(np.float32)
+    n = u.shape[0]
+    B = V * n
+    zt = torch.from_numpy(np.ascontiguousarray(np.broadcast_to(z_t, (B, 2, V))))
+    zd = torch.from_numpy(np.ascontiguousarray(np.broadcast_to(z_d, (B, 1, V))))
+    draft = torch.from_numpy(np.repeat(np.arange(V), n).astype(np.int32).reshape(B, 1))
+    uu = torch.from_numpy(np.tile(u, (V, 1)))
+    nn, tt = sd.accept_sample(zt.cuda(), zd.cuda(), draft.cuda(), uu.cuda(), T)
+    first = tt[:, 0].cpu().numpy().reshape(V, n)
+    q = np.exp((z_d[0] - z_d[0].max()) / T)
+    q /= q.sum()
+    p = np.exp((z_t[0] - z_t[0].max()) / T)
+    p /= p.sum()
+    dist = sum(q[x] * np.bincount(first[x], minlength=V) / n for x in range(V))
+    np.testing.assert_allclose(dist, p, atol=2.0 / N + 1e-6)

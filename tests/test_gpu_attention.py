@@ -1,0 +1,115 @@
+"""GPU parity of sd_verify_attention against the float64 oracle (Eq. verify).
+
+The oracle reads the very bf16 values the kernel read (rotated Q and the
+cache after the append, copied back from the device), so the comparison
+isolates the attention arithmetic. Bar: max-abs error <= 1e-2.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2606_31160_gb300 import sd, workloads
+from tests.helpers import ATTN_ATOL, ensure_lib, run_verify_layer, to64
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    ensure_lib()
+
+
+def _oracle_out(q, cache, scenes=None, heads=None):
+    lens = cache.len.cpu().numpy()
+    qq, kk, vv = to64(q), to64(cache.k), to64(cache.v)
+    if scenes is None:
+        return oracle.verify_attention(qq, kk, vv, lens), slice(None)
+    sel = list(scenes)
+    return oracle.verify_attention(qq[sel], kk[sel], vv[sel], lens[sel]), sel
+
+
+def _assert_close(got, ref):
+    err = np.abs(got - ref)
+    assert np.isfinite(got).all()
+    assert err.max() <= ATTN_ATOL, (float(err.max()), float(np.sqrt((err ** 2).mean())))
+
+
+@pytest.mark.parametrize("make", [workloads.tiny, workloads.target_layer])
+def test_workload_layers(make):
+    case = make()
+    q, _, cache, out = run_verify_layer(case)
+    assert cache.len.cpu().tolist() == [int(x) + case.R for x in case.prefix]
+    ref, _ = _oracle_out(q, cache)
+    _assert_close(to64(out), ref)
+
+
+def _random_case(seed, B, R, Hq, Hkv, D, prefix, cap, tail):
+    rng = np.random.default_rng(seed)
+    prefix = np.asarray(prefix)
+    k = rng.standard_normal((B, Hkv, cap, D)).astype(np.float32)
+    v = rng.standard_normal((B, Hkv, cap, D)).astype(np.float32)
+    for b in range(B):  # stale rows past the valid length
+        k[b, :, prefix[b] + R:] = tail
+        v[b, :, prefix[b] + R:] = tail
+    q = workloads.to_bf16(rng.standard_normal((B, R, Hq, D)))
+    cache = sd.KVCache(workloads.to_bf16(k).cuda(), workloads.to_bf16(v).cuda(),
+                       torch.from_numpy((prefix + R).astype(np.int32)).cuda())
+    return q.cuda(), cache
+
+
+@pytest.mark.parametrize("B,R,Hq,Hkv,D,prefix", [
+    (1, 1, 4, 4, 64, [0]),              # single key
+    (1, 1, 16, 4, 128, [4096]),         # draft decode shape (K = 0)
+    (2, 2, 8, 8, 128, [15, 16]),        # G = 1, ragged around a 16-key block
+    (3, 5, 4, 1, 64, [1, 17, 300]),
+    (2, 8, 32, 8, 128, [4095, 1000]),   # target shape, ragged
+    (2, 8, 64, 8, 128, [63, 129]),      # G * R = 64 (two row groups)
+    (1, 17, 32, 8, 128, [2000]),        # K = 16: G * R = 68 (two row blocks)
+    (2, 16, 64, 8, 64, [33, 700]),      # G * R = 128
+    (1, 3, 6, 2, 128, [50]),            # G = 3, odd packing
+])
+@pytest.mark.parametrize("tail", [0.0, np.nan])
+def test_random_shapes_and_stale_tail(B, R, Hq, Hkv, D, prefix, tail):
+    cap = max(prefix) + R + 21
+    q, cache = _random_case(7 + B * R, B, R, Hq, Hkv, D, prefix, cap, tail)
+    out = sd.verify_attention(q, cache)
+    ref, _ = _oracle_out(q, cache)
+    _assert_close(to64(out), ref)
+
+
+def test_explicit_scale():
+    q, cache = _random_case(3, 1, 4, 8, 2, 64, [100], 120, 0.0)
+    out = sd.verify_attention(q, cache, scale=0.05)
+    qq, kk, vv = to64(q), to64(cache.k), to64(cache.v)
+    ref = oracle.verify_attention(qq, kk, vv, cache.len.cpu().numpy(), scale=0.05)
+    _assert_close(to64(out), ref)
+
+
+def test_deterministic_across_calls():
+    q, cache = _random_case(5, 2, 8, 32, 8, 128, [3000, 4096], 4200, 0.0)
+    a = sd.verify_attention(q, cache)
+    b = sd.verify_attention(q, cache)
+    assert torch.equal(a, b)
+
+
+@pytest.mark.slow
+@pytest.mark.parametrize("B,L,K", [(1, 2048, 1), (8, 4096, 7), (32, 16384, 16), (32, 8192, 2)])
+def test_sweep_full_size_sampled(B, L, K):
+    # full-size batched sweep, checked on sampled scenes (oracle cost)
+    case = workloads.sweep_case(B, L, K)
+    q, _, cache, out = run_verify_layer(case)
+    scenes = sorted({0, B // 2, B - 1})
+    ref, sel = _oracle_out(q, cache, scenes)
+    _assert_close(to64(out)[sel], ref)
+
+
+def test_invalid_length_sets_error_and_leaves_output():
+    q, cache = _random_case(9, 2, 4, 8, 2, 64, [10, 20], 40, 0.0)
+    sd.get_device_error()
+    cache.len.copy_(torch.tensor([2, 99], dtype=torch.int32))  # scene 0: len < R; scene 1: > cap
+    out = torch.full_like(q, 7.0)
+    sd.verify_attention(q, cache, out=out)
+    bits = sd.get_device_error()
+    assert bits & sd.SD_DEVERR_LENGTH
+    assert torch.all(out == 7.0)
