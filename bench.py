@@ -314,6 +314,9 @@ def main():
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--cpu-budget", type=float, default=12.0, help="seconds of oracle time (rank 0)")
+    ap.add_argument("--only", choices=["attention", "accept", "step"], default=None,
+                    help="profiling mode: run one kernel family eagerly `steps` times on the "
+                         "target-layer workload (for ncu captures); prints no bench line")
     args = ap.parse_args()
     world, rank, local = dist_env()
     if args.warmup < 3:
@@ -321,6 +324,8 @@ def main():
 
     if args.impl == "reference":
         return reference_arm(args, world, rank)
+    if args.only:
+        return profile_only(args)
 
     import torch.distributed as dist
     torch.cuda.set_device(local)
@@ -465,6 +470,30 @@ def main():
     if world > 1:
         dist.barrier()
         dist.destroy_process_group()
+
+
+def profile_only(args):
+    """Eager launches of one kernel family on the 36-layer target workload,
+    for profiler captures (a handful of launches, no timing output)."""
+    from paper_2606_31160_gb300 import build, sd
+    build.build()
+    torch.cuda.set_device(0)
+    st = Step(torch.device("cuda", 0))
+    st.run()  # one full step: rope, append, attention, accept, rollback
+    torch.cuda.synchronize()
+    for l in range(LAYERS):  # leave every cache holding L + R keys
+        sd.kv_append(st.caches[l], st.k[l], st.v[l])
+    for i in range(args.steps):
+        if args.only == "attention":
+            sd.verify_attention(st.q[i % LAYERS], st.caches[i % LAYERS], out=st.out[i % LAYERS])
+        elif args.only == "accept":
+            st.accept_only()
+        else:
+            st.lens.fill_(L)
+            st.run()
+    torch.cuda.synchronize()
+    print(json.dumps({"profile_only": args.only, "launches": args.steps,
+                      "device_error": sd.get_device_error()}))
 
 
 def reference_arm(args, world, rank):

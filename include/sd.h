@@ -134,6 +134,13 @@ sd_status sd_kv_rollback(int32_t* len, int count, int B, const int32_t* committe
                          int n_appended, sd_stream_t stream);
 
 /*
+ * Workspace bytes sd_verify_attention needs for this shape on the CURRENT
+ * device (the split plan depends on its SM count): 0 when the batch alone
+ * fills the GPU and no split merge is needed. capacity = cache capacity.
+ */
+size_t sd_verify_attention_workspace(int B, int R, int Hq, int Hkv, int D, int capacity);
+
+/*
  * Verify attention (Eq. verify, Sec. 2.2): for scene b, query head h (KV head
  * g = h / G) and row i < R,
  *   o[b][i][h] = softmax_n( q[b][i][h] . k[b][g][n] * scale ) v[b][g][n],
@@ -144,12 +151,20 @@ sd_status sd_kv_rollback(int32_t* len, int count, int B, const int32_t* committe
  *   out: [B][R][Hq][D] bf16.
  *   scale: 0 selects 1/sqrt(D).
  * The G*R query rows that share a KV head are packed into one tile, so each
- * K/V row is read from HBM once. Requires D in {64, 128}, Hq % Hkv == 0 and
+ * K/V row is read from HBM once; when B*Hkv alone cannot fill the GPU each
+ * head's keys are split over several CTAs whose partial softmax states merge
+ * through `workspace` (sd_verify_attention_workspace bytes, zero-filled
+ * before its first use and left zeroed by every completed call; calls that
+ * share a workspace must not overlap on the device; after SD_ERR_TIMEOUT it
+ * must be zero-filled again). Requires D in {64, 128}, Hq % Hkv == 0 and
  * G*R <= 128. A scene with len[b] < R or len[b] > capacity sets
- * SD_DEVERR_LENGTH and its output is left unwritten. No workspace.
+ * SD_DEVERR_LENGTH and its output is left unwritten. The first call per
+ * device and shape should come before any stream capture (it sets kernel
+ * attributes and queries the occupancy).
  */
 sd_status sd_verify_attention(const void* q, const sd_kv_cache* cache, void* out,
-                              int R, int Hq, float scale, sd_stream_t stream);
+                              int R, int Hq, float scale, void* workspace, size_t ws_bytes,
+                              sd_stream_t stream);
 
 /*
  * Workspace bytes sd_accept_greedy needs for (B, R = K + 1, V).

@@ -25,7 +25,8 @@ extern "C" sd_status sd_get_device_error(sd_stream_t stream, uint32_t* bits) {
     return SD_ERR_CUDA;
   }
   cudaError_t (*take[])(uint32_t*) = {sd_take_error_rope, sd_take_error_kv,
-                                      sd_take_error_attention, sd_take_error_greedy,
+                                      sd_take_error_attention, sd_take_error_attention_tc,
+                                      sd_take_error_greedy,
                                       sd_take_error_sample};
   for (auto fn : take) {
     if (fn(bits) != cudaSuccess) {

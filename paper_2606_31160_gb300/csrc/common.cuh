@@ -32,8 +32,17 @@ __device__ __forceinline__ void sd_set_error(uint32_t bits) { atomicOr(&sd_err_w
 cudaError_t sd_take_error_rope(uint32_t* bits);
 cudaError_t sd_take_error_kv(uint32_t* bits);
 cudaError_t sd_take_error_attention(uint32_t* bits);
+cudaError_t sd_take_error_attention_tc(uint32_t* bits);
 cudaError_t sd_take_error_greedy(uint32_t* bits);
 cudaError_t sd_take_error_sample(uint32_t* bits);
+
+// Verify attention on the tcgen05 path (attention_tc.cu). Sets *handled when
+// the shape is one it serves (head_dim 128, G * R <= 32) and it launched.
+sd_status sd_internal_verify_attention_tc(const void* q, const sd_kv_cache* cache, void* out,
+                                          int R, int Hq, float scale_log2, cudaStream_t stream,
+                                          bool* handled);
+// Whether the tcgen05 path serves this shape on the current device.
+bool sd_internal_tc_serves(int B, int R, int Hq, int Hkv, int D, int cap);
 
 // ---------------------------------------------------------------------------
 // Host helpers

@@ -47,7 +47,8 @@ _SIGNATURES = {
     "sd_rope_apply_1d": ([_vp, _vp, _i, _i, _i, _i, _i, _vp, _f, _vp], _i),
     "sd_kv_append": ([ctypes.POINTER(KVCacheStruct), _vp, _vp, _i, _vp], _i),
     "sd_kv_rollback": ([_vp, _i, _i, _vp, _i, _vp], _i),
-    "sd_verify_attention": ([_vp, ctypes.POINTER(KVCacheStruct), _vp, _i, _i, _f, _vp], _i),
+    "sd_verify_attention_workspace": ([_i, _i, _i, _i, _i, _i], _sz),
+    "sd_verify_attention": ([_vp, ctypes.POINTER(KVCacheStruct), _vp, _i, _i, _f, _vp, _sz, _vp], _i),
     "sd_accept_greedy_workspace": ([_i, _i, _i], _sz),
     "sd_accept_greedy": ([_vp, _i, _i, _i, _i, _vp, _vp, _vp, _vp, _vp, _sz, _vp], _i),
     "sd_accept_sample_workspace": ([_i, _i, _i], _sz),
@@ -191,16 +192,33 @@ def kv_rollback(lens, committed, n_appended):
 
 # ----------------------------------------------------------------- attention
 
-def verify_attention(q, cache, out=None, scale=0.0):
-    """Causal GQA verify attention of q [B,R,Hq,D] (rotated) over the cache (appended)."""
+def attention_workspace_bytes(B, R, Hq, Hkv, D, capacity):
+    return int(lib().sd_verify_attention_workspace(B, R, Hq, Hkv, D, capacity))
+
+
+_attn_ws = {}
+
+
+def verify_attention(q, cache, out=None, scale=0.0, ws=None):
+    """Causal GQA verify attention of q [B,R,Hq,D] (rotated) over the cache (appended).
+    ws: the split-merge workspace (see sd_verify_attention_workspace); when None a
+    zero-filled one is kept per (device, shape) and reused by later calls."""
     B, R, Hq, D = q.shape
     if cache.shape[0] != B or cache.shape[3] != D:
         raise ValueError("q and cache disagree")
     if out is None:
         out = torch.empty_like(q)
+    if ws is None:
+        need = attention_workspace_bytes(B, R, Hq, cache.shape[1], D, cache.shape[2])
+        key = (q.device.index, need)
+        if need and key not in _attn_ws:
+            _attn_ws[key] = workspace(need, q.device)
+        ws = _attn_ws.get(key)
+    wp = _dev(ws, "ws") if ws is not None else ctypes.c_void_p(0)
+    nbytes = ws.numel() * ws.element_size() if ws is not None else 0
     _check(lib().sd_verify_attention(_dev(q, "q", torch.bfloat16), cache.struct,
-                                     _dev(out, "out", torch.bfloat16), R, Hq, float(scale), _stream()),
-           "sd_verify_attention")
+                                     _dev(out, "out", torch.bfloat16), R, Hq, float(scale), wp, nbytes,
+                                     _stream()), "sd_verify_attention")
     return out
 
 

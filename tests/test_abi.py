@@ -17,7 +17,7 @@ def lib():
 
 def test_every_header_symbol_is_exported(lib):
     names = sd.header_symbols()
-    assert len(names) >= 12
+    assert len(names) >= 13
     for name in names:
         assert hasattr(lib, name), name
     out = subprocess.run(["nm", "-D", "--defined-only", sd.LIB_PATH], capture_output=True, text=True).stdout
@@ -56,17 +56,17 @@ def test_workspace_queries_are_host_arithmetic(lib):
 def test_bad_arguments_return_status_before_launch(lib):
     null = ctypes.c_void_p(0)
     # NULL cache / unsupported head dim / bad GQA ratio
-    assert lib.sd_verify_attention(null, None, null, 8, 32, 0.0, null) == 1
+    assert lib.sd_verify_attention(null, None, null, 8, 32, 0.0, null, 0, null) == 1
     cache = sd.KVCacheStruct(16, 16, 16, 1, 8, 64, 96)
-    assert lib.sd_verify_attention(ctypes.c_void_p(16), ctypes.byref(cache), ctypes.c_void_p(16), 8, 32, 0.0, null) == 2
+    assert lib.sd_verify_attention(ctypes.c_void_p(16), ctypes.byref(cache), ctypes.c_void_p(16), 8, 32, 0.0, null, 0, null) == 2
     cache = sd.KVCacheStruct(16, 16, 16, 1, 3, 64, 128)
-    assert lib.sd_verify_attention(ctypes.c_void_p(16), ctypes.byref(cache), ctypes.c_void_p(16), 8, 32, 0.0, null) == 1
+    assert lib.sd_verify_attention(ctypes.c_void_p(16), ctypes.byref(cache), ctypes.c_void_p(16), 8, 32, 0.0, null, 0, null) == 1
     # G * R beyond the packed-tile limit
     cache = sd.KVCacheStruct(16, 16, 16, 1, 1, 64, 128)
-    assert lib.sd_verify_attention(ctypes.c_void_p(16), ctypes.byref(cache), ctypes.c_void_p(16), 17, 8, 0.0, null) == 2
+    assert lib.sd_verify_attention(ctypes.c_void_p(16), ctypes.byref(cache), ctypes.c_void_p(16), 17, 8, 0.0, null, 0, null) == 2
     # misaligned pointer
     cache = sd.KVCacheStruct(18, 16, 16, 1, 8, 64, 128)
-    assert lib.sd_verify_attention(ctypes.c_void_p(16), ctypes.byref(cache), ctypes.c_void_p(16), 8, 32, 0.0, null) == 1
+    assert lib.sd_verify_attention(ctypes.c_void_p(16), ctypes.byref(cache), ctypes.c_void_p(16), 8, 32, 0.0, null, 0, null) == 1
     # rope: unsupported head dim, bad sections
     sec = (ctypes.c_int32 * 3)(16, 24, 24)
     assert lib.sd_rope_apply(ctypes.c_void_p(16), ctypes.c_void_p(16), 1, 8, 32, 8, 96, ctypes.c_void_p(16), sec, 0, 1e6, null) == 2
@@ -86,4 +86,4 @@ def test_bad_arguments_return_status_before_launch(lib):
                                 ctypes.c_void_p(16), 1 << 20, null) == 1
     # empty batches are a no-op success
     cache = sd.KVCacheStruct(0, 0, 0, 0, 8, 64, 128)
-    assert lib.sd_verify_attention(null, ctypes.byref(cache), null, 8, 32, 0.0, null) == 0
+    assert lib.sd_verify_attention(null, ctypes.byref(cache), null, 8, 32, 0.0, null, 0, null) == 0

@@ -113,3 +113,24 @@ def test_invalid_length_sets_error_and_leaves_output():
     bits = sd.get_device_error()
     assert bits & sd.SD_DEVERR_LENGTH
     assert torch.all(out == 7.0)
+
+
+def test_workspace_is_required_and_left_zeroed():
+    # G * R = 64 takes the mma.sync kernel, whose splits merge through the workspace
+    q, cache = _random_case(11, 1, 8, 64, 8, 128, [4000], 4200, 0.0)
+    need = sd.attention_workspace_bytes(1, 8, 64, 8, 128, 4200)
+    assert need > 0   # one scene x 8 KV heads cannot fill the GPU: splits merge
+    out = torch.empty_like(q)
+    small = sd.workspace(16)
+    with pytest.raises(sd.SDError):
+        sd.verify_attention(q, cache, out=out, ws=small)
+    ws = sd.workspace(need)
+    a = sd.verify_attention(q, cache, ws=ws).clone()
+    b = sd.verify_attention(q, cache, ws=ws)
+    assert torch.equal(a, b)
+    units = 8
+    assert sd.get_device_error() == 0
+    # the arrival / departure counters are re-armed after every call
+    n_sp_part = need - units * 8 - 256
+    cnt = ws[n_sp_part:n_sp_part + units * 8].view(torch.int32)
+    assert int(cnt.abs().sum()) == 0
