@@ -190,6 +190,28 @@ sd_status sd_accept_greedy(const void* logits, sd_dtype dtype, int B, int K, int
                            sd_stream_t stream);
 
 /*
+ * Greedy acceptance without a caller workspace (the paper has no counterpart:
+ * this serves callers that cannot allocate device memory -- a serving loop
+ * whose pool belongs to another runtime, a pre-planned graph that forbids
+ * allocation while it runs, a host with no device allocator).
+ * Same arguments, results and rules as sd_accept_greedy minus ws / ws_bytes.
+ * Its scratch is a fixed array inside the library of
+ * sd_accept_greedy_noalloc_max_bytes() bytes (1 MiB: per-scene tickets for up
+ * to 4096 scenes, then B * (K + 1) * ceil(V / 4096) partials of 8 bytes), held
+ * on every device that loads the library until the process exits. Larger
+ * shapes return SD_ERR_WORKSPACE. Allocates nothing. The first call on a
+ * device resolves the array's device address (make it before any stream
+ * capture). All calls share the array: calls that overlap on the device race
+ * and must not be issued; every completed call leaves it ready for the next.
+ */
+sd_status sd_accept_greedy_noalloc(const void* logits, sd_dtype dtype, int B, int K, int V,
+                                   const int32_t* draft, int32_t* n_emit, int32_t* tokens,
+                                   int32_t* argmax, sd_stream_t stream);
+
+/* Bytes of the fixed scratch array behind sd_accept_greedy_noalloc. */
+size_t sd_accept_greedy_noalloc_max_bytes(void);
+
+/*
  * Workspace bytes sd_accept_sample needs for (B, K, V).
  */
 size_t sd_accept_sample_workspace(int B, int K, int V);

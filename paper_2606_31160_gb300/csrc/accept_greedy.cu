@@ -15,6 +15,8 @@
 // deterministic.
 #include "common.cuh"
 
+#include <mutex>
+
 SD_DEFINE_ERROR_ACCESSOR(sd_take_error_greedy)
 
 namespace {
@@ -204,25 +206,23 @@ extern "C" size_t sd_accept_greedy_workspace(int B, int K, int V) {
   return ws_bytes_for(B, K + 1, n_chunks);
 }
 
-extern "C" sd_status sd_accept_greedy(const void* logits, sd_dtype dtype, int B, int K, int V,
-                                      const int32_t* draft, int32_t* n_emit, int32_t* tokens,
-                                      int32_t* argmax, void* ws, size_t ws_bytes,
-                                      sd_stream_t stream) {
+// Host-side argument checks shared by both entry points.
+static sd_status check_args(const void* logits, sd_dtype dtype, int B, int K, int V,
+                            const int32_t* draft, int32_t* n_emit, int32_t* tokens) {
   if (B < 0 || K < 0 || V <= 0) return SD_ERR_INVALID_ARG;
   if (dtype != SD_BF16 && dtype != SD_F32) return SD_ERR_INVALID_ARG;
   if (K + 1 > 128 || B > 65535) return SD_ERR_UNSUPPORTED;
   if (B == 0) return SD_OK;
   if (!logits || !n_emit || !tokens || (K > 0 && !draft)) return SD_ERR_INVALID_ARG;
+  return SD_OK;
+}
+
+static sd_status launch(const void* logits, sd_dtype dtype, int B, int K, int V,
+                        const int32_t* draft, int32_t* n_emit, int32_t* tokens, int32_t* argmax,
+                        float2* part, uint32_t* ticket, int chunk, int n_chunks,
+                        cudaStream_t st) {
   const int R = K + 1;
-  int chunk, n_chunks;
-  plan(B, R, V, &chunk, &n_chunks);
-  const size_t need = ws_bytes_for(B, R, n_chunks);
-  if (!ws || ws_bytes < need || !sd_aligned16(ws)) return SD_ERR_WORKSPACE;
-  auto* part = static_cast<float2*>(ws);
-  auto* ticket = reinterpret_cast<uint32_t*>(static_cast<char*>(ws) +
-                                             static_cast<size_t>(B) * R * n_chunks * sizeof(float2));
   const dim3 grid(n_chunks, R, B);
-  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   if (dtype == SD_BF16)
     greedy_kernel<__nv_bfloat16><<<grid, kThreads, 0, st>>>(
         static_cast<const __nv_bfloat16*>(logits), R, V, chunk, n_chunks, draft, n_emit, tokens,
@@ -233,4 +233,86 @@ extern "C" sd_status sd_accept_greedy(const void* logits, sd_dtype dtype, int B,
                                                     ticket);
   SD_CHECK_LAUNCH();
   return SD_OK;
+}
+
+extern "C" sd_status sd_accept_greedy(const void* logits, sd_dtype dtype, int B, int K, int V,
+                                      const int32_t* draft, int32_t* n_emit, int32_t* tokens,
+                                      int32_t* argmax, void* ws, size_t ws_bytes,
+                                      sd_stream_t stream) {
+  const sd_status chk = check_args(logits, dtype, B, K, V, draft, n_emit, tokens);
+  if (chk != SD_OK || B == 0) return chk;
+  const int R = K + 1;
+  int chunk, n_chunks;
+  plan(B, R, V, &chunk, &n_chunks);
+  const size_t need = ws_bytes_for(B, R, n_chunks);
+  if (!ws || ws_bytes < need || !sd_aligned16(ws)) return SD_ERR_WORKSPACE;
+  auto* part = static_cast<float2*>(ws);
+  auto* ticket = reinterpret_cast<uint32_t*>(static_cast<char*>(ws) +
+                                             static_cast<size_t>(B) * R * n_chunks * sizeof(float2));
+  return launch(logits, dtype, B, K, V, draft, n_emit, tokens, argmax, part, ticket, chunk, n_chunks,
+                reinterpret_cast<cudaStream_t>(stream));
+}
+
+// ---------------------------------------------------------------------------
+// Allocation-free variant. Some callers cannot allocate device memory at the
+// point where they accept drafts: a serving loop whose memory pool is owned
+// and fully carved up by another runtime, a pre-planned inference graph that
+// forbids allocation once it runs, or an embedded host that has no device
+// allocator at all. For them the scratch this kernel needs lives in a
+// file-scope device array of fixed size, loaded with the library (every GPU
+// that loads it holds these bytes until the process exits).
+//
+// Layout: tickets of up to kNoAllocMaxB scenes at the front, so their place
+// never moves with the call's shape and no partial result lands on them; the
+// per-chunk partials follow. The array starts zeroed when the module loads,
+// and every completed call leaves the tickets at zero again; the partials
+// need no clearing. All calls share the array: calls that overlap on the GPU
+// (other streams, other threads) race and must not be issued.
+// ---------------------------------------------------------------------------
+constexpr size_t kNoAllocBytes = size_t(1) << 20;  // 1 MiB
+constexpr int kNoAllocMaxB = 4096;
+constexpr size_t kNoAllocTicketBytes = kNoAllocMaxB * sizeof(uint32_t);
+static __device__ __align__(256) unsigned char g_greedy_scratch[kNoAllocBytes];
+
+// Device address of the array on the current device, resolved once per device
+// (host code cannot use the symbol itself: it is a host-side stand-in).
+static void* noalloc_scratch() {
+  static void* ptrs[64] = {nullptr};
+  static std::mutex mu;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) {
+    (void)cudaGetLastError();
+    return nullptr;
+  }
+  std::lock_guard<std::mutex> lock(mu);
+  if (!ptrs[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_greedy_scratch) != cudaSuccess || !p) {
+      (void)cudaGetLastError();
+      return nullptr;
+    }
+    ptrs[dev] = p;
+  }
+  return ptrs[dev];
+}
+
+extern "C" size_t sd_accept_greedy_noalloc_max_bytes(void) { return kNoAllocBytes; }
+
+extern "C" sd_status sd_accept_greedy_noalloc(const void* logits, sd_dtype dtype, int B, int K,
+                                              int V, const int32_t* draft, int32_t* n_emit,
+                                              int32_t* tokens, int32_t* argmax,
+                                              sd_stream_t stream) {
+  const sd_status chk = check_args(logits, dtype, B, K, V, draft, n_emit, tokens);
+  if (chk != SD_OK || B == 0) return chk;
+  const int R = K + 1;
+  int chunk, n_chunks;
+  plan(B, R, V, &chunk, &n_chunks);
+  const size_t part_bytes = static_cast<size_t>(B) * R * n_chunks * sizeof(float2);
+  if (B > kNoAllocMaxB || kNoAllocTicketBytes + part_bytes > kNoAllocBytes) return SD_ERR_WORKSPACE;
+  void* scratch = noalloc_scratch();
+  if (!scratch) return SD_ERR_CUDA;
+  auto* ticket = static_cast<uint32_t*>(scratch);
+  auto* part = reinterpret_cast<float2*>(static_cast<char*>(scratch) + kNoAllocTicketBytes);
+  return launch(logits, dtype, B, K, V, draft, n_emit, tokens, argmax, part, ticket, chunk, n_chunks,
+                reinterpret_cast<cudaStream_t>(stream));
 }

@@ -51,6 +51,8 @@ _SIGNATURES = {
     "sd_verify_attention": ([_vp, ctypes.POINTER(KVCacheStruct), _vp, _i, _i, _f, _vp, _sz, _vp], _i),
     "sd_accept_greedy_workspace": ([_i, _i, _i], _sz),
     "sd_accept_greedy": ([_vp, _i, _i, _i, _i, _vp, _vp, _vp, _vp, _vp, _sz, _vp], _i),
+    "sd_accept_greedy_noalloc": ([_vp, _i, _i, _i, _i, _vp, _vp, _vp, _vp, _vp], _i),
+    "sd_accept_greedy_noalloc_max_bytes": ([], _sz),
     "sd_accept_sample_workspace": ([_i, _i, _i], _sz),
     "sd_accept_sample": ([_vp, _vp, _i, _i, _i, _f, _vp, _vp, _vp, _vp, _vp, _sz, _vp], _i),
     "sd_get_device_error": ([_vp, ctypes.POINTER(ctypes.c_uint32)], _i),
@@ -251,6 +253,27 @@ def accept_greedy(logits, draft, ws=None, n_emit=None, tokens=None, argmax=None)
                                   _dev(n_emit, "n_emit", torch.int32), _dev(tokens, "tokens", torch.int32),
                                   _dev(argmax, "argmax", torch.int32), _dev(ws, "ws"), ws.numel() * ws.element_size(),
                                   _stream()), "sd_accept_greedy")
+    return n_emit, tokens, argmax
+
+
+def accept_greedy_noalloc(logits, draft, n_emit=None, tokens=None, argmax=None):
+    """sd_accept_greedy_noalloc: greedy acceptance with the library's fixed
+    scratch array instead of a caller workspace (no device allocation)."""
+    B, R, V = logits.shape
+    K = R - 1
+    dt = {torch.bfloat16: SD_BF16, torch.float32: SD_F32}.get(logits.dtype)
+    if dt is None:
+        raise ValueError("logits must be bf16 or fp32")
+    dev = logits.device
+    n_emit = torch.empty(B, dtype=torch.int32, device=dev) if n_emit is None else n_emit
+    tokens = torch.empty((B, R), dtype=torch.int32, device=dev) if tokens is None else tokens
+    argmax = torch.empty((B, R), dtype=torch.int32, device=dev) if argmax is None else argmax
+    draft_p = _dev(draft, "draft", torch.int32) if K > 0 else ctypes.c_void_p(0)
+    _check(lib().sd_accept_greedy_noalloc(_dev(logits, "logits"), dt, B, K, V, draft_p,
+                                          _dev(n_emit, "n_emit", torch.int32),
+                                          _dev(tokens, "tokens", torch.int32),
+                                          _dev(argmax, "argmax", torch.int32), _stream()),
+           "sd_accept_greedy_noalloc")
     return n_emit, tokens, argmax
 
 
