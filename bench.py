@@ -78,7 +78,7 @@ def measured_peaks():
 
 
 def kernel_source_hash():
-    path = os.path.join(ROOT, "paper_2606_31160_gb300", "csrc", "attention.cu")
+    path = os.path.join(ROOT, "paper_2606_31160_gb300", "csrc", "attention_tc.cu")
     with open(path, "rb") as f:
         return hashlib.sha256(f.read()).hexdigest()
 
@@ -437,7 +437,7 @@ def main():
         "accept_us": round(ms_accept * 1e3, 3),
         "bytes_per_step": step_bytes(1),
         "roofline": {
-            "kernel": "sd_verify_attention (verify_attn_kernel<128,2,1>)",
+            "kernel": "sd_verify_attention -> verify_attn_tc_kernel (tcgen05, head_dim 128, G*R <= 32)",
             "bound": "hbm",
             "achieved": round(achieved, 1),
             "peak": peak,
