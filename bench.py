@@ -13,6 +13,9 @@ of all 36 layers to the committed length. After the timed work of a step the
 lengths are put back to L (one 144-byte device copy) so that every step
 processes the same L = 4096 workload.
 
+Each layer is one sd_verify_layer call (M-RoPE + append + attention in one
+tcgen05 kernel); layers after the first are programmatic dependent launches
+that stream their cached prefix while the previous layer still runs.
 The 36 caches (605 MB) exceed the 129 MB L2, so every step streams its KV
 from HBM: "inputs larger than L2". The whole step is captured once in a CUDA
 graph and replayed. Multi-GPU: one independent replica per rank (scenes are
@@ -189,6 +192,8 @@ class Step:
                        for l, c in enumerate(self.cases)]
         self.out = torch.empty_like(self.q)
         self.ws = sd.workspace(sd.greedy_workspace_bytes(1, K, V), device)
+        need = sd.layer_workspace_bytes(1, R, HQ, HKV, D, self.caches[0].shape[2])
+        self.ws_layer = [sd.workspace(need, device) for _ in range(LAYERS)]
         self.n_emit = torch.zeros(1, dtype=torch.int32, device=device)
         self.tokens = torch.zeros((1, R), dtype=torch.int32, device=device)
         self.argmax = torch.zeros((1, R), dtype=torch.int32, device=device)
@@ -196,7 +201,21 @@ class Step:
         for c in self.cases:  # free host copies of the caches
             c.k_cache = c.v_cache = None
 
+    def layers(self):
+        for l in range(LAYERS):
+            self.sd.verify_layer(self.q[l], self.k[l], self.v[l], self.pos, SECTIONS, self.caches[l], 0, BASE,
+                                 out=self.out[l], ws=self.ws_layer[l], early=l > 0)
+
     def run(self):
+        sd = self.sd
+        self.layers()
+        sd.accept_greedy(self.logits, self.draft, ws=self.ws, n_emit=self.n_emit, tokens=self.tokens,
+                         argmax=self.argmax)
+        sd.kv_rollback(self.lens, self.n_emit, R)
+        self.lens.copy_(self.lens0, non_blocking=True)
+
+    def run_unfused(self):
+        """The same step with rope, append and attention as separate kernels."""
         sd = self.sd
         for l in range(LAYERS):
             sd.rope_apply(self.q[l], self.k[l], self.pos, SECTIONS, 0, BASE)
@@ -205,6 +224,11 @@ class Step:
         sd.accept_greedy(self.logits, self.draft, ws=self.ws, n_emit=self.n_emit, tokens=self.tokens,
                          argmax=self.argmax)
         sd.kv_rollback(self.lens, self.n_emit, R)
+        self.lens.copy_(self.lens0, non_blocking=True)
+
+    def layers_only(self):
+        """The 36 fused layer launches alone, lengths put back after them."""
+        self.layers()
         self.lens.copy_(self.lens0, non_blocking=True)
 
     def attention_only(self):
@@ -314,7 +338,7 @@ def main():
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--cpu-budget", type=float, default=12.0, help="seconds of oracle time (rank 0)")
-    ap.add_argument("--only", choices=["attention", "accept", "step"], default=None,
+    ap.add_argument("--only", choices=["attention", "layer", "accept", "step"], default=None,
                     help="profiling mode: run one kernel family eagerly `steps` times on the "
                          "target-layer workload (for ncu captures); prints no bench line")
     args = ap.parse_args()
@@ -342,8 +366,15 @@ def main():
     for _ in range(2):
         st.run()
     torch.cuda.synchronize()
-    g_step = capture(st.run)
+    st.run_unfused()
+    for l in range(LAYERS):  # the standalone attention needs the appended rows
+        sd.kv_append(st.caches[l], st.k[l], st.v[l])
     g_attn = capture(st.attention_only)
+    st.lens.copy_(st.lens0)
+    torch.cuda.synchronize()
+    g_step = capture(st.run)
+    g_layers = capture(st.layers_only)
+    g_unfused = capture(st.run_unfused)
     g_acc = capture(st.accept_only)
     for _ in range(args.warmup):
         g_step.replay()
@@ -372,10 +403,18 @@ def main():
     ms_total = float(t.item())
     ms_step = ms_total / args.steps
 
-    # ---- dominant kernel: verify attention alone (36 distinct caches per replay)
+    # ---- dominant kernel: the fused verify layer, its 36 launches alone
+    #      (distinct caches, chained as programmatic dependent launches)
     reps = max(20, min(2000, args.steps))
-    ms_attn_launch = time_graph(g_attn, reps) / LAYERS
+    ms_layer_launch = time_graph(g_layers, reps) / LAYERS
     ms_accept = time_graph(g_acc, reps)
+    ms_unfused = time_graph(g_unfused, max(20, min(500, args.steps)))
+    # the standalone attention kernel over appended caches, for reference
+    for l in range(LAYERS):
+        sd.kv_append(st.caches[l], st.k[l], st.v[l])
+    ms_attn_launch = time_graph(g_attn, reps) / LAYERS
+    st.lens.copy_(st.lens0)
+    torch.cuda.synchronize()
 
     # ---- end to end: pinned host inputs -> device, step, result -> host
     e2e_steps = max(10, min(500, args.steps))
@@ -406,7 +445,7 @@ def main():
     peak, peak_kind = measured_peaks()
     bytes_step = step_bytes(1) * world
     value = bytes_step / (ms_step * 1e-3) / 1e9
-    achieved = attention_bytes(1) / (ms_attn_launch * 1e-3) / 1e9
+    achieved = layer_bytes(1) / (ms_layer_launch * 1e-3) / 1e9
     traffic = ncu_traffic()
     cpu_gbs, cpu_layers, cpu_s = time_oracle(args.cpu_budget)
     line = {
@@ -430,14 +469,17 @@ def main():
             "parallelism": "replicas" if world > 1 else "single-gpu",
             "l2": "inputs larger than L2: 36 distinct KV caches (605 MB) streamed per step",
             "timing": "CUDA graph of one step, replayed; CUDA events on the launching stream",
+            "layer_kernel": "fused M-RoPE + KV append + verify attention per layer (sd_verify_layer)",
         },
         "verify_step_us": round(ms_step * 1e3, 3),
         "per_layer_us": round(ms_step * 1e3 / LAYERS, 3),
+        "layer_us": round(ms_layer_launch * 1e3, 3),
         "attention_us": round(ms_attn_launch * 1e3, 3),
+        "unfused_verify_step_us": round(ms_unfused * 1e3, 3),
         "accept_us": round(ms_accept * 1e3, 3),
         "bytes_per_step": step_bytes(1),
         "roofline": {
-            "kernel": "sd_verify_attention -> verify_attn_tc_kernel (tcgen05, head_dim 128, G*R <= 32)",
+            "kernel": "sd_verify_layer -> verify_attn_tc_kernel<fused> (M-RoPE + append + attention, tcgen05)",
             "bound": "hbm",
             "achieved": round(achieved, 1),
             "peak": peak,
@@ -445,7 +487,8 @@ def main():
             "unit": "GB/s",
             "frac": round(achieved / peak, 4),
             "traffic": traffic,
-            "algorithmic_bytes_per_launch": attention_bytes(1),
+            "algorithmic_bytes_per_launch": layer_bytes(1),
+            "timing": "36 chained launches of the layer kernel in one graph; average = total / 36",
         },
         "cpu_baseline": {
             "value": round(cpu_gbs, 4),
@@ -463,7 +506,7 @@ def main():
             "h2d_bytes_per_step": st.h2d_bytes,
             "d2h_bytes_per_step": st.d2h_bytes,
         },
-        "gpu_launches": args.steps * (3 * LAYERS + 2),
+        "gpu_launches": args.steps * (LAYERS + 2),
         "clocks": clocks.summary(),
     }
     print(json.dumps(line), flush=True)
@@ -486,6 +529,11 @@ def profile_only(args):
     for i in range(args.steps):
         if args.only == "attention":
             sd.verify_attention(st.q[i % LAYERS], st.caches[i % LAYERS], out=st.out[i % LAYERS])
+        elif args.only == "layer":
+            l = i % LAYERS
+            st.lens[l].fill_(L)
+            sd.verify_layer(st.q[l], st.k[l], st.v[l], st.pos, SECTIONS, st.caches[l], 0, BASE,
+                            out=st.out[l], ws=st.ws_layer[l])
         elif args.only == "accept":
             st.accept_only()
         else:

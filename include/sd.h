@@ -166,6 +166,44 @@ sd_status sd_verify_attention(const void* q, const sd_kv_cache* cache, void* out
                               int R, int Hq, float scale, void* workspace, size_t ws_bytes,
                               sd_stream_t stream);
 
+/* sd_verify_layer flag: see below. */
+#define SD_LAYER_PREFIX_EARLY 1
+
+/*
+ * Workspace bytes sd_verify_layer needs on the CURRENT device for this shape.
+ */
+size_t sd_verify_layer_workspace(int B, int R, int Hq, int Hkv, int D, int capacity);
+
+/*
+ * One attention layer of the verify pass in one call (Eq. verify, Sec. 2.2):
+ * the M-RoPE rotation of the R new query and key rows (Sec. 2.3 Eq. rope-3d,
+ * Sec. 3.2 Eqs. axis-assign, mrope-phase), their append to the cache (Eq.
+ * commit) and the verify attention over the prefix plus the new rows.
+ * Equal to sd_rope_apply(q, k_new, ...) + sd_kv_append(cache, k_new, v_new)
+ * + sd_verify_attention(q, cache, out): q and k_new are rotated in place,
+ * rows len[b] .. len[b]+R-1 of the cache receive k_new / v_new, len[b] += R,
+ * and out receives the attention. Here len[b] on entry is the PREFIX length.
+ *   q [B][R][Hq][D], k_new / v_new [B][R][Hkv][D] bf16, pos [B][R][3] int32,
+ *   sections (host), interleaved, base: as for sd_rope_apply; scale as for
+ *   sd_verify_attention.
+ *   workspace: sd_verify_layer_workspace() bytes, zero-filled before first
+ *   use, left zeroed by every completed call; calls sharing it must not
+ *   overlap on the device -- calls flagged SD_LAYER_PREFIX_EARLY overlap
+ *   their predecessor, so give each layer its own workspace.
+ *   flags: SD_LAYER_PREFIX_EARLY declares that the kernel issued just before
+ *   this call on the stream writes neither this layer's cache nor its len
+ *   (true for every layer but the first of a verify pass, when the layers are
+ *   issued back to back). The call is then a programmatic dependent launch
+ *   that streams the cached prefix while its predecessor still runs.
+ * For head_dim 128 and G * R <= 32 this is one tcgen05 kernel; other shapes
+ * run the three kernels in sequence. A scene whose append would pass the
+ * capacity sets SD_DEVERR_KV_OVERFLOW and is left untouched.
+ */
+sd_status sd_verify_layer(void* q, void* k_new, const void* v_new, const int32_t* pos,
+                          const int32_t sections[3], int interleaved, float base,
+                          const sd_kv_cache* cache, void* out, int R, int Hq, float scale,
+                          void* workspace, size_t ws_bytes, int flags, sd_stream_t stream);
+
 /*
  * Workspace bytes sd_accept_greedy needs for (B, R = K + 1, V).
  */

@@ -51,8 +51,8 @@ constexpr uint32_t kSpinLimit = 1u << 20;
 constexpr int kOffQ = kRing;
 constexpr int kOffP = kOffQ + kQ;
 constexpr int kOffBar = kOffP + 2 * kP;
-// barriers: full[3] empty[3] s_full[2] s_free[2] p_full[2] o_done[2] q_full recv
-constexpr int kNumBars = 3 + 3 + 2 + 2 + 2 + 2 + 1 + 1;
+// barriers: full[3] empty[3] s_full[2] s_free[2] p_full[2] o_done[2] q_full recv append
+constexpr int kNumBars = 3 + 3 + 2 + 2 + 2 + 2 + 1 + 1 + 1;
 constexpr int kOffMisc = kOffBar + kNumBars * 8;
 // misc: tmem slot (4), grow flag (4), red[4][32] + 2 x 4 warp flags, mnew[32], corr[32]
 constexpr int kOffRed = kOffMisc + 16;
@@ -205,20 +205,43 @@ __device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32
 }
 
 struct TcArgs {
-  const __nv_bfloat16* q;
+  const __nv_bfloat16* q;   // rotated q rows (standalone attention)
   __nv_bfloat16* out;
-  const int32_t* len;
+  int32_t* len;
+  // fused verify layer only
+  __nv_bfloat16* qw;        // raw q rows, rotated in place
+  __nv_bfloat16* k_new;     // raw new key rows [B][R][Hkv][D], rotated in place
+  const __nv_bfloat16* v_new;
+  __nv_bfloat16* kc;        // cache K / V [B][Hkv][cap][D] (append target)
+  __nv_bfloat16* vc;
+  const int32_t* pos;       // [B][R][3]
+  uint32_t* ticket;         // [B] per-scene CTA tickets (zeroed, re-armed)
+  int early;                // the prefix may be streamed before the dependency wait
   int R, Hq, Hkv, G, M, cap, n_mblocks;
   float scale_log2;
 };
 
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void griddep_launch() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 // ------------------------------------------------------------------ kernel
+// kFused = false: attention over a cache that already holds the R new rows,
+// with the rotated query rows loaded by TMA.
+// kFused = true: the whole verify layer -- M-RoPE of the raw query and key
+// rows, the KV append and the attention -- with len[b] the prefix length.
+// Prefix tiles are independent of the kernel that precedes this one in the
+// stream (for every layer but the first of a step), so when a.early is set
+// they stream before the programmatic-dependency wait.
+template <bool kFused>
 __global__ void __launch_bounds__(kThreads, 1)
     verify_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k128,
                           const __grid_constant__ CUtensorMap tm_v128,
                           const __grid_constant__ CUtensorMap tm_k32,
                           const __grid_constant__ CUtensorMap tm_v32,
-                          const __grid_constant__ CUtensorMap tm_q, const TcArgs a) {
+                          const __grid_constant__ CUtensorMap tm_q, const TcArgs a,
+                          const RopeTable tab) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
@@ -234,6 +257,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   auto ODONE = [&](int b) { return bar(12 + b); };
   const uint32_t QFULL = bar(14);
   const uint32_t RECV = bar(15);  // the cluster merge's incoming partial rows
+  const uint32_t APPEND = bar(16);  // fused: the new K/V rows are in the cache
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + kOffMisc);
   int* grow_flag = reinterpret_cast<int*>(smem + kOffMisc + 4);
   float* red = reinterpret_cast<float*>(smem + kOffRed);    // [4][32]
@@ -259,8 +283,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(PFULL(i), 4);
       mbar_init(ODONE(i), 1);
     }
-    mbar_init(QFULL, 129);  // producer's expect_tx + 128 softmax threads
+    mbar_init(QFULL, kFused ? 128 : 129);  // (producer's expect_tx +) 128 softmax threads
     mbar_init(RECV, 1);
+    mbar_init(APPEND, 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (warp == 1) {
@@ -277,29 +302,57 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem_s = tmem;          // S buffer b at column 32 * b
   const uint32_t tmem_o = tmem + 64;     // O^T
 
-  const int n_keys = a.len[b];
-  const bool valid = n_keys >= a.R && n_keys <= a.cap;
-  if (!valid && rank == 0 && threadIdx.x == 0 && blockIdx.y == 0) sd_set_error(SD_DEVERR_LENGTH);
+  if (kFused && !a.early) griddep_wait();  // len and the prefix may come from the previous kernel
+  int n_keys, L_pre;
+  bool valid;
+  if (kFused) {
+    L_pre = a.len[b];
+    n_keys = L_pre + a.R;
+    valid = L_pre >= 0 && n_keys <= a.cap;
+    if (!valid && rank == 0 && threadIdx.x == 0 && blockIdx.y == 0)
+      sd_set_error(L_pre < 0 ? SD_DEVERR_LENGTH : SD_DEVERR_KV_OVERFLOW);
+  } else {
+    n_keys = a.len[b];
+    valid = n_keys >= a.R && n_keys <= a.cap;
+    L_pre = n_keys - a.R;
+    if (!valid && rank == 0 && threadIdx.x == 0 && blockIdx.y == 0) sd_set_error(SD_DEVERR_LENGTH);
+  }
   const int nblk = valid ? (n_keys + 31) / 32 : 0;
-  const int blk_begin = static_cast<int>((static_cast<long long>(rank) * nblk) / csize);
-  const int blk_end = static_cast<int>((static_cast<long long>(rank + 1) * nblk) / csize);
+  int blk_begin, blk_end;
+  if (kFused) {
+    // blocks wholly inside the prefix split evenly; the last CTA also takes
+    // the block(s) holding the new rows, which it appends itself
+    const int blk_new0 = valid ? L_pre / 32 : 0;
+    blk_begin = static_cast<int>((static_cast<long long>(rank) * blk_new0) / csize);
+    blk_end = rank == csize - 1 ? nblk
+                                : static_cast<int>((static_cast<long long>(rank + 1) * blk_new0) / csize);
+  } else {
+    blk_begin = static_cast<int>((static_cast<long long>(rank) * nblk) / csize);
+    blk_end = static_cast<int>((static_cast<long long>(rank + 1) * nblk) / csize);
+  }
   const int key_begin = blk_begin * 32;
   const int key_end = min(blk_end * 32, n_keys);
   const int n_tiles = (blk_end - blk_begin + 3) / 4;
+  const bool owns_new = kFused && valid && rank == csize - 1;
+  const int t_new = owns_new ? (L_pre / 32 - blk_begin) / 4 : n_tiles;  // first tile with new rows
 
   if (warp == 0) {
     // -------------------------------------------------------------- producer
     if (lane == 0 && n_tiles > 0) {
-      // the packed query tile first: box (64 d, G heads, R rows) lands as
-      // rows p = i * G + g of 128 bytes, the B operand's K-major layout
-      mbar_expect_tx(QFULL, static_cast<uint32_t>(2 * a.M * 128));
-      for (int h = 0; h < 2; ++h) tma_load_3d(qs + h * kQHalf, &tm_q, QFULL, h * 64, kvh * a.G, b * a.R);
+      if (!kFused) {
+        // the packed query tile first: box (64 d, G heads, R rows) lands as
+        // rows p = i * G + g of 128 bytes, the B operand's K-major layout
+        mbar_expect_tx(QFULL, static_cast<uint32_t>(2 * a.M * 128));
+        for (int h = 0; h < 2; ++h)
+          tma_load_3d(qs + h * kQHalf, &tm_q, QFULL, h * 64, kvh * a.G, b * a.R);
+      }
       asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_k128)) : "memory");
       asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_v128)) : "memory");
       const int z = b * a.Hkv + kvh;
       for (int t = 0; t < n_tiles; ++t) {
         const int s = t % kStages;
         if (t >= kStages) mbar_wait(EMPTY(s), ((t / kStages) - 1) & 1);
+        if (kFused && t == t_new) mbar_wait(APPEND, 0);  // the new rows are in the cache
         const int nb = min(4, blk_end - blk_begin - 4 * t);
         const int y0 = key_begin + t * kStageKeys;
         const uint32_t kst = base + s * kStage, vst = kst + kKV;
@@ -366,15 +419,64 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int quarter = warp & 3;          // TMEM lane quarter of this warp
     const int kl = quarter * 32 + lane;    // key lane of S^T / d lane of O^T
     const uint32_t lane_off = static_cast<uint32_t>(quarter * 32) << 16;
-    // query rows past M stay zero (the TMA box covers rows 0..M-1 only)
-    for (int idx = st; idx < (kRows - a.M) * 16; idx += 128) {
-      const int row = a.M + idx / 16, c = idx % 16;
-      asm volatile("st.shared.v4.u32 [%0], {%1,%1,%1,%1};" ::"r"(qs + (c >> 3) * kQHalf + row * 128 + (c & 7) * 16),
-                   "r"(0)
-                   : "memory");
+    if (!kFused) {
+      // query rows past M stay zero (the TMA box covers rows 0..M-1 only)
+      for (int idx = st; idx < (kRows - a.M) * 16; idx += 128) {
+        const int row = a.M + idx / 16, c = idx % 16;
+        asm volatile("st.shared.v4.u32 [%0], {%1,%1,%1,%1};" ::"r"(qs + (c >> 3) * kQHalf + row * 128 + (c & 7) * 16),
+                     "r"(0)
+                     : "memory");
+      }
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      mbar_arrive(QFULL);
+    } else {
+      // the raw rows come from earlier kernels; once they are visible every
+      // older kernel has finished, so the next layer may launch
+      griddep_wait();
+      if (st == 0) griddep_launch();
+      // M-RoPE of the packed query rows, straight into the swizzled tile
+      for (int idx = st; idx < kRows * 16; idx += 128) {
+        const int row = idx / 16, c = idx % 16;
+        const int p = mblock * kRows + row;
+        uint32_t w[4] = {0u, 0u, 0u, 0u};
+        if (valid && p < a.M) {
+          const int i = p / a.G, gq = p % a.G;
+          const uint4 v = *reinterpret_cast<const uint4*>(
+              a.qw + ((static_cast<long long>(b) * a.R + i) * a.Hq + kvh * a.G + gq) * kD + c * 8);
+          w[0] = v.x; w[1] = v.y; w[2] = v.z; w[3] = v.w;
+          const int32_t* pp = a.pos + (static_cast<long long>(b) * a.R + i) * 3;
+          const int p3[3] = {pp[0], pp[1], pp[2]};
+          sd_rope_rotate8(w, c, p3, tab);
+        }
+        asm volatile("st.shared.v4.u32 [%0], {%1,%2,%3,%4};" ::"r"(
+                         qs + (c >> 3) * kQHalf + row * 128 + (((c & 7) ^ (row & 7)) << 4)),
+                     "r"(w[0]), "r"(w[1]), "r"(w[2]), "r"(w[3])
+                     : "memory");
+      }
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      mbar_arrive(QFULL);
+      if (owns_new) {
+        // M-RoPE of this head's new key rows and the append of K and V; the
+        // rotated keys also go back to k_new, like the standalone rotation
+        for (int idx = st; idx < a.R * 16; idx += 128) {
+          const int i = idx / 16, c = idx % 16;
+          const long long src = ((static_cast<long long>(b) * a.R + i) * a.Hkv + kvh) * kD + c * 8;
+          const long long dst = ((static_cast<long long>(b) * a.Hkv + kvh) * a.cap + L_pre + i) * kD + c * 8;
+          const uint4 kv = *reinterpret_cast<const uint4*>(a.k_new + src);
+          uint32_t w[4] = {kv.x, kv.y, kv.z, kv.w};
+          const int32_t* pp = a.pos + (static_cast<long long>(b) * a.R + i) * 3;
+          const int p3[3] = {pp[0], pp[1], pp[2]};
+          sd_rope_rotate8(w, c, p3, tab);
+          const uint4 kr = make_uint4(w[0], w[1], w[2], w[3]);
+          *reinterpret_cast<uint4*>(a.kc + dst) = kr;
+          *reinterpret_cast<uint4*>(a.k_new + src) = kr;
+          *reinterpret_cast<uint4*>(a.vc + dst) = *reinterpret_cast<const uint4*>(a.v_new + src);
+        }
+        asm volatile("fence.proxy.async.global;" ::: "memory");  // visible to the TMA loads
+        named_bar_sync(2, 128);
+        if (st == 0) mbar_arrive(APPEND);
+      }
     }
-    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-    mbar_arrive(QFULL);
 
     const int L_prefix = n_keys - a.R;
     const float sl = a.scale_log2;
@@ -586,8 +688,31 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
   }
+  if (kFused && rank == 0 && warp >= 2) {
+    // every CTA of the cluster read the raw query rows before its main loop
+    // (the cluster barrier above is behind all of them): store the rotated rows
+    for (int idx = threadIdx.x - 64; idx < a.M * 16 && valid; idx += 128) {
+      const int row = idx / 16, c = idx % 16;
+      const int p = mblock * kRows + row;
+      if (p >= a.M) continue;
+      const int i = p / a.G, gq = p % a.G;
+      const uint4 v = *reinterpret_cast<const uint4*>(smem + kOffQ + (c >> 3) * kQHalf + row * 128 +
+                                                      (((c & 7) ^ (row & 7)) << 4));
+      *reinterpret_cast<uint4*>(a.qw + ((static_cast<long long>(b) * a.R + i) * a.Hq + kvh * a.G + gq) * kD +
+                                c * 8) = v;
+    }
+  }
   tc_fence_before();
   __syncthreads();  // every tensor-memory read is done
+  if (kFused && threadIdx.x == 0) {
+    // the last CTA of the scene to finish advances its length: every CTA of
+    // the scene read len[b] before it got here
+    const uint32_t total = gridDim.x * gridDim.y;
+    if (atomicAdd(&a.ticket[b], 1u) == total - 1) {
+      if (valid) a.len[b] = L_pre + a.R;
+      a.ticket[b] = 0;
+    }
+  }
   if (warp == 1) {
     tc_fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
@@ -662,10 +787,15 @@ DevState* state() {
   DevState& s = st[dev];
   if (!s.ready) {
     s.ready = true;
-    auto kern = verify_attn_tc_kernel;
+    auto kern = verify_attn_tc_kernel<false>;
+    auto kern_f = verify_attn_tc_kernel<true>;
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes) !=
             cudaSuccess ||
         cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
+            cudaSuccess ||
+        cudaFuncSetAttribute(kern_f, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes) !=
+            cudaSuccess ||
+        cudaFuncSetAttribute(kern_f, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
             cudaSuccess) {
       (void)cudaGetLastError();
       return &s;
@@ -726,12 +856,49 @@ static bool tc_enabled() {
   return on;
 }
 
+static int serving_cluster(int B, int R, int Hq, int Hkv, int D, int cap);
+
 bool sd_internal_tc_serves(int B, int R, int Hq, int Hkv, int D, int cap) {
-  if (!tc_enabled() || D != kD || Hkv <= 0 || Hq % Hkv) return false;
-  if ((Hq / Hkv) * R > kRows) return false;
+  return serving_cluster(B, R, Hq, Hkv, D, cap) > 0;
+}
+
+template <bool kFused>
+static sd_status launch_tc(const sd_kv_cache* cache, const void* q_for_map, const TcArgs& a,
+                    const RopeTable& tab, int cs, bool pdl, cudaStream_t stream) {
+  const int B = cache->batch, Hkv = cache->n_kv_heads, cap = cache->capacity;
+  CUtensorMap k128, v128, k32, v32, qm;
+  if (!make_map(&k128, cache->k, cap, B * Hkv, 128) || !make_map(&v128, cache->v, cap, B * Hkv, 128) ||
+      !make_map(&k32, cache->k, cap, B * Hkv, 32) || !make_map(&v32, cache->v, cap, B * Hkv, 32) ||
+      !make_q_map(&qm, q_for_map, B, a.R, a.Hq, a.G))
+    return SD_ERR_CUDA;
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = cs;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  cfg.gridDim = dim3(cs, Hkv, B);
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.dynamicSmemBytes = kSmemBytes;
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 2 : 1;
+  if (cudaLaunchKernelEx(&cfg, verify_attn_tc_kernel<kFused>, k128, v128, k32, v32, qm, a, tab) !=
+      cudaSuccess) {
+    (void)cudaGetLastError();
+    return SD_ERR_CUDA;
+  }
+  return SD_OK;
+}
+
+static int serving_cluster(int B, int R, int Hq, int Hkv, int D, int cap) {
+  if (!tc_enabled() || D != kD || Hkv <= 0 || Hq % Hkv) return 0;
+  if ((Hq / Hkv) * R > kRows) return 0;
   DevState* s = state();
-  if (!s || !s->ok) return false;
-  return pick_cluster(*s, static_cast<long long>(B) * Hkv, cap) > 0;
+  if (!s || !s->ok) return 0;
+  return pick_cluster(*s, static_cast<long long>(B) * Hkv, cap);
 }
 
 // Routed here by sd_verify_attention for head_dim 128 and G * R <= 32.
@@ -739,49 +906,55 @@ sd_status sd_internal_verify_attention_tc(const void* q, const sd_kv_cache* cach
                                           int R, int Hq, float scale_log2, cudaStream_t stream,
                                           bool* handled) {
   *handled = false;
-  const int B = cache->batch, Hkv = cache->n_kv_heads, cap = cache->capacity;
-  if (!tc_enabled() || cache->head_dim != kD) return SD_OK;
-  const int G = Hq / Hkv;
-  const int M = G * R;
-  if (M > kRows) return SD_OK;
-  DevState* s = state();
-  if (!s || !s->ok) return SD_OK;
-  const long long units = static_cast<long long>(B) * Hkv;
-  const int cs = pick_cluster(*s, units, cap);
+  const int B = cache->batch, Hkv = cache->n_kv_heads;
+  const int cs = serving_cluster(B, R, Hq, Hkv, cache->head_dim, cache->capacity);
   if (cs <= 0) return SD_OK;
-  CUtensorMap k128, v128, k32, v32, qm;
-  if (!make_map(&k128, cache->k, cap, B * Hkv, 128) || !make_map(&v128, cache->v, cap, B * Hkv, 128) ||
-      !make_map(&k32, cache->k, cap, B * Hkv, 32) || !make_map(&v32, cache->v, cap, B * Hkv, 32) ||
-      !make_q_map(&qm, q, B, R, Hq, G))
-    return SD_ERR_CUDA;
-  TcArgs a;
+  TcArgs a = {};
   a.q = static_cast<const __nv_bfloat16*>(q);
   a.out = static_cast<__nv_bfloat16*>(out);
   a.len = cache->len;
   a.R = R;
   a.Hq = Hq;
   a.Hkv = Hkv;
-  a.G = G;
-  a.M = M;
-  a.cap = cap;
+  a.G = Hq / Hkv;
+  a.M = a.G * R;
+  a.cap = cache->capacity;
   a.n_mblocks = 1;
   a.scale_log2 = scale_log2;
-  cudaLaunchConfig_t cfg = {};
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = cs;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
-  cfg.gridDim = dim3(cs, Hkv, B);
-  cfg.blockDim = dim3(kThreads, 1, 1);
-  cfg.dynamicSmemBytes = kSmemBytes;
-  cfg.stream = stream;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  RopeTable tab = {};
   *handled = true;
-  if (cudaLaunchKernelEx(&cfg, verify_attn_tc_kernel, k128, v128, k32, v32, qm, a) != cudaSuccess) {
-    (void)cudaGetLastError();
-    return SD_ERR_CUDA;
-  }
-  return SD_OK;
+  return launch_tc<false>(cache, q, a, tab, cs, false, stream);
+}
+
+// The fused verify layer (rope + append + attention) on the tcgen05 path.
+sd_status sd_internal_verify_layer_tc(void* q, void* k_new, const void* v_new, const int32_t* pos,
+                                      const RopeTable& tab, const sd_kv_cache* cache, void* out,
+                                      int R, int Hq, float scale_log2, uint32_t* ticket, int early,
+                                      cudaStream_t stream, bool* handled) {
+  *handled = false;
+  const int B = cache->batch, Hkv = cache->n_kv_heads;
+  const int cs = serving_cluster(B, R, Hq, Hkv, cache->head_dim, cache->capacity);
+  if (cs <= 0) return SD_OK;
+  TcArgs a = {};
+  a.q = static_cast<const __nv_bfloat16*>(q);
+  a.out = static_cast<__nv_bfloat16*>(out);
+  a.len = cache->len;
+  a.qw = static_cast<__nv_bfloat16*>(q);
+  a.k_new = static_cast<__nv_bfloat16*>(k_new);
+  a.v_new = static_cast<const __nv_bfloat16*>(v_new);
+  a.kc = static_cast<__nv_bfloat16*>(cache->k);
+  a.vc = static_cast<__nv_bfloat16*>(cache->v);
+  a.pos = pos;
+  a.ticket = ticket;
+  a.early = early ? 1 : 0;
+  a.R = R;
+  a.Hq = Hq;
+  a.Hkv = Hkv;
+  a.G = Hq / Hkv;
+  a.M = a.G * R;
+  a.cap = cache->capacity;
+  a.n_mblocks = 1;
+  a.scale_log2 = scale_log2;
+  *handled = true;
+  return launch_tc<true>(cache, q, a, tab, cs, early != 0, stream);
 }

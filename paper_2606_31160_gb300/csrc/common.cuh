@@ -44,6 +44,14 @@ sd_status sd_internal_verify_attention_tc(const void* q, const sd_kv_cache* cach
 // Whether the tcgen05 path serves this shape on the current device.
 bool sd_internal_tc_serves(int B, int R, int Hq, int Hkv, int D, int cap);
 
+struct RopeTable;
+// The fused verify layer on the tcgen05 path (attention_tc.cu); *handled is
+// set when the shape is served and the kernel launched.
+sd_status sd_internal_verify_layer_tc(void* q, void* k_new, const void* v_new, const int32_t* pos,
+                                      const RopeTable& tab, const sd_kv_cache* cache, void* out,
+                                      int R, int Hq, float scale_log2, uint32_t* ticket, int early,
+                                      cudaStream_t stream, bool* handled);
+
 // ---------------------------------------------------------------------------
 // Host helpers
 // ---------------------------------------------------------------------------
@@ -76,8 +84,59 @@ static inline int sd_num_sms() {
 __device__ __forceinline__ float sd_bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float sd_bf16_hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
 
+// ---------------------------------------------------------------------------
+// RoPE (Sec. 2.3 Eq. rope-1d, Sec. 3.2 Eqs. axis-assign, mrope-phase) shared by
+// the standalone rotation kernel and the fused verify-layer kernel, so both
+// produce identical bits. The angle theta_d * p is carried in TURNS:
+// tau_d = theta_d / (2 pi) as an fp32 hi/lo pair; p * tau_d is formed with an
+// exact fma split, whole turns are dropped (an exact subtraction) and
+// sincospif evaluates the remaining fraction, so the reduced angle is
+// accurate to ~1e-7 rad for any |p| < 2^24.
+// ---------------------------------------------------------------------------
+constexpr int kRopeMaxPairs = 64;  // D <= 128
+
+struct RopeTable {
+  float tau_hi[kRopeMaxPairs];  // fp32 part of theta_d / (2 pi)
+  float tau_lo[kRopeMaxPairs];  // remainder theta_d / (2 pi) - tau_hi
+  int8_t axis[kRopeMaxPairs];   // a(d) in {0 = T, 1 = H, 2 = W}
+};
+
+// Fills the table for head dim D; sections == nullptr gives the 1-D table.
+// Returns false for sections that do not sum to D / 2.
+bool sd_internal_rope_table(int D, const int32_t* sections, int interleaved, float base,
+                            RopeTable* tab);
+
+// Fractional turns of p * tau, in [-0.5, 0.5] up to rounding.
+__device__ __forceinline__ float sd_frac_turns(float p, float hi, float lo) {
+  const float a = p * hi;          // rounded product
+  const float e = fmaf(p, hi, -a); // its exact rounding error
+  const float f = a - rintf(a);    // exact: whole turns removed
+  return f + fmaf(p, lo, e);
+}
+
+// Rotate 4 adjacent pairs (8 bf16 packed in w[4]) of head-vector chunk `vec`
+// (pairs 4*vec .. 4*vec+3) at coordinates p3 (t, h, w).
+__device__ __forceinline__ void sd_rope_rotate8(uint32_t (&w)[4], int vec, const int (&p3)[3],
+                                                const RopeTable& tab);
+
 // Two floats -> packed bf16x2 (round to nearest even), lo in the low half.
 __device__ __forceinline__ uint32_t sd_pack_bf16x2(float lo, float hi) {
   __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<uint32_t*>(&v);
+}
+
+__device__ __forceinline__ void sd_rope_rotate8(uint32_t (&w)[4], int vec, const int (&p3)[3],
+                                                const RopeTable& tab) {
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    const int d = vec * 4 + j;
+    const float p = static_cast<float>(p3[tab.axis[d]]);
+    float s, c;
+    sincospif(2.0f * sd_frac_turns(p, tab.tau_hi[d], tab.tau_lo[d]), &s, &c);
+    const float x = sd_bf16_lo(w[j]);
+    const float y = sd_bf16_hi(w[j]);
+    const float xr = fmaf(x, c, -y * s);
+    const float yr = fmaf(x, s, y * c);
+    w[j] = sd_pack_bf16x2(xr, yr);
+  }
 }

@@ -10,13 +10,9 @@
 // one head row; the whole launch is a few thousand threads and is bound by
 // launch latency, not bandwidth.
 //
-// Angle precision. theta_d * p reaches ~1.6e4 rad at the positions of the
-// longest workloads, where an fp32 product alone is off by ~1e-3 rad. The
-// angle is instead carried in TURNS: the host gives tau_d = theta_d / (2 pi)
-// as an fp32 hi/lo pair; the device forms p * tau_d with an exact fma split,
-// drops the whole turns (an exact subtraction) and evaluates
-// sincospif(2 * frac), so the reduced angle is accurate to ~1e-7 rad for any
-// |p| < 2^24.
+// Angle precision: theta_d * p reaches ~1.6e4 rad at the positions of the
+// longest workloads, where an fp32 product alone is off by ~1e-3 rad; the
+// turn-based reduction in common.cuh keeps it at ~1e-7 rad.
 #include "common.cuh"
 
 #include <math.h>
@@ -24,22 +20,6 @@
 SD_DEFINE_ERROR_ACCESSOR(sd_take_error_rope)
 
 namespace {
-
-constexpr int kMaxPairs = 64;  // D <= 128
-
-struct RopeTable {
-  float tau_hi[kMaxPairs];   // fp32 part of theta_d / (2 pi)
-  float tau_lo[kMaxPairs];   // remainder theta_d / (2 pi) - tau_hi
-  int8_t axis[kMaxPairs];    // a(d) in {0 = T, 1 = H, 2 = W}
-};
-
-// Fractional turns of p * tau, in [-0.5, 0.5] up to rounding.
-__device__ __forceinline__ float frac_turns(float p, float hi, float lo) {
-  float a = p * hi;                 // rounded product
-  float e = fmaf(p, hi, -a);        // its exact rounding error
-  float f = a - rintf(a);           // exact: whole turns removed
-  return f + fmaf(p, lo, e);
-}
 
 // One thread: 8 consecutive elements (4 pairs) of one head row.
 template <int D, bool kFlat>
@@ -60,8 +40,8 @@ __global__ void __launch_bounds__(256) rope_kernel(__nv_bfloat16* __restrict__ q
     __nv_bfloat16* base = head < hq ? q + ((row * hq + head) * D)
                                     : k + ((row * hkv + (head - hq)) * D);
     uint4* ptr = reinterpret_cast<uint4*>(base) + vec;
-    uint4 w = *ptr;
-    uint32_t words[4] = {w.x, w.y, w.z, w.w};
+    const uint4 v = *ptr;
+    uint32_t words[4] = {v.x, v.y, v.z, v.w};
     int p3[3];
     if (kFlat) {
       p3[0] = p3[1] = p3[2] = pos[row];
@@ -70,48 +50,9 @@ __global__ void __launch_bounds__(256) rope_kernel(__nv_bfloat16* __restrict__ q
       p3[1] = pos[row * 3 + 1];
       p3[2] = pos[row * 3 + 2];
     }
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const int d = vec * 4 + j;
-      const float p = (float)p3[tab.axis[d]];
-      float s, c;
-      sincospif(2.0f * frac_turns(p, tab.tau_hi[d], tab.tau_lo[d]), &s, &c);
-      const float x = sd_bf16_lo(words[j]);
-      const float y = sd_bf16_hi(words[j]);
-      const float xr = fmaf(x, c, -y * s);
-      const float yr = fmaf(x, s, y * c);
-      words[j] = sd_pack_bf16x2(xr, yr);
-    }
+    sd_rope_rotate8(words, vec, p3, tab);
     *ptr = make_uint4(words[0], words[1], words[2], words[3]);
   }
-}
-
-bool build_table(int D, const int32_t* sections, int interleaved, float base, RopeTable* tab) {
-  const int pairs = D / 2;
-  if (sections) {
-    if (sections[0] < 0 || sections[1] < 0 || sections[2] < 0) return false;
-    if (sections[0] + sections[1] + sections[2] != pairs) return false;
-  }
-  const double two_pi = 6.283185307179586476925286766559;
-  for (int d = 0; d < pairs; ++d) {
-    const double theta = pow((double)base, -2.0 * d / (double)D);
-    const double tau = theta / two_pi;
-    tab->tau_hi[d] = (float)tau;
-    tab->tau_lo[d] = (float)(tau - (double)tab->tau_hi[d]);
-    int a = 0;
-    if (sections) {
-      if (interleaved) a = d % 3;
-      else if (d < sections[0]) a = 0;
-      else if (d < sections[0] + sections[1]) a = 1;
-      else a = 2;
-    }
-    tab->axis[d] = (int8_t)a;
-  }
-  for (int d = pairs; d < kMaxPairs; ++d) {
-    tab->tau_hi[d] = tab->tau_lo[d] = 0.f;
-    tab->axis[d] = 0;
-  }
-  return true;
 }
 
 sd_status launch(void* q, void* k, int B, int R, int Hq, int Hkv, int D, const int32_t* pos,
@@ -127,7 +68,8 @@ sd_status launch(void* q, void* k, int B, int R, int Hq, int Hkv, int D, const i
   if (!pos) return SD_ERR_INVALID_ARG;
   if (!flat && !sections) return SD_ERR_INVALID_ARG;
   RopeTable tab;
-  if (!build_table(D, flat ? nullptr : sections, interleaved, base, &tab)) return SD_ERR_INVALID_ARG;
+  if (!sd_internal_rope_table(D, flat ? nullptr : sections, interleaved, base, &tab))
+    return SD_ERR_INVALID_ARG;
   const long long total = rows * (Hq + Hkv) * (D / 8);
   const int threads = 256;
   long long blocks = (total + threads - 1) / threads;
@@ -147,6 +89,36 @@ sd_status launch(void* q, void* k, int B, int R, int Hq, int Hkv, int D, const i
 }
 
 }  // namespace
+
+bool sd_internal_rope_table(int D, const int32_t* sections, int interleaved, float base,
+                            RopeTable* tab) {
+  const int pairs = D / 2;
+  if (pairs > kRopeMaxPairs) return false;
+  if (sections) {
+    if (sections[0] < 0 || sections[1] < 0 || sections[2] < 0) return false;
+    if (sections[0] + sections[1] + sections[2] != pairs) return false;
+  }
+  const double two_pi = 6.283185307179586476925286766559;
+  for (int d = 0; d < pairs; ++d) {
+    const double theta = pow((double)base, -2.0 * d / (double)D);
+    const double tau = theta / two_pi;
+    tab->tau_hi[d] = (float)tau;
+    tab->tau_lo[d] = (float)(tau - (double)tab->tau_hi[d]);
+    int a = 0;
+    if (sections) {
+      if (interleaved) a = d % 3;
+      else if (d < sections[0]) a = 0;
+      else if (d < sections[0] + sections[1]) a = 1;
+      else a = 2;
+    }
+    tab->axis[d] = (int8_t)a;
+  }
+  for (int d = pairs; d < kRopeMaxPairs; ++d) {
+    tab->tau_hi[d] = tab->tau_lo[d] = 0.f;
+    tab->axis[d] = 0;
+  }
+  return true;
+}
 
 extern "C" sd_status sd_rope_apply(void* q, void* k, int B, int R, int Hq, int Hkv, int D,
                                    const int32_t* pos, const int32_t sections[3],

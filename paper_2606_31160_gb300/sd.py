@@ -49,6 +49,9 @@ _SIGNATURES = {
     "sd_kv_rollback": ([_vp, _i, _i, _vp, _i, _vp], _i),
     "sd_verify_attention_workspace": ([_i, _i, _i, _i, _i, _i], _sz),
     "sd_verify_attention": ([_vp, ctypes.POINTER(KVCacheStruct), _vp, _i, _i, _f, _vp, _sz, _vp], _i),
+    "sd_verify_layer_workspace": ([_i, _i, _i, _i, _i, _i], _sz),
+    "sd_verify_layer": ([_vp, _vp, _vp, _vp, ctypes.POINTER(ctypes.c_int32), _i, _f,
+                         ctypes.POINTER(KVCacheStruct), _vp, _i, _i, _f, _vp, _sz, _i, _vp], _i),
     "sd_accept_greedy_workspace": ([_i, _i, _i], _sz),
     "sd_accept_greedy": ([_vp, _i, _i, _i, _i, _vp, _vp, _vp, _vp, _vp, _sz, _vp], _i),
     "sd_accept_greedy_noalloc": ([_vp, _i, _i, _i, _i, _vp, _vp, _vp, _vp, _vp], _i),
@@ -221,6 +224,44 @@ def verify_attention(q, cache, out=None, scale=0.0, ws=None):
     _check(lib().sd_verify_attention(_dev(q, "q", torch.bfloat16), cache.struct,
                                      _dev(out, "out", torch.bfloat16), R, Hq, float(scale), wp, nbytes,
                                      _stream()), "sd_verify_attention")
+    return out
+
+
+SD_LAYER_PREFIX_EARLY = 1
+
+
+def layer_workspace_bytes(B, R, Hq, Hkv, D, capacity):
+    return int(lib().sd_verify_layer_workspace(B, R, Hq, Hkv, D, capacity))
+
+
+def verify_layer(q, k_new, v_new, pos, sections, cache, interleaved=0, base=1e6, out=None, scale=0.0,
+                 ws=None, early=False):
+    """sd_verify_layer: M-RoPE of q / k_new (in place), append of k_new / v_new at
+    len[b] (the prefix length on entry; len += R) and the verify attention; returns out.
+    early=True sets SD_LAYER_PREFIX_EARLY (the previous kernel on the stream writes
+    neither this layer's cache nor its len)."""
+    B, R, Hq, D = q.shape
+    Hkv = k_new.shape[2]
+    if tuple(k_new.shape) != (B, R, Hkv, D) or k_new.shape != v_new.shape or tuple(pos.shape) != (B, R, 3):
+        raise ValueError("shape mismatch")
+    if cache.shape[0] != B or cache.shape[1] != Hkv or cache.shape[3] != D:
+        raise ValueError("q and cache disagree")
+    if out is None:
+        out = torch.empty_like(q)
+    if ws is None:
+        # one workspace per layer cache: calls with early=True overlap the
+        # previous layer's kernel, so layers must not share their tickets
+        need = layer_workspace_bytes(B, R, Hq, Hkv, D, cache.shape[2])
+        ws = getattr(cache, "_layer_ws", None)
+        if ws is None or ws.numel() < need:
+            ws = workspace(need, q.device)
+            cache._layer_ws = ws
+    sec = (ctypes.c_int32 * 3)(*[int(x) for x in sections])
+    _check(lib().sd_verify_layer(_dev(q, "q", torch.bfloat16), _dev(k_new, "k_new", torch.bfloat16),
+                                 _dev(v_new, "v_new", torch.bfloat16), _dev(pos, "pos", torch.int32), sec,
+                                 int(interleaved), float(base), cache.struct, _dev(out, "out", torch.bfloat16),
+                                 R, Hq, float(scale), _dev(ws, "ws"), ws.numel() * ws.element_size(),
+                                 SD_LAYER_PREFIX_EARLY if early else 0, _stream()), "sd_verify_layer")
     return out
 
 

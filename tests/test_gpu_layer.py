@@ -1,0 +1,104 @@
+"""The fused verify layer (sd_verify_layer: M-RoPE + append + attention in one
+call) against the three separate calls and against the float64 oracle,
+including back-to-back layers issued as programmatic dependent launches."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2606_31160_gb300 import sd, workloads
+from tests.helpers import ATTN_ATOL, ensure_lib, gpu_case, pair_magnitude, rope_bound, to64
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    ensure_lib()
+
+
+def _unfused(case):
+    q, k_new, v_new, pos, cache = gpu_case(case)
+    sd.rope_apply(q, k_new, pos, case.sections, case.interleaved, case.base)
+    sd.kv_append(cache, k_new, v_new)
+    out = sd.verify_attention(q, cache)
+    torch.cuda.synchronize()
+    return q, k_new, cache, out
+
+
+def _fused(case, early=False):
+    q, k_new, v_new, pos, cache = gpu_case(case)
+    out = sd.verify_layer(q, k_new, v_new, pos, case.sections, cache, case.interleaved, case.base,
+                          early=early)
+    torch.cuda.synchronize()
+    return q, k_new, cache, out
+
+
+def _check_against_oracle(case, q, cache, out):
+    pos = case.pos.numpy()[:, :, None, :]
+    ref_q = oracle.mrope_apply(to64(case.q), pos, case.sections, case.interleaved, case.base)
+    assert np.all(np.abs(to64(q) - ref_q) <= rope_bound(ref_q, pair_magnitude(to64(case.q))))
+    ref_o = oracle.verify_attention(to64(q), to64(cache.k), to64(cache.v), cache.len.cpu().numpy())
+    err = np.abs(to64(out) - ref_o).max()
+    assert np.isfinite(to64(out)).all() and err <= ATTN_ATOL, err
+
+
+@pytest.mark.parametrize("make", [workloads.target_layer, workloads.tiny])
+def test_fused_equals_separate_calls(make):
+    case = make()
+    qa, ka, ca, oa = _unfused(case)
+    qb, kb, cb, ob = _fused(case)
+    assert torch.equal(qa, qb) and torch.equal(ka, kb)            # identical rotations
+    assert torch.equal(ca.k, cb.k) and torch.equal(ca.v, cb.v)    # identical appends
+    assert torch.equal(ca.len, cb.len)
+    _check_against_oracle(case, qb, cb, ob)
+    assert (ob.float() - oa.float()).abs().max().item() <= 2 * ATTN_ATOL
+    assert sd.get_device_error() == 0
+
+
+@pytest.mark.parametrize("prefix", [[0, 31, 32], [33, 4095, 64], [5, 127, 128]])
+def test_fused_ragged_batch(prefix):
+    B = len(prefix)
+    R = 8
+    qpos = np.stack([workloads.text_positions(int(p) + 1, R) for p in prefix])
+    case = workloads.verify_case(workloads.TARGET_LAYER, B=B, Hq=32, Hkv=8, D=128, prefix=prefix, K=R - 1,
+                                 sections=(16, 24, 24), base=1e6, query_pos=qpos, cap=max(prefix) + R + 40,
+                                 layer=77, tail_fill=float("nan"))
+    q, _, cache, out = _fused(case)
+    assert cache.len.cpu().tolist() == [p + R for p in prefix]
+    _check_against_oracle(case, q, cache, out)
+    assert sd.get_device_error() == 0
+
+
+def test_back_to_back_layers_with_early_prefix():
+    # a stack of layers issued back to back: every layer after the first may
+    # start streaming its prefix while the previous one runs
+    cases = [workloads.target_layer(layer=l) for l in range(6)]
+    runs = []
+    for early in (False, True):
+        outs = []
+        state = [gpu_case(c) for c in cases]
+        for l, (q, k_new, v_new, pos, cache) in enumerate(state):
+            outs.append(sd.verify_layer(q, k_new, v_new, pos, cases[l].sections, cache, 0, 1e6,
+                                        early=early and l > 0))
+        torch.cuda.synchronize()
+        runs.append((outs, state))
+    for (oa, sa), (ob, sb) in [(runs[0], runs[1])]:
+        for l in range(len(cases)):
+            assert torch.equal(oa[l], ob[l])
+            assert torch.equal(sa[l][4].k, sb[l][4].k) and torch.equal(sa[l][4].len, sb[l][4].len)
+    q, _, _, _, cache = runs[1][1][3]
+    _check_against_oracle(cases[3], q, cache, runs[1][0][3])
+    assert sd.get_device_error() == 0
+
+
+def test_fused_overflow_sets_error_and_leaves_scene():
+    case = workloads.target_layer()
+    q, k_new, v_new, pos, cache = gpu_case(case)
+    cache.len.fill_(case.cap - 3)            # R = 8 rows do not fit
+    out = torch.full_like(q, 5.0)
+    sd.get_device_error()
+    sd.verify_layer(q, k_new, v_new, pos, case.sections, cache, 0, 1e6, out=out)
+    assert sd.get_device_error() & sd.SD_DEVERR_KV_OVERFLOW
+    assert cache.len.item() == case.cap - 3
+    assert torch.all(out == 5.0)
