@@ -1,25 +1,43 @@
 // K3 on the 5th-generation tensor cores (tcgen05 + TMEM): verify attention
 // of the K + 1 new rows against the cached prefix (Eq. verify, Sec. 2.2),
-// for head_dim 128 and up to 32 packed query rows per KV head.
+// for head_dim 128 and up to 32 packed query rows per KV head, and the fused
+// verify layer (M-RoPE of Sec. 2.3 / Sec. 3.2 + the KV append of Eq. commit +
+// the attention) on the same machinery.
 //
 // The packed query tile is small (G*R = 32 rows for 32 q / 8 KV heads and
 // K = 7), so both products run TRANSPOSED, with the 128-wide dimension on the
 // MMA's M side and no padding waste:
 //     S^T[128 keys][32 rows] = K_tile[128 keys][128 d] . Q^T      (K-major A, B)
-//     O^T[128 d][32 rows]   += V_tile^T[128 d][128 keys] . P^T     (MN-major A, K-major B)
+//     O^T[128 d][32 rows]   += V_tile^T[128 d][128 keys] . P^T     (MN-major A, B)
 // Both accumulators live in tensor memory (S double-buffered): 96 columns.
 //
-// Warp roles in a CTA (192 threads):
+// Warp roles in a CTA (320 threads):
 //   warp 0      TMA producer: 128-key stages of K and V (128B-swizzled boxes)
-//   warp 1      allocates tensor memory; one lane issues every tcgen05.mma
-//   warps 2..5  softmax: thread t owns key lane t of S^T (all 32 rows of it):
-//               masks, row maxima by a warp butterfly + one shared exchange,
-//               P = exp2(S - m) in bf16 into shared memory, lazy O rescale
-//               (only when a row maximum grows) through tcgen05.ld/st.
+//   warp 1      allocates tensor memory; one lane issues every tcgen05.mma.
+//               S runs two tiles ahead: per tile it issues PV(t) and commits
+//               "PV(t) done" (stage t is free), then S(t+2) and commits
+//               "S(t+2) ready" (which also implies PV(t) done, so the softmax
+//               needs no other wait). Two commits a tile: each drains the
+//               MMA pipe for ~180 cycles.
+//   warps 2..9  softmax: thread (t, h) owns key lane t of S^T and query rows
+//               16h .. 16h+15; P = exp2(S - ref) goes to shared memory as
+//               P^T (64-byte swizzled, MN-major), two 16-byte stores a thread.
+//
+// Softmax with a fixed reference. The reference of a row is the exact maximum
+// of the CTA's first tile; every later tile uses it unchanged, so the loop has
+// no cross-warp step and O is never rescaled. The result is exact as long as
+// no score exceeds its reference by more than kSlack (log2 units), which keeps
+// every weight below 2^kSlack and every sum far inside fp32 range; each thread
+// tracks the largest excess it saw, and a CTA where some excess is larger runs
+// the whole range a second time with the exact maxima as references.
+//
 // Work split: one thread-block cluster per (scene, KV head); its CTAs take
-// contiguous 32-key-aligned ranges of the valid keys, and their (m, l, O)
-// partials merge through distributed shared memory at the end. Every wait
-// is bounded (SD_DEVERR_TIMEOUT instead of a hang).
+// contiguous 32-key-aligned ranges of the keys, and their (m, l, O) partials
+// merge through distributed shared memory at the end. In the fused layer the
+// tensor-core loop covers the cached prefix only; the R new keys (rotated in
+// shared memory, never re-read from the cache) enter as one more partial that
+// each CTA forms on the CUDA cores for the rows it merges. Every wait is
+// bounded (SD_DEVERR_TIMEOUT instead of a hang).
 #include "common.cuh"
 
 #include <cuda.h>
@@ -42,24 +60,34 @@ constexpr int kStage = 2 * kKV;             // 64 KB
 constexpr int kRing = kStages * kStage;     // 192 KB
 constexpr int kQHalf = kRows * 128;         // 4 KB
 constexpr int kQ = 2 * kQHalf;              // 8 KB
-constexpr int kP = 2 * kQHalf;              // one P buffer [32 rows][128 keys] bf16, 8 KB
-constexpr int kThreads = 192;
+constexpr int kPRow = kRows * 2;            // one key of P^T: 32 rows in bf16 (64 B)
+constexpr int kP = kStageKeys * kPRow;      // one P^T buffer (8 KB)
+constexpr int kMaxNew = 16;                 // new rows the fused kernel takes
+constexpr int kNewRow = kD * 2;             // one new key / value row (256 B)
+constexpr int kSoftWarps = 8;
+constexpr int kSoftThreads = 32 * kSoftWarps;
+constexpr int kThreads = 64 + kSoftThreads;
 constexpr int kTmemCols = 128;              // S0 | S1 | O  (32 columns each)
 constexpr uint32_t kSpinLimit = 1u << 20;
+constexpr float kSlack = 64.f;              // log2 units a score may exceed its reference by
 
 // shared memory layout (offsets from the 1024-aligned base)
 constexpr int kOffQ = kRing;
-constexpr int kOffP = kOffQ + kQ;
-constexpr int kOffBar = kOffP + 2 * kP;
-// barriers: full[3] empty[3] s_full[2] s_free[2] p_full[2] o_done[2] q_full recv append
-constexpr int kNumBars = 3 + 3 + 2 + 2 + 2 + 2 + 1 + 1 + 1;
-constexpr int kOffMisc = kOffBar + kNumBars * 8;
-// misc: tmem slot (4), grow flag (4), red[4][32] + 2 x 4 warp flags, mnew[32], corr[32]
-constexpr int kOffRed = kOffMisc + 16;
-constexpr int kOffMnew = kOffRed + 4 * 32 * 4 + 32;
-constexpr int kOffCorr = kOffMnew + 32 * 4;
-constexpr int kSmemBytes = kOffCorr + 32 * 4 + 1024;
+constexpr int kOffP = kOffQ + kQ;           // also the rotation table before the loop
+constexpr int kOffNewK = kOffP + 2 * kP;
+constexpr int kOffNewV = kOffNewK + kMaxNew * kNewRow;
+constexpr int kOffBar = kOffNewV + kMaxNew * kNewRow;
+// barriers: full[3] p_full[2] s_ready[2] pv_done[3] q_full recv decide
+constexpr int kNumBars = 3 + 2 + 2 + 3 + 1 + 1 + 1;
+constexpr int kOffMisc = (kOffBar + kNumBars * 8 + 15) / 16 * 16;  // tmem slot, excess flag, decision, len
+constexpr int kOffRowA = kOffMisc + 16;           // [32] per-row results (reductions)
+constexpr int kOffRef = kOffRowA + kRows * 4;     // [32] per-row references
+constexpr int kSmemBytes = kOffRef + kRows * 4 + 1024;
 static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
+static_assert(kOffQ % 1024 == 0 && kOffP % 1024 == 0 && kOffNewK % 16 == 0 && kOffNewV % 16 == 0 &&
+                  kOffBar % 8 == 0 && kOffRowA % 16 == 0 && kOffRef % 16 == 0,
+              "alignment of the shared-memory regions (swizzle atoms, vector accesses, mbarriers)");
+static_assert(kMaxNew * 64 * 8 <= 2 * kP, "rotation table fits the P buffers");
 
 // cluster merge buffers (in the ring, free once this CTA's last MMA is done):
 // a partial row is [O(128) | m | l | 2 pad] fp32 = 528 bytes
@@ -67,7 +95,11 @@ constexpr int kRowF = kD + 4;
 constexpr int kRowBytes = kRowF * 4;
 constexpr int kSend = 0;                            // this CTA's 32 rows
 constexpr int kRecv = 20 * 1024;                    // 32 slots received from the peers
-static_assert(kRecv >= kRows * kRowBytes && kRecv + kRows * kRowBytes <= kRing, "merge buffers");
+constexpr int kNewS = 40 * 1024;                    // new-key scores of the merged rows
+constexpr int kWRow = 2 * 16 + 4;                   // merge weights of a row: csize + R, 1 / l
+constexpr int kMergeW = kNewS + kRows * kMaxNew * 4;
+static_assert(kRecv >= kRows * kRowBytes && kRecv + kRows * kRowBytes <= kNewS, "merge buffers");
+static_assert(kMergeW + kRows * kWRow * 4 <= kRing, "merge buffers");
 
 __device__ __forceinline__ uint32_t smem_addr(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -93,10 +125,14 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
+__device__ __noinline__ void mbar_timed_out() { sd_set_error(SD_DEVERR_TIMEOUT); }
+// One small loop per call site (the timeout report is out of line): the code
+// that the warps run at the same time must stay inside the instruction cache.
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
+#pragma unroll 1
   for (uint32_t i = 0; i < kSpinLimit; ++i)
     if (mbar_try_wait(bar, parity)) return true;
-  sd_set_error(SD_DEVERR_TIMEOUT);
+  mbar_timed_out();
   return false;
 }
 __device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap* map, uint32_t bar,
@@ -111,6 +147,12 @@ __device__ __forceinline__ float ex2(float x) {
   float y;
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
+}
+// two floats -> bf16x2 (round to nearest even), lo in the low half
+__device__ __forceinline__ uint32_t cvt_bf16x2(float lo, float hi) {
+  uint32_t r;
+  asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+  return r;
 }
 __device__ __forceinline__ void named_bar_sync(int id, int threads) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(threads) : "memory");
@@ -135,13 +177,20 @@ __device__ __forceinline__ uint32_t cluster_map(uint32_t addr, uint32_t rank) {
   asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
   return r;
 }
+__device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t x, uint32_t y, uint32_t z,
+                                             uint32_t w) {
+  asm volatile("st.shared.v4.u32 [%0], {%1,%2,%3,%4};" ::"r"(addr), "r"(x), "r"(y), "r"(z), "r"(w)
+               : "memory");
+}
 // ---------------------------------------------------------------- tcgen05
-// Shared-memory matrix descriptor, 128-byte swizzle (sm_100 family format):
-// start address, leading / stride byte offsets (>> 4), version 1, layout 2.
-__device__ __forceinline__ uint64_t umma_desc(uint32_t addr, uint32_t lbo, uint32_t sbo) {
+// Shared-memory matrix descriptor (sm_100 family format): start address,
+// leading / stride byte offsets (>> 4), version 1, layout type (2 = 128-byte
+// swizzle, 4 = 64-byte swizzle).
+__device__ __forceinline__ uint64_t umma_desc(uint32_t addr, uint32_t lbo, uint32_t sbo,
+                                              uint64_t layout = 2) {
   return static_cast<uint64_t>((addr >> 4) & 0x3FFF) |
          (static_cast<uint64_t>((lbo >> 4) & 0x3FFF) << 16) |
-         (static_cast<uint64_t>((sbo >> 4) & 0x3FFF) << 32) | (1ull << 46) | (2ull << 61);
+         (static_cast<uint64_t>((sbo >> 4) & 0x3FFF) << 32) | (1ull << 46) | (layout << 61);
 }
 // Instruction descriptor, kind::f16: fp32 accumulate, bf16 A and B.
 constexpr uint32_t umma_idesc(int M, int N, int a_mn_major, int b_mn_major) {
@@ -150,7 +199,7 @@ constexpr uint32_t umma_idesc(int M, int N, int a_mn_major, int b_mn_major) {
          (static_cast<uint32_t>(M >> 4) << 24);
 }
 constexpr uint32_t kIdescS = umma_idesc(128, kRows, 0, 0);
-constexpr uint32_t kIdescO = umma_idesc(128, kRows, 1, 0);
+constexpr uint32_t kIdescO = umma_idesc(128, kRows, 1, 1);
 
 __device__ __forceinline__ void umma(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc,
                                      int accumulate) {
@@ -172,36 +221,44 @@ __device__ __forceinline__ void tc_fence_after() {
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
 }
 
-#define SD_R32(r)                                                                              \
-  "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),          \
-      "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),  \
-      "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),            \
-      "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),            \
-      "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
-#define SD_W32(r)                                                                              \
-  "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),      \
-      "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]),        \
-      "r"(r[15]), "r"(r[16]), "r"(r[17]), "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]),      \
-      "r"(r[22]), "r"(r[23]), "r"(r[24]), "r"(r[25]), "r"(r[26]), "r"(r[27]), "r"(r[28]),      \
-      "r"(r[29]), "r"(r[30]), "r"(r[31])
-
-// 32 consecutive fp32 columns of this warp's 32 TMEM lanes -> 32 registers
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
+// 16 consecutive fp32 columns of this warp's 32 TMEM lanes -> 16 registers
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
   asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
-      "%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
-      : SD_R32(r)
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
+      "%14,%15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15])
       : "r"(taddr));
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
-__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32]) {
-  asm volatile(
-      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,"
-      "%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(
-          taddr),
-      SD_W32(r)
-      : "memory");
-  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+
+// Per-row reduction (max or sum) over the 128 key lanes of a CTA, for the 256
+// softmax threads: thread (key lane kl, rows row0 .. row0 + 15) contributes
+// v[j] to row row0 + j. The values pass through buf ([32 rows][128] fp32,
+// 16 KB, free while this runs); the 32 results land in out[32]. Called by
+// all softmax threads; compact on purpose (it runs once or twice a launch).
+template <bool kMax>
+__device__ __forceinline__ void rows_reduce(const float (&v)[16], int kl, int row0, int st, float* buf,
+                                            float* out) {
+#pragma unroll
+  for (int j = 0; j < 16; ++j) buf[(row0 + j) * 128 + kl] = v[j];
+  asm volatile("bar.sync 2, 256;" ::: "memory");
+  const int r = st >> 3, part = st & 7;  // 8 threads per row, 16 values each
+  const float4* src = reinterpret_cast<const float4*>(buf + r * 128 + part * 16);
+  float acc = kMax ? -INFINITY : 0.f;
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const float4 x = src[q];
+    acc = kMax ? fmaxf(acc, fmaxf(fmaxf(x.x, x.y), fmaxf(x.z, x.w))) : acc + ((x.x + x.y) + (x.z + x.w));
+  }
+#pragma unroll
+  for (int w = 1; w < 8; w <<= 1) {
+    const float o = __shfl_xor_sync(0xffffffffu, acc, w);
+    acc = kMax ? fmaxf(acc, o) : acc + o;
+  }
+  if (part == 0) out[r] = acc;
+  asm volatile("bar.sync 2, 256;" ::: "memory");
 }
 
 struct TcArgs {
@@ -216,8 +273,9 @@ struct TcArgs {
   __nv_bfloat16* vc;
   const int32_t* pos;       // [B][R][3]
   uint32_t* ticket;         // [B] per-scene CTA tickets (zeroed, re-armed)
-  int early;                // the prefix may be streamed before the dependency wait
+  int early;                // prefix, len and pos may be read before the dependency wait
   int R, Hq, Hkv, G, M, cap, n_mblocks;
+  float inv_g;              // 1 / G: p / G == int((p + 0.5) / G) exactly for the p < 32 used here
   float scale_log2;
 };
 
@@ -231,15 +289,13 @@ __device__ __forceinline__ void griddep_launch() {
 // with the rotated query rows loaded by TMA.
 // kFused = true: the whole verify layer -- M-RoPE of the raw query and key
 // rows, the KV append and the attention -- with len[b] the prefix length.
-// Prefix tiles are independent of the kernel that precedes this one in the
-// stream (for every layer but the first of a step), so when a.early is set
-// they stream before the programmatic-dependency wait.
+// Prefix tiles, len and pos are independent of the kernel that precedes this
+// one in the stream (for every layer but the first of a step), so when
+// a.early is set they are read before the programmatic-dependency wait.
 template <bool kFused>
 __global__ void __launch_bounds__(kThreads, 1)
     verify_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k128,
                           const __grid_constant__ CUtensorMap tm_v128,
-                          const __grid_constant__ CUtensorMap tm_k32,
-                          const __grid_constant__ CUtensorMap tm_v32,
                           const __grid_constant__ CUtensorMap tm_q, const TcArgs a,
                           const RopeTable tab) {
   extern __shared__ uint8_t smem_raw[];
@@ -248,22 +304,27 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t base = smem_addr(smem);
   const uint32_t qs = base + kOffQ;
   auto bar = [&](int i) { return base + kOffBar + 8u * i; };
-  // barrier indices
+  // barrier indices; T counts tiles over both passes. SREADY(T) (two slots)
+  // and PVDONE(T) (one slot per stage) are tcgen05.commit arrivals. A slot's
+  // next phase cannot complete before its waiter has seen the current one:
+  // S(T + 2) needs PFULL(T), which follows the wait for SREADY(T); PV(T + 3)
+  // needs tile T + 3, loaded only after the wait for PVDONE(T).
   auto FULL = [&](int s) { return bar(s); };
-  auto EMPTY = [&](int s) { return bar(3 + s); };
-  auto SFULL = [&](int b) { return bar(6 + b); };
-  auto SFREE = [&](int b) { return bar(8 + b); };
-  auto PFULL = [&](int b) { return bar(10 + b); };
-  auto ODONE = [&](int b) { return bar(12 + b); };
-  const uint32_t QFULL = bar(14);
-  const uint32_t RECV = bar(15);  // the cluster merge's incoming partial rows
-  const uint32_t APPEND = bar(16);  // fused: the new K/V rows are in the cache
+  auto PFULL = [&](int b) { return bar(3 + b); };
+  auto SREADY = [&](int T) { return bar(5 + (T & 1)); };
+  auto PVDONE = [&](int T) { return bar(7 + T % kStages); };
+  auto sready_parity = [](int T) { return static_cast<uint32_t>((T >> 1) & 1); };
+  auto pvdone_parity = [](int T) { return static_cast<uint32_t>((T / kStages) & 1); };
+  const uint32_t QFULL = bar(10);
+  const uint32_t RECV = bar(11);    // the cluster merge's incoming partial rows
+  const uint32_t DECIDE = bar(12);  // whether the range runs a second time
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + kOffMisc);
-  int* grow_flag = reinterpret_cast<int*>(smem + kOffMisc + 4);
-  float* red = reinterpret_cast<float*>(smem + kOffRed);    // [4][32]
-  float* s_mnew = reinterpret_cast<float*>(smem + kOffMnew);
-  float* s_corr = reinterpret_cast<float*>(smem + kOffCorr);
+  int* s_excess = reinterpret_cast<int*>(smem + kOffMisc + 4);
+  int* s_redo = reinterpret_cast<int*>(smem + kOffMisc + 8);
+  float* row_a = reinterpret_cast<float*>(smem + kOffRowA);  // [32] reduction results
+  float* row_ref = reinterpret_cast<float*>(smem + kOffRef); // [32] references
 
+  auto gdiv = [&](int p) { return __float2int_rz((static_cast<float>(p) + 0.5f) * a.inv_g); };
   const int rank = blockIdx.x;
   const int csize = gridDim.x;
   const int kvh = blockIdx.y % a.Hkv;
@@ -275,17 +336,17 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
       mbar_init(FULL(s), 1);
-      mbar_init(EMPTY(s), 1);
+      mbar_init(PVDONE(s), 1);
     }
     for (int i = 0; i < 2; ++i) {
-      mbar_init(SFULL(i), 1);
-      mbar_init(SFREE(i), 4);
-      mbar_init(PFULL(i), 4);
-      mbar_init(ODONE(i), 1);
+      mbar_init(PFULL(i), kSoftWarps);
+      mbar_init(SREADY(i), 1);
     }
-    mbar_init(QFULL, kFused ? 128 : 129);  // (producer's expect_tx +) 128 softmax threads
+    mbar_init(QFULL, kFused ? 1 : 2);  // (producer's expect_tx +) one softmax thread
     mbar_init(RECV, 1);
-    mbar_init(APPEND, 1);
+    mbar_init(DECIDE, 1);
+    *s_excess = 0;
+    *s_redo = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (warp == 1) {
@@ -295,6 +356,23 @@ __global__ void __launch_bounds__(kThreads, 1)
                  : "memory");
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
+  if (kFused && !a.early) griddep_wait();  // len, pos and the prefix may come from the previous kernel
+  int* s_len = reinterpret_cast<int*>(smem + kOffMisc + 12);
+  if (threadIdx.x == 0) {
+    const int len0 = a.len[b];
+    *s_len = len0;
+    if (kFused) {
+      // advance the scene's length once every CTA of the scene has read it:
+      // the last CTA to take a ticket writes it (the fence orders this CTA's
+      // read before its ticket)
+      __threadfence();
+      const uint32_t total = gridDim.x * gridDim.y;
+      if (atomicAdd(&a.ticket[b], 1u) == total - 1) {
+        if (len0 >= 0 && len0 + a.R <= a.cap) a.len[b] = len0 + a.R;
+        a.ticket[b] = 0;
+      }
+    }
+  }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -302,72 +380,65 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem_s = tmem;          // S buffer b at column 32 * b
   const uint32_t tmem_o = tmem + 64;     // O^T
 
-  if (kFused && !a.early) griddep_wait();  // len and the prefix may come from the previous kernel
   int n_keys, L_pre;
   bool valid;
   if (kFused) {
-    L_pre = a.len[b];
+    L_pre = *s_len;
     n_keys = L_pre + a.R;
     valid = L_pre >= 0 && n_keys <= a.cap;
     if (!valid && rank == 0 && threadIdx.x == 0 && blockIdx.y == 0)
       sd_set_error(L_pre < 0 ? SD_DEVERR_LENGTH : SD_DEVERR_KV_OVERFLOW);
   } else {
-    n_keys = a.len[b];
+    n_keys = *s_len;
     valid = n_keys >= a.R && n_keys <= a.cap;
     L_pre = n_keys - a.R;
     if (!valid && rank == 0 && threadIdx.x == 0 && blockIdx.y == 0) sd_set_error(SD_DEVERR_LENGTH);
   }
-  const int nblk = valid ? (n_keys + 31) / 32 : 0;
-  int blk_begin, blk_end;
-  if (kFused) {
-    // blocks wholly inside the prefix split evenly; the last CTA also takes
-    // the block(s) holding the new rows, which it appends itself
-    const int blk_new0 = valid ? L_pre / 32 : 0;
-    blk_begin = static_cast<int>((static_cast<long long>(rank) * blk_new0) / csize);
-    blk_end = rank == csize - 1 ? nblk
-                                : static_cast<int>((static_cast<long long>(rank + 1) * blk_new0) / csize);
-  } else {
-    blk_begin = static_cast<int>((static_cast<long long>(rank) * nblk) / csize);
-    blk_end = static_cast<int>((static_cast<long long>(rank + 1) * nblk) / csize);
-  }
+  // the tensor-core loop covers the prefix (fused) or every key (standalone)
+  const int loop_keys = valid ? (kFused ? L_pre : n_keys) : 0;
+  const int nblk = (loop_keys + 31) / 32;
+  const int blk_begin = static_cast<int>((static_cast<long long>(rank) * nblk) / csize);
+  const int blk_end = static_cast<int>((static_cast<long long>(rank + 1) * nblk) / csize);
   const int key_begin = blk_begin * 32;
-  const int key_end = min(blk_end * 32, n_keys);
+  const int key_end = min(blk_end * 32, loop_keys);
   const int n_tiles = (blk_end - blk_begin + 3) / 4;
-  const bool owns_new = kFused && valid && rank == csize - 1;
-  const int t_new = owns_new ? (L_pre / 32 - blk_begin) / 4 : n_tiles;  // first tile with new rows
 
   if (warp == 0) {
     // -------------------------------------------------------------- producer
-    if (lane == 0 && n_tiles > 0) {
-      if (!kFused) {
+    if (lane == 0) {
+      if (!kFused && n_tiles > 0) {
         // the packed query tile first: box (64 d, G heads, R rows) lands as
         // rows p = i * G + g of 128 bytes, the B operand's K-major layout
         mbar_expect_tx(QFULL, static_cast<uint32_t>(2 * a.M * 128));
         for (int h = 0; h < 2; ++h)
           tma_load_3d(qs + h * kQHalf, &tm_q, QFULL, h * 64, kvh * a.G, b * a.R);
       }
-      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_k128)) : "memory");
-      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_v128)) : "memory");
-      const int z = b * a.Hkv + kvh;
-      for (int t = 0; t < n_tiles; ++t) {
-        const int s = t % kStages;
-        if (t >= kStages) mbar_wait(EMPTY(s), ((t / kStages) - 1) & 1);
-        if (kFused && t == t_new) mbar_wait(APPEND, 0);  // the new rows are in the cache
-        const int nb = min(4, blk_end - blk_begin - 4 * t);
-        const int y0 = key_begin + t * kStageKeys;
-        const uint32_t kst = base + s * kStage, vst = kst + kKV;
-        mbar_expect_tx(FULL(s), static_cast<uint32_t>(nb * 32 * 128 * 2 * 2));
-        if (nb == 4) {
-          for (int h = 0; h < 2; ++h) {
-            tma_load_3d(kst + h * kHalf, &tm_k128, FULL(s), h * 64, y0, z);
-            tma_load_3d(vst + h * kHalf, &tm_v128, FULL(s), h * 64, y0, z);
+      if (n_tiles > 0) {
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_k128)) : "memory");
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_v128)) : "memory");
+        const int z = b * a.Hkv + kvh;
+        for (int pass = 0; pass < 2; ++pass) {
+          if (pass == 1) {
+            // every MMA of pass 0 is done when the decision is out
+            mbar_wait(DECIDE, 0);
+            if (!*reinterpret_cast<volatile int*>(s_redo)) break;
           }
-        } else {
-          for (int j = 0; j < nb; ++j)
+          for (int t = 0; t < n_tiles; ++t) {
+            const int T = pass * n_tiles + t;
+            const int s = T % kStages;
+            // stage s last held tile T - 3 (all of pass 0 is done before pass 1 starts)
+            if (t >= kStages) mbar_wait(PVDONE(T - kStages), pvdone_parity(T - kStages));
+            // a whole 128-row box even for a short last tile: keys past the
+            // range are masked, rows past the capacity arrive zero-filled
+            const int y0 = key_begin + t * kStageKeys;
+            const uint32_t kst = base + s * kStage, vst = kst + kKV;
+            mbar_expect_tx(FULL(s), static_cast<uint32_t>(kStage));
+#pragma unroll
             for (int h = 0; h < 2; ++h) {
-              tma_load_3d(kst + h * kHalf + j * 4096, &tm_k32, FULL(s), h * 64, y0 + 32 * j, z);
-              tma_load_3d(vst + h * kHalf + j * 4096, &tm_v32, FULL(s), h * 64, y0 + 32 * j, z);
+              tma_load_3d(kst + h * kHalf, &tm_k128, FULL(s), h * 64, y0, z);
+              tma_load_3d(vst + h * kHalf, &tm_v128, FULL(s), h * 64, y0, z);
             }
+          }
         }
       }
     }
@@ -378,341 +449,447 @@ __global__ void __launch_bounds__(kThreads, 1)
     // -------------------------------------------------------------- MMA issue
     if (lane == 0 && n_tiles > 0) {
       mbar_wait(QFULL, 0);
-      auto issue_pv = [&](int u) {
-        const int bb = u & 1, s = u % kStages;
-        mbar_wait(PFULL(bb), (u >> 1) & 1);
-        tc_fence_after();
-        const uint32_t vst = base + s * kStage + kKV;
-        const uint32_t pb = base + kOffP + bb * kP;
-#pragma unroll
-        for (int kk = 0; kk < 8; ++kk) {
-          const uint64_t ad = umma_desc(vst + kk * 2048, kHalf, 1024);      // V^T: MN-major
-          const uint64_t bd = umma_desc(pb + (kk >> 2) * kQHalf + (kk & 3) * 32, 16, 1024);
-          umma(tmem_o, ad, bd, kIdescO, (u > 0 || kk > 0) ? 1 : 0);
+      // base descriptors; a K step only moves the start address (low field, no carry)
+      const uint64_t dK0 = umma_desc(base, 16, 1024);              // K tile: K-major
+      const uint64_t dV0 = umma_desc(base + kKV, kHalf, 1024);     // V^T: MN-major
+      const uint64_t dQ = umma_desc(qs, 16, 1024);                 // Q: K-major
+      const uint64_t dP0 = umma_desc(base + kOffP, 0, 512, 4);     // P^T: MN-major, 64B swizzle
+      // Two issue sites with every K-step offset a compile-time constant (one
+      // 64-bit add per descriptor): a rolled or shared issue loop measured
+      // ~1.8 us slower per layer.
+      for (int pass = 0; pass < 2; ++pass) {
+        if (pass == 1) {
+          mbar_wait(DECIDE, 0);
+          if (!*reinterpret_cast<volatile int*>(s_redo)) break;
         }
-        umma_commit(ODONE(bb));
-        umma_commit(EMPTY(s));
-      };
-      for (int t = 0; t < n_tiles; ++t) {
-        const int s = t % kStages, bb = t & 1;
-        mbar_wait(FULL(s), (t / kStages) & 1);
-        if (t >= 2) mbar_wait(SFREE(bb), ((t >> 1) - 1) & 1);
-        tc_fence_after();
-        const uint32_t kst = base + s * kStage;
+        const int T0 = pass * n_tiles;
+        // S(0), S(1) first; then per tile PV(t) and S(t + 2)
+        for (int t = -2; t < n_tiles; ++t) {
+          if (t >= 0) {
+            const int T = T0 + t;
+            mbar_wait(PFULL(T & 1), (T >> 1) & 1);
+            tc_fence_after();
+            const uint64_t dv = dV0 + static_cast<uint64_t>(((T % kStages) * kStage) >> 4);
+            const uint64_t dp = dP0 + static_cast<uint64_t>(((T & 1) * kP) >> 4);
 #pragma unroll
-        for (int kk = 0; kk < 8; ++kk) {
-          const uint64_t ad = umma_desc(kst + (kk >> 2) * kHalf + (kk & 3) * 32, 16, 1024);
-          const uint64_t bd = umma_desc(qs + (kk >> 2) * kQHalf + (kk & 3) * 32, 16, 1024);
-          umma(tmem_s + 32 * bb, ad, bd, kIdescS, kk > 0 ? 1 : 0);
+            for (int kk = 0; kk < 8; ++kk)
+              umma(tmem_o, dv + (kk * 2048 >> 4), dp + (kk * 1024 >> 4), kIdescO, (t > 0 || kk > 0) ? 1 : 0);
+            umma_commit(PVDONE(T));
+          }
+          if (t + 2 < n_tiles) {
+            // S(T) reuses the S buffer of tile T - 2, read before PFULL(T - 2)
+            const int T = T0 + t + 2, st_ = T % kStages;
+            mbar_wait(FULL(st_), (T / kStages) & 1);
+            tc_fence_after();
+            const uint64_t dk = dK0 + static_cast<uint64_t>((st_ * kStage) >> 4);
+            const uint32_t ts = tmem_s + 32 * (T & 1);
+#pragma unroll
+            for (int kk = 0; kk < 8; ++kk)
+              umma(ts, dk + (((kk >> 2) * kHalf + (kk & 3) * 32) >> 4),
+                   dQ + (((kk >> 2) * kQHalf + (kk & 3) * 32) >> 4), kIdescS, kk > 0 ? 1 : 0);
+            umma_commit(SREADY(T));
+          }
         }
-        umma_commit(SFULL(bb));
-        if (t >= 1) issue_pv(t - 1);
       }
-      issue_pv(n_tiles - 1);
     }
     __syncwarp();
     cluster_arrive();
     cluster_wait();
   } else {
     // -------------------------------------------------------------- softmax
-    const int st = threadIdx.x - 64;       // 0..127
+    const int st = threadIdx.x - 64;       // 0..255
+    const int half = (warp - 2) >> 2;      // query rows 16*half .. 16*half + 15
     const int quarter = warp & 3;          // TMEM lane quarter of this warp
     const int kl = quarter * 32 + lane;    // key lane of S^T / d lane of O^T
     const uint32_t lane_off = static_cast<uint32_t>(quarter * 32) << 16;
+    const int row0 = 16 * half;            // first query row of this thread
+    const float2* cs_tab = reinterpret_cast<const float2*>(smem + kOffP);  // [R][64] (cos, sin)
     if (!kFused) {
       // query rows past M stay zero (the TMA box covers rows 0..M-1 only)
-      for (int idx = st; idx < (kRows - a.M) * 16; idx += 128) {
+      for (int idx = st; idx < (kRows - a.M) * 16; idx += kSoftThreads) {
         const int row = a.M + idx / 16, c = idx % 16;
-        asm volatile("st.shared.v4.u32 [%0], {%1,%1,%1,%1};" ::"r"(qs + (c >> 3) * kQHalf + row * 128 + (c & 7) * 16),
-                     "r"(0)
-                     : "memory");
+        st_shared_v4(qs + (c >> 3) * kQHalf + row * 128 + (c & 7) * 16, 0u, 0u, 0u, 0u);
       }
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-      mbar_arrive(QFULL);
+      named_bar_sync(2, kSoftThreads);
+      if (st == 0) mbar_arrive(QFULL);
     } else {
-      // the raw rows come from earlier kernels; once they are visible every
-      // older kernel has finished, so the next layer may launch
-      griddep_wait();
-      if (st == 0) griddep_launch();
-      // M-RoPE of the packed query rows, straight into the swizzled tile
-      for (int idx = st; idx < kRows * 16; idx += 128) {
-        const int row = idx / 16, c = idx % 16;
-        const int p = mblock * kRows + row;
-        uint32_t w[4] = {0u, 0u, 0u, 0u};
-        if (valid && p < a.M) {
-          const int i = p / a.G, gq = p % a.G;
-          const uint4 v = *reinterpret_cast<const uint4*>(
-              a.qw + ((static_cast<long long>(b) * a.R + i) * a.Hq + kvh * a.G + gq) * kD + c * 8);
-          w[0] = v.x; w[1] = v.y; w[2] = v.z; w[3] = v.w;
-          const int32_t* pp = a.pos + (static_cast<long long>(b) * a.R + i) * 3;
-          const int p3[3] = {pp[0], pp[1], pp[2]};
-          sd_rope_rotate8(w, c, p3, tab);
+      // rotation table of the R new positions: (cos, sin) per (row, pair)
+      if (valid) {
+        float2* tabw = reinterpret_cast<float2*>(smem + kOffP);
+#pragma unroll 1
+        for (int idx = st; idx < a.R * 64; idx += kSoftThreads) {
+          const int i = idx >> 6, d = idx & 63;
+          const int32_t pc = a.pos[(static_cast<long long>(b) * a.R + i) * 3 + tab.axis[d]];
+          tabw[idx] = sd_rope_cs(static_cast<float>(pc), d, tab);
         }
-        asm volatile("st.shared.v4.u32 [%0], {%1,%2,%3,%4};" ::"r"(
-                         qs + (c >> 3) * kQHalf + row * 128 + (((c & 7) ^ (row & 7)) << 4)),
-                     "r"(w[0]), "r"(w[1]), "r"(w[2]), "r"(w[3])
-                     : "memory");
+      }
+      named_bar_sync(2, kSoftThreads);  // the rotation table is complete
+      // this thread's pieces: query chunks (row, 16-byte chunk c) u = 0, 1 and
+      // one chunk of a new key / value row
+      const __nv_bfloat16* q_src[2];
+      int q_cs[2];
+      bool q_ok[2];
+#pragma unroll
+      for (int u = 0; u < 2; ++u) {
+        const int idx = st + u * kSoftThreads, p = mblock * kRows + (idx >> 4), c = idx & 15;
+        const int i = gdiv(p);
+        q_ok[u] = valid && p < a.M;
+        q_src[u] = a.qw + ((static_cast<long long>(b) * a.R + i) * a.Hq + kvh * a.G + (p - i * a.G)) * kD + c * 8;
+        q_cs[u] = i * 64 + c * 4;
+      }
+      const bool has_kv = valid && st < a.R * 16;
+      const long long kv_src = ((static_cast<long long>(b) * a.R + (st >> 4)) * a.Hkv + kvh) * kD + (st & 15) * 8;
+      // Iteration 0 runs BEFORE the dependency wait on whatever the rows hold:
+      // it brings this code into the instruction cache and the rows into L2,
+      // and iteration 1 overwrites everything it stored. The loads bypass L1
+      // (.cg) so that iteration 1 cannot hit a line read before the wait.
+#pragma unroll 1
+      for (int it = 0; it < 2; ++it) {
+        if (it == 1 && a.early) griddep_wait();  // the raw rows come from earlier kernels
+        uint4 qv[2], kv = make_uint4(0, 0, 0, 0), vv = make_uint4(0, 0, 0, 0);
+#pragma unroll
+        for (int u = 0; u < 2; ++u)
+          qv[u] = q_ok[u] ? __ldcg(reinterpret_cast<const uint4*>(q_src[u])) : make_uint4(0, 0, 0, 0);
+        if (has_kv) {
+          kv = __ldcg(reinterpret_cast<const uint4*>(a.k_new + kv_src));
+          vv = __ldcg(reinterpret_cast<const uint4*>(a.v_new + kv_src));
+        }
+        // M-RoPE of the packed query rows, straight into the swizzled tile
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+          const int idx = st + u * kSoftThreads, row = idx >> 4, c = idx & 15;
+          uint32_t w[4] = {qv[u].x, qv[u].y, qv[u].z, qv[u].w};
+          if (q_ok[u]) {
+            const float2* cs = cs_tab + q_cs[u];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) w[j] = sd_rope_pair(w[j], cs[j].x, cs[j].y);
+          }
+          st_shared_v4(qs + (c >> 3) * kQHalf + row * 128 + (((c & 7) ^ (row & 7)) << 4), w[0], w[1],
+                       w[2], w[3]);
+        }
+        // the new key rows (rotated) and value rows of this head
+        if (has_kv) {
+          const int i = st >> 4, c = st & 15;
+          const float2* cs = cs_tab + i * 64 + c * 4;
+          uint32_t w[4] = {kv.x, kv.y, kv.z, kv.w};
+#pragma unroll
+          for (int j = 0; j < 4; ++j) w[j] = sd_rope_pair(w[j], cs[j].x, cs[j].y);
+          st_shared_v4(base + kOffNewK + i * kNewRow + c * 16, w[0], w[1], w[2], w[3]);
+          st_shared_v4(base + kOffNewV + i * kNewRow + c * 16, vv.x, vv.y, vv.z, vv.w);
+        }
       }
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-      mbar_arrive(QFULL);
-      if (owns_new) {
-        // M-RoPE of this head's new key rows and the append of K and V; the
-        // rotated keys also go back to k_new, like the standalone rotation
-        for (int idx = st; idx < a.R * 16; idx += 128) {
-          const int i = idx / 16, c = idx % 16;
-          const long long src = ((static_cast<long long>(b) * a.R + i) * a.Hkv + kvh) * kD + c * 8;
-          const long long dst = ((static_cast<long long>(b) * a.Hkv + kvh) * a.cap + L_pre + i) * kD + c * 8;
-          const uint4 kv = *reinterpret_cast<const uint4*>(a.k_new + src);
-          uint32_t w[4] = {kv.x, kv.y, kv.z, kv.w};
-          const int32_t* pp = a.pos + (static_cast<long long>(b) * a.R + i) * 3;
-          const int p3[3] = {pp[0], pp[1], pp[2]};
-          sd_rope_rotate8(w, c, p3, tab);
-          const uint4 kr = make_uint4(w[0], w[1], w[2], w[3]);
-          *reinterpret_cast<uint4*>(a.kc + dst) = kr;
-          *reinterpret_cast<uint4*>(a.k_new + src) = kr;
-          *reinterpret_cast<uint4*>(a.vc + dst) = *reinterpret_cast<const uint4*>(a.v_new + src);
-        }
-        asm volatile("fence.proxy.async.global;" ::: "memory");  // visible to the TMA loads
-        named_bar_sync(2, 128);
-        if (st == 0) mbar_arrive(APPEND);
+      named_bar_sync(2, kSoftThreads);  // Q is complete; the rotation table is no longer read
+      if (st == 0) {
+        mbar_arrive(QFULL);
+        // every older kernel has finished: the next layer may launch
+        griddep_launch();
       }
     }
 
-    const int L_prefix = n_keys - a.R;
     const float sl = a.scale_log2;
-    // Reference maximum per query row (log2 units), identical in every
-    // softmax thread. It is set exactly on the first tile; later tiles keep it
-    // unless some score exceeds it by more than kSlack, so exp2(s - ref) <= 2^8
-    // stays exact in bf16 / fp32 and the common tile needs no cross-warp work.
-    constexpr float kSlack = 8.f;
-    float mref[32];
-    float lp[32];  // per-row partial sums of this thread's key lane
+    float ref[16];  // reference per query row (log2 units), -inf: no key yet
+    float lp[16];   // per-row partial sums of this thread's key lane
+    float ex[16];   // largest score - reference seen
 #pragma unroll
-    for (int j = 0; j < 32; ++j) {
-      mref[j] = -INFINITY;
+    for (int j = 0; j < 16; ++j) {
+      ref[j] = -INFINITY;
       lp[j] = 0.f;
+      ex[j] = -INFINITY;
     }
-
-    for (int t = 0; t < n_tiles; ++t) {
-      const int bb = t & 1, s = t % kStages;
-      const int key0 = key_begin + t * kStageKeys;
+    const int L_prefix = n_keys - a.R;
+    // per-key-lane masks of a tile: the key range, and the causal limit of the
+    // new rows that the standalone kernel's range contains
+    auto tile_mask = [&](int key0, bool (&ok)[16]) {
       const int key = key0 + kl;
-      mbar_wait(SFULL(bb), (t >> 1) & 1);
-      tc_fence_after();
-      uint32_t r[32];
-      tmem_ld32(tmem_s + 32 * bb + lane_off, r);
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(SFREE(bb));
-      // scale, range / causal mask
-      float sv[32];
       const bool key_ok = key < key_end;
-      const bool tail = key0 + kStageKeys - 1 > L_prefix;
-      bool over = false;
+      const bool tail = !kFused && key0 + kStageKeys - 1 > L_prefix;
 #pragma unroll
-      for (int j = 0; j < 32; ++j) {
-        float x = key_ok ? __uint_as_float(r[j]) * sl : -INFINITY;
-        if (tail) {
-          const int p = mblock * kRows + j;
-          const int lim = min(L_prefix + p / a.G, n_keys - 1);
-          if (key > lim) x = -INFINITY;
-        }
-        sv[j] = x;
-        over |= x > mref[j] + kSlack;
+      for (int j = 0; j < 16; ++j) {
+        ok[j] = key_ok;
+        if (tail) ok[j] = ok[j] && key <= min(L_prefix + gdiv(mblock * kRows + row0 + j), n_keys - 1);
       }
-      // do the four warps agree to keep the references? (one barrier)
-      const bool warp_over = __any_sync(0xffffffffu, over);
-      // flags are double-buffered by tile parity: a warp that runs ahead to
-      // the next tile cannot overwrite a slot another warp has yet to read
-      volatile int* flags = reinterpret_cast<volatile int*>(red) + 128 + 4 * bb;
-      if (lane == 0) flags[quarter] = warp_over ? 1 : 0;
-      named_bar_sync(2, 128);
-      const bool slow = (flags[0] | flags[1] | flags[2] | flags[3]) != 0;
-      bool rescale = false;
-      if (slow) {
-        // exact row maxima of this tile: warp butterfly (lane ends with row
-        // `lane`), then across the four warps through shared memory
-        float v[32];
+    };
+    if (n_tiles > 0) {
+      // references: exact row maxima of the first tile (through the P buffers,
+      // which no P has used yet)
+      mbar_wait(SREADY(0), 0);
+      tc_fence_after();
+      uint32_t r[16];
+      tmem_ld16(tmem_s + row0 + lane_off, r);
+      bool ok[16];
+      tile_mask(key_begin, ok);
+      float v[16];
 #pragma unroll
-        for (int j = 0; j < 32; ++j) v[j] = sv[j];
+      for (int j = 0; j < 16; ++j) v[j] = ok[j] ? __uint_as_float(r[j]) * sl : -INFINITY;
+      rows_reduce<true>(v, kl, row0, st, reinterpret_cast<float*>(smem + kOffP), row_ref);
+      const float4* rr4 = reinterpret_cast<const float4*>(row_ref + row0);
 #pragma unroll
-        for (int w = 16; w >= 1; w >>= 1) {
-          const bool upper = (lane & w) != 0;
+      for (int j4 = 0; j4 < 4; ++j4) {
+        const float4 x = rr4[j4];
+        ref[4 * j4 + 0] = x.x;
+        ref[4 * j4 + 1] = x.y;
+        ref[4 * j4 + 2] = x.z;
+        ref[4 * j4 + 3] = x.w;
+      }
+    }
+    bool redo = false;
+    for (int pass = 0; pass < 2; ++pass) {
+      if (pass == 1 && !redo) break;
+      for (int t = 0; t < n_tiles; ++t) {
+        const int T = pass * n_tiles + t;
+        const int bb = T & 1, s = T % kStages;
+        const int key0 = key_begin + t * kStageKeys;
+        const int key = key0 + kl;
+        mbar_wait(SREADY(T), sready_parity(T));  // S(T) is ready, and so PV(T - 2) is done
+        tc_fence_after();
+        uint32_t r[16];
+        tmem_ld16(tmem_s + 32 * bb + row0 + lane_off, r);
+        const bool key_ok = key < key_end;
+        bool ok[16];
+        tile_mask(key0, ok);
+        // P = exp2(S * scale - ref) in bf16; l partials from the same rounded weights
+        uint32_t pw[8];
 #pragma unroll
-          for (int i = 0; i < w; ++i) {
-            const float send = upper ? v[i] : v[i + w];
-            const float keep = upper ? v[i + w] : v[i];
-            v[i] = fmaxf(keep, __shfl_xor_sync(0xffffffffu, send, w));
+        for (int j = 0; j < 16; j += 2) {
+          const float m0 = ref[j] == -INFINITY ? 0.f : ref[j];
+          const float m1 = ref[j + 1] == -INFINITY ? 0.f : ref[j + 1];
+          const float y0 = ok[j] ? fmaf(__uint_as_float(r[j]), sl, -m0) : -INFINITY;
+          const float y1 = ok[j + 1] ? fmaf(__uint_as_float(r[j + 1]), sl, -m1) : -INFINITY;
+          ex[j] = fmaxf(ex[j], y0);
+          ex[j + 1] = fmaxf(ex[j + 1], y1);
+          const uint32_t w = cvt_bf16x2(ex2(y0), ex2(y1));
+          pw[j >> 1] = w;
+          lp[j] += sd_bf16_lo(w);
+          lp[j + 1] += sd_bf16_hi(w);
+        }
+        // P^T key row kl (its buffer's previous tile, T - 2, is done: see above): 64 bytes = 4 chunks of 8 query rows, 64-byte swizzle
+        const uint32_t prow = base + kOffP + bb * kP + kl * kPRow;
+        const int sw = (kl >> 1) & 3;
+        st_shared_v4(prow + (((2 * half) ^ sw) << 4), pw[0], pw[1], pw[2], pw[3]);
+        st_shared_v4(prow + (((2 * half + 1) ^ sw) << 4), pw[4], pw[5], pw[6], pw[7]);
+        if (!key_ok) {
+          // stale or foreign key row: zero its V row so 0 * NaN cannot reach O
+          const uint32_t vrow = base + s * kStage + kKV + half * kHalf + kl * 128;
+#pragma unroll
+          for (int c = 0; c < 8; ++c) st_shared_v4(vrow + c * 16, 0u, 0u, 0u, 0u);
+        }
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(PFULL(bb));
+      }
+      if (n_tiles > 0) {
+        // every MMA of the pass is done (the slot's previous phase, PV(Tl - 3),
+        // is implied by SREADY(Tl))
+        const int Tl = pass * n_tiles + n_tiles - 1;
+        mbar_wait(PVDONE(Tl), pvdone_parity(Tl));
+      }
+      if (pass == 0) {
+        // did any score exceed its reference by more than kSlack?
+        bool over = false;
+#pragma unroll
+        for (int j = 0; j < 16; ++j) over |= ex[j] > kSlack;
+        if (__any_sync(0xffffffffu, over) && lane == 0) atomicOr(s_excess, 1);
+        named_bar_sync(2, kSoftThreads);
+        redo = *reinterpret_cast<volatile int*>(s_excess) != 0;
+        if (st == 0) {
+          *s_redo = redo ? 1 : 0;
+          mbar_arrive(DECIDE);
+        }
+        if (redo) {
+          // second pass with the exact row maxima of the whole range (every
+          // MMA is done: the P buffers are free)
+          rows_reduce<true>(ex, kl, row0, st, reinterpret_cast<float*>(smem + kOffP), row_a);
+#pragma unroll
+          for (int j = 0; j < 16; ++j) {
+            const float e = row_a[row0 + j];
+            const float m0 = ref[j] == -INFINITY ? 0.f : ref[j];
+            ref[j] = e == -INFINITY ? -INFINITY : m0 + e;
+            lp[j] = 0.f;
+          }
+          if (quarter == 0 && lane < 16) {
+            const float e = row_a[row0 + lane];
+            const float m0 = row_ref[row0 + lane] == -INFINITY ? 0.f : row_ref[row0 + lane];
+            row_ref[row0 + lane] = e == -INFINITY ? -INFINITY : m0 + e;
           }
         }
-        red[quarter * 32 + lane] = v[0];
-        named_bar_sync(2, 128);
-        if (quarter == 0) {
-          const float smax = fmaxf(fmaxf(red[lane], red[32 + lane]), fmaxf(red[64 + lane], red[96 + lane]));
-          const float old = s_mnew[lane];
-          const float nw = t == 0 ? smax : fmaxf(old, smax);
-          s_corr[lane] = (t == 0 || old == -INFINITY || nw == old) ? 1.f : ex2(old - nw);
-          s_mnew[lane] = nw;
-          const bool grow = t > 0 && old != -INFINITY && nw > old;
-          const bool any_grow = __any_sync(0xffffffffu, grow);
-          if (lane == 0) *grow_flag = any_grow ? 1 : 0;
-        }
-        named_bar_sync(2, 128);
-        rescale = *grow_flag != 0;
-#pragma unroll
-        for (int j = 0; j < 32; ++j) mref[j] = s_mnew[j];
-        if (rescale) {
-#pragma unroll
-          for (int j = 0; j < 32; ++j) lp[j] *= s_corr[j];
-        }
       }
-      // P = exp2(S - ref) in bf16; l partials from the same rounded weights
-      uint16_t pb[32];
-#pragma unroll
-      for (int j = 0; j < 32; ++j) {
-        const float mb = mref[j] == -INFINITY ? 0.f : mref[j];
-        const __nv_bfloat16 h = __float2bfloat16_rn(ex2(sv[j] - mb));
-        pb[j] = *reinterpret_cast<const uint16_t*>(&h);
-        lp[j] += __bfloat162float(h);
-      }
-      // P buffer bb is free once PV of tile t-2 is done
-      if (t >= 2) mbar_wait(ODONE(bb), ((t >> 1) - 1) & 1);
-      if (rescale) {
-        // O^T holds PV of tiles < t at the old references: wait for PV t-1,
-        // then scale column j (query row j) of this thread's d lane
-        mbar_wait(ODONE((t - 1) & 1), ((t - 1) >> 1) & 1);
-        tc_fence_after();
-        uint32_t o[32];
-        tmem_ld32(tmem_o + lane_off, o);
-#pragma unroll
-        for (int j = 0; j < 32; ++j) o[j] = __float_as_uint(__uint_as_float(o[j]) * s_corr[j]);
-        tmem_st32(tmem_o + lane_off, o);
-      }
-      const uint32_t pbuf = base + kOffP + bb * kP + (kl >> 6) * kQHalf;
-      const int kc = (kl & 63) >> 3, kw = (kl & 7) * 2;
-#pragma unroll
-      for (int j = 0; j < 32; ++j) {
-        const uint32_t addr = pbuf + j * 128 + ((kc ^ (j & 7)) << 4) + kw;
-        asm volatile("st.shared.u16 [%0], %1;" ::"r"(addr), "h"(pb[j]) : "memory");
-      }
-      if (!key_ok) {
-        // stale or foreign key row: zero its V row so 0 * NaN cannot reach O
-        const uint32_t vrow = base + s * kStage + kKV + kl * 128;
-#pragma unroll
-        for (int h = 0; h < 2; ++h)
-#pragma unroll
-          for (int c = 0; c < 8; ++c)
-            asm volatile("st.shared.v4.u32 [%0], {%1,%1,%1,%1};" ::"r"(vrow + h * kHalf + c * 16),
-                         "r"(0)
-                         : "memory");
-      }
-      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(PFULL(bb));
     }
 
-    // ---- CTA partial: O^T (tensor memory) of this thread's d lane, and the
-    //      per-row m (reference) and l (sum over all 128 key lanes)
-    float o_f[32];
+    // ---- CTA partial: O^T (tensor memory) of this thread's d lane and rows,
+    //      and the per-row m (reference) and l (sum over all 128 key lanes)
+    float o_f[16];
     if (n_tiles > 0) {
-      mbar_wait(ODONE((n_tiles - 1) & 1), ((n_tiles - 1) >> 1) & 1);
       tc_fence_after();
-      uint32_t o[32];
-      tmem_ld32(tmem_o + lane_off, o);
+      uint32_t o[16];
+      tmem_ld16(tmem_o + row0 + lane_off, o);
 #pragma unroll
-      for (int j = 0; j < 32; ++j) o_f[j] = __uint_as_float(o[j]);
+      for (int j = 0; j < 16; ++j) o_f[j] = __uint_as_float(o[j]);
     } else {
 #pragma unroll
-      for (int j = 0; j < 32; ++j) o_f[j] = 0.f;
+      for (int j = 0; j < 16; ++j) o_f[j] = 0.f;
     }
     // every MMA of this CTA is done: its ring may now receive peers' partials
     cluster_arrive();
+    // stage the partial row-major: row j = [O(128) | m | l | pad], 528 bytes;
+    // the l terms of the 128 key lanes go through the (free) P buffers
+    float* send = reinterpret_cast<float*>(smem + kSend);
+    float* lbuf = reinterpret_cast<float*>(smem + kOffP);  // [32 rows][128 key lanes]
 #pragma unroll
-    for (int w = 16; w >= 1; w >>= 1) {
-      const bool upper = (lane & w) != 0;
+    for (int j = 0; j < 16; ++j) {
+      send[(row0 + j) * kRowF + kl] = o_f[j];
+      lbuf[(row0 + j) * 128 + kl] = lp[j];
+    }
+    named_bar_sync(2, kSoftThreads);
+    {
+      const int r = st >> 3, part = st & 7;  // 8 threads per row, 16 key lanes each
+      const float4* src = reinterpret_cast<const float4*>(lbuf + r * 128 + part * 16);
+      float l = 0.f;
 #pragma unroll
-      for (int i = 0; i < w; ++i) {
-        const float send = upper ? lp[i] : lp[i + w];
-        const float keep = upper ? lp[i + w] : lp[i];
-        lp[i] = keep + __shfl_xor_sync(0xffffffffu, send, w);
+      for (int q4 = 0; q4 < 4; ++q4) {
+        const float4 x = src[q4];
+        l += (x.x + x.y) + (x.z + x.w);
+      }
+      l += __shfl_xor_sync(0xffffffffu, l, 1);
+      l += __shfl_xor_sync(0xffffffffu, l, 2);
+      l += __shfl_xor_sync(0xffffffffu, l, 4);
+      if (part == 0) {
+        send[r * kRowF + kD] = n_tiles > 0 ? row_ref[r] : -INFINITY;
+        send[r * kRowF + kD + 1] = l;
       }
     }
-    named_bar_sync(2, 128);
-    red[quarter * 32 + lane] = lp[0];
-    named_bar_sync(2, 128);
-    const float l_row = (red[lane] + red[32 + lane]) + (red[64 + lane] + red[96 + lane]);
-    const float m_row = n_tiles > 0 ? s_mnew[lane] : -INFINITY;
-    // stage the partial row-major: row j = [O(128) | m | l | pad], 528 bytes
-    float* send = reinterpret_cast<float*>(smem + kSend);
-#pragma unroll
-    for (int j = 0; j < 32; ++j) send[j * kRowF + kl] = o_f[j];
-    if (quarter == 0) {
-      send[lane * kRowF + kD] = m_row;
-      send[lane * kRowF + kD + 1] = l_row;
-    }
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-    named_bar_sync(2, 128);
+    named_bar_sync(2, kSoftThreads);
     const int rpc = kRows / csize;
     if (st == 0) mbar_expect_tx(RECV, static_cast<uint32_t>(csize * rpc * kRowBytes));
     cluster_wait();  // every peer's ring is free to receive
-    if (st == 0) {
-      // rows [c * rpc, (c + 1) * rpc) go to rank c, into its slots [rank * rpc, ...)
-      for (int c = 0; c < csize; ++c)
-        bulk_copy_s2s(cluster_map(base + kRecv + rank * rpc * kRowBytes, c),
-                      base + kSend + c * rpc * kRowBytes, static_cast<uint32_t>(rpc * kRowBytes),
-                      cluster_map(RECV, c));
+    if (st < csize) {
+      // thread c sends rows [c * rpc, (c + 1) * rpc) to rank c, into its slots [rank * rpc, ...)
+      bulk_copy_s2s(cluster_map(base + kRecv + rank * rpc * kRowBytes, st),
+                    base + kSend + st * rpc * kRowBytes, static_cast<uint32_t>(rpc * kRowBytes),
+                    cluster_map(RECV, st));
       asm volatile("cp.async.bulk.commit_group;" ::: "memory");
-      asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
     }
-    // ---- local merge of the rows this CTA owns; slot c * rpc + rr came from rank c
+    const int mrow0 = rank * rpc;  // the rows this CTA merges
+    float* s_new = reinterpret_cast<float*>(smem + kNewS);  // [rpc][R] scores of the new keys
+    if (kFused && valid) {
+      // new-key scores (log2 units) of the merged rows, 8 threads per dot product;
+      // query row p = i * G + g sees new keys 0..i (Eq. verify's causal mask)
+      const int sub = lane & 7;
+      const int n_pairs = rpc * a.R;
+#pragma unroll 1
+      for (int pr0 = (st >> 5) * 4; pr0 < n_pairs; pr0 += kSoftThreads / 8) {  // warp-uniform
+        const int pr = min(pr0 + (lane >> 3), n_pairs - 1);
+        const bool act = pr0 + (lane >> 3) < n_pairs;
+        const int rr = pr / a.R, n = pr % a.R;
+        const int row = mrow0 + rr;
+        const int p = mblock * kRows + row;
+        float acc = 0.f;
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+          const int c = 2 * sub + u;
+          const uint4 qw4 = *reinterpret_cast<const uint4*>(smem + kOffQ + (c >> 3) * kQHalf + row * 128 +
+                                                             (((c & 7) ^ (row & 7)) << 4));
+          const uint4 kw4 = *reinterpret_cast<const uint4*>(smem + kOffNewK + n * kNewRow + c * 16);
+          const uint32_t qa[4] = {qw4.x, qw4.y, qw4.z, qw4.w};
+          const uint32_t ka[4] = {kw4.x, kw4.y, kw4.z, kw4.w};
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            acc = fmaf(sd_bf16_lo(qa[j]), sd_bf16_lo(ka[j]), acc);
+            acc = fmaf(sd_bf16_hi(qa[j]), sd_bf16_hi(ka[j]), acc);
+          }
+        }
+        acc += __shfl_xor_sync(0xffffffffu, acc, 1);
+        acc += __shfl_xor_sync(0xffffffffu, acc, 2);
+        acc += __shfl_xor_sync(0xffffffffu, acc, 4);
+        if (sub == 0 && act) s_new[pr] = (p < a.M && n <= gdiv(p)) ? acc * sl : -INFINITY;
+      }
+      named_bar_sync(2, kSoftThreads);
+    }
+    // ---- merge of the rows this CTA owns; slot c * rpc + rr came from rank c.
+    // Weights first, one warp per row: lane j < csize takes partial j, lane
+    // csize + n new key n; then every output is a sum of independent loads.
     mbar_wait(RECV, 0);
     const float* recv = reinterpret_cast<const float*>(smem + kRecv);
-    for (int rr = 0; rr < rpc; ++rr) {
-      const int row = rank * rpc + rr;
-      const int p = mblock * kRows + row;
-      float mmax = -INFINITY;
-      for (int c = 0; c < csize; ++c) mmax = fmaxf(mmax, recv[(c * rpc + rr) * kRowF + kD]);
-      float acc = 0.f, lsum = 0.f;
-      for (int c = 0; c < csize; ++c) {
-        const float* slot = recv + (c * rpc + rr) * kRowF;
-        const float mc = slot[kD];
-        const float f = mc == -INFINITY ? 0.f : ex2(mc - mmax);
-        acc = fmaf(f, slot[kl], acc);
-        lsum = fmaf(f, slot[kD + 1], lsum);
+    float* s_w = reinterpret_cast<float*>(smem + kMergeW);  // [rpc][kWRow]: weights, then 1 / l
+    const int n_new = (kFused && valid) ? a.R : 0;
+#pragma unroll 1
+    for (int rr = warp - 2; rr < rpc; rr += kSoftWarps) {
+      float m = -INFINITY, l = 0.f;
+      if (lane < csize) {
+        m = recv[(lane * rpc + rr) * kRowF + kD];
+        l = recv[(lane * rpc + rr) * kRowF + kD + 1];
+      } else if (lane < csize + n_new) {
+        m = s_new[rr * a.R + (lane - csize)];
+        l = 1.f;
       }
-      if (valid && p < a.M && lsum > 0.f) {
-        const int i = p / a.G, gq = p % a.G;
-        a.out[((static_cast<long long>(b) * a.R + i) * a.Hq + kvh * a.G + gq) * kD + kl] =
-            __float2bfloat16_rn(acc / lsum);
+      float mmax = m;
+#pragma unroll
+      for (int w = 16; w >= 1; w >>= 1) mmax = fmaxf(mmax, __shfl_xor_sync(0xffffffffu, mmax, w));
+      const float f = m == -INFINITY ? 0.f : ex2(m - mmax);
+      float lsum = f * l;
+#pragma unroll
+      for (int w = 16; w >= 1; w >>= 1) lsum += __shfl_xor_sync(0xffffffffu, lsum, w);
+      if (lane < csize + n_new) s_w[rr * kWRow + lane] = f;
+      if (lane == 0) s_w[rr * kWRow + kWRow - 1] = lsum > 0.f ? 1.f / lsum : 0.f;
+    }
+    named_bar_sync(2, kSoftThreads);
+#pragma unroll 1
+    for (int idx = st; idx < rpc * kD; idx += kSoftThreads) {
+      const int rr = idx / kD, d = idx % kD;
+      const int row = mrow0 + rr;
+      const int p = mblock * kRows + row;
+      const float* w = s_w + rr * kWRow;
+      float acc = 0.f;
+#pragma unroll 4
+      for (int c = 0; c < csize; ++c) acc = fmaf(w[c], recv[(c * rpc + rr) * kRowF + d], acc);
+      const __nv_bfloat16* nv = reinterpret_cast<const __nv_bfloat16*>(smem + kOffNewV) + d;
+#pragma unroll 4
+      for (int n = 0; n < n_new; ++n) acc = fmaf(w[csize + n], __bfloat162float(nv[n * kD]), acc);
+      const float inv_l = w[kWRow - 1];
+      if (valid && p < a.M && inv_l > 0.f) {
+        const int i = gdiv(p), gq = (p - gdiv(p) * a.G);
+        a.out[((static_cast<long long>(b) * a.R + i) * a.Hq + kvh * a.G + gq) * kD + d] =
+            __float2bfloat16_rn(acc * inv_l);
       }
     }
-  }
-  if (kFused && rank == 0 && warp >= 2) {
-    // every CTA of the cluster read the raw query rows before its main loop
-    // (the cluster barrier above is behind all of them): store the rotated rows
-    for (int idx = threadIdx.x - 64; idx < a.M * 16 && valid; idx += 128) {
-      const int row = idx / 16, c = idx % 16;
-      const int p = mblock * kRows + row;
-      if (p >= a.M) continue;
-      const int i = p / a.G, gq = p % a.G;
-      const uint4 v = *reinterpret_cast<const uint4*>(smem + kOffQ + (c >> 3) * kQHalf + row * 128 +
-                                                      (((c & 7) ^ (row & 7)) << 4));
-      *reinterpret_cast<uint4*>(a.qw + ((static_cast<long long>(b) * a.R + i) * a.Hq + kvh * a.G + gq) * kD +
-                                c * 8) = v;
+    if (st < csize) asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+    if (kFused && valid) {
+      // every CTA of the cluster read the raw rows before its main loop (the
+      // cluster barrier above is behind all of them): store the rotated query
+      // rows (rank 0), and append the new key / value rows and store the
+      // rotated keys back (last rank)
+      if (rank == 0) {
+#pragma unroll 1
+        for (int idx = st; idx < kRows * 16; idx += kSoftThreads) {
+          const int row = idx / 16, c = idx % 16;
+          const int p = mblock * kRows + row;
+          if (p >= a.M) continue;
+          const uint4 v = *reinterpret_cast<const uint4*>(smem + kOffQ + (c >> 3) * kQHalf + row * 128 +
+                                                          (((c & 7) ^ (row & 7)) << 4));
+          *reinterpret_cast<uint4*>(a.qw + ((static_cast<long long>(b) * a.R + gdiv(p)) * a.Hq + kvh * a.G +
+                                            (p - gdiv(p) * a.G)) * kD + c * 8) = v;
+        }
+      }
+      if (rank == csize - 1) {
+#pragma unroll 1
+        for (int idx = st; idx < a.R * 16; idx += kSoftThreads) {
+          const int i = idx / 16, c = idx % 16;
+          const long long src = ((static_cast<long long>(b) * a.R + i) * a.Hkv + kvh) * kD + c * 8;
+          const long long dst = ((static_cast<long long>(b) * a.Hkv + kvh) * a.cap + L_pre + i) * kD + c * 8;
+          const uint4 kr = *reinterpret_cast<const uint4*>(smem + kOffNewK + i * kNewRow + c * 16);
+          *reinterpret_cast<uint4*>(a.kc + dst) = kr;
+          *reinterpret_cast<uint4*>(a.k_new + src) = kr;
+          *reinterpret_cast<uint4*>(a.vc + dst) =
+              *reinterpret_cast<const uint4*>(smem + kOffNewV + i * kNewRow + c * 16);
+        }
+      }
     }
   }
   tc_fence_before();
   __syncthreads();  // every tensor-memory read is done
-  if (kFused && threadIdx.x == 0) {
-    // the last CTA of the scene to finish advances its length: every CTA of
-    // the scene read len[b] before it got here
-    const uint32_t total = gridDim.x * gridDim.y;
-    if (atomicAdd(&a.ticket[b], 1u) == total - 1) {
-      if (valid) a.len[b] = L_pre + a.R;
-      a.ticket[b] = 0;
-    }
-  }
   if (warp == 1) {
     tc_fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
@@ -866,9 +1043,8 @@ template <bool kFused>
 static sd_status launch_tc(const sd_kv_cache* cache, const void* q_for_map, const TcArgs& a,
                     const RopeTable& tab, int cs, bool pdl, cudaStream_t stream) {
   const int B = cache->batch, Hkv = cache->n_kv_heads, cap = cache->capacity;
-  CUtensorMap k128, v128, k32, v32, qm;
+  CUtensorMap k128, v128, qm;
   if (!make_map(&k128, cache->k, cap, B * Hkv, 128) || !make_map(&v128, cache->v, cap, B * Hkv, 128) ||
-      !make_map(&k32, cache->k, cap, B * Hkv, 32) || !make_map(&v32, cache->v, cap, B * Hkv, 32) ||
       !make_q_map(&qm, q_for_map, B, a.R, a.Hq, a.G))
     return SD_ERR_CUDA;
   cudaLaunchConfig_t cfg = {};
@@ -885,7 +1061,7 @@ static sd_status launch_tc(const sd_kv_cache* cache, const void* q_for_map, cons
   cfg.stream = stream;
   cfg.attrs = attr;
   cfg.numAttrs = pdl ? 2 : 1;
-  if (cudaLaunchKernelEx(&cfg, verify_attn_tc_kernel<kFused>, k128, v128, k32, v32, qm, a, tab) !=
+  if (cudaLaunchKernelEx(&cfg, verify_attn_tc_kernel<kFused>, k128, v128, qm, a, tab) !=
       cudaSuccess) {
     (void)cudaGetLastError();
     return SD_ERR_CUDA;
@@ -918,6 +1094,7 @@ sd_status sd_internal_verify_attention_tc(const void* q, const sd_kv_cache* cach
   a.Hkv = Hkv;
   a.G = Hq / Hkv;
   a.M = a.G * R;
+  a.inv_g = 1.0f / static_cast<float>(a.G);
   a.cap = cache->capacity;
   a.n_mblocks = 1;
   a.scale_log2 = scale_log2;
@@ -933,6 +1110,7 @@ sd_status sd_internal_verify_layer_tc(void* q, void* k_new, const void* v_new, c
                                       cudaStream_t stream, bool* handled) {
   *handled = false;
   const int B = cache->batch, Hkv = cache->n_kv_heads;
+  if (R > kMaxNew) return SD_OK;  // the new rows are held in shared memory
   const int cs = serving_cluster(B, R, Hq, Hkv, cache->head_dim, cache->capacity);
   if (cs <= 0) return SD_OK;
   TcArgs a = {};
@@ -952,6 +1130,7 @@ sd_status sd_internal_verify_layer_tc(void* q, void* k_new, const void* v_new, c
   a.Hkv = Hkv;
   a.G = Hq / Hkv;
   a.M = a.G * R;
+  a.inv_g = 1.0f / static_cast<float>(a.G);
   a.cap = cache->capacity;
   a.n_mblocks = 1;
   a.scale_log2 = scale_log2;

@@ -114,10 +114,12 @@ __device__ __forceinline__ float sd_frac_turns(float p, float hi, float lo) {
   return f + fmaf(p, lo, e);
 }
 
-// Rotate 4 adjacent pairs (8 bf16 packed in w[4]) of head-vector chunk `vec`
-// (pairs 4*vec .. 4*vec+3) at coordinates p3 (t, h, w).
-__device__ __forceinline__ void sd_rope_rotate8(uint32_t (&w)[4], int vec, const int (&p3)[3],
-                                                const RopeTable& tab);
+// (cos, sin) of the rotation angle theta_d * p of pair d at coordinate p.
+__device__ __forceinline__ float2 sd_rope_cs(float p, int d, const RopeTable& tab) {
+  float s, c;
+  sincospif(2.0f * sd_frac_turns(p, tab.tau_hi[d], tab.tau_lo[d]), &s, &c);
+  return make_float2(c, s);
+}
 
 // Two floats -> packed bf16x2 (round to nearest even), lo in the low half.
 __device__ __forceinline__ uint32_t sd_pack_bf16x2(float lo, float hi) {
@@ -125,18 +127,21 @@ __device__ __forceinline__ uint32_t sd_pack_bf16x2(float lo, float hi) {
   return *reinterpret_cast<uint32_t*>(&v);
 }
 
+// Rotate one pair (x, y) packed as bf16x2 by the angle with cosine c, sine s.
+__device__ __forceinline__ uint32_t sd_rope_pair(uint32_t w, float c, float s) {
+  const float x = sd_bf16_lo(w);
+  const float y = sd_bf16_hi(w);
+  return sd_pack_bf16x2(fmaf(x, c, -y * s), fmaf(x, s, y * c));
+}
+
+// Rotate 4 adjacent pairs (8 bf16 packed in w[4]) of head-vector chunk `vec`
+// (pairs 4*vec .. 4*vec+3) at coordinates p3 (t, h, w).
 __device__ __forceinline__ void sd_rope_rotate8(uint32_t (&w)[4], int vec, const int (&p3)[3],
                                                 const RopeTable& tab) {
 #pragma unroll
   for (int j = 0; j < 4; ++j) {
     const int d = vec * 4 + j;
-    const float p = static_cast<float>(p3[tab.axis[d]]);
-    float s, c;
-    sincospif(2.0f * sd_frac_turns(p, tab.tau_hi[d], tab.tau_lo[d]), &s, &c);
-    const float x = sd_bf16_lo(w[j]);
-    const float y = sd_bf16_hi(w[j]);
-    const float xr = fmaf(x, c, -y * s);
-    const float yr = fmaf(x, s, y * c);
-    w[j] = sd_pack_bf16x2(xr, yr);
+    const float2 cs = sd_rope_cs(static_cast<float>(p3[tab.axis[d]]), d, tab);
+    w[j] = sd_rope_pair(w[j], cs.x, cs.y);
   }
 }
