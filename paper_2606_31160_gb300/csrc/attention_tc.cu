@@ -731,8 +731,10 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
       for (int j = 0; j < 16; ++j) o_f[j] = 0.f;
     }
-    // every MMA of this CTA is done: its ring may now receive peers' partials
-    cluster_arrive();
+    // every MMA of this CTA is done: its ring may now receive peers' partials.
+    // Relaxed: no data passes through this barrier (the tensor core's reads of
+    // the ring are complete, PVDONE was waited), it only orders execution.
+    asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
     // stage the partial row-major: row j = [O(128) | m | l | pad], 528 bytes;
     // the l terms of the 128 key lanes go through the (free) P buffers
     float* send = reinterpret_cast<float*>(smem + kSend);
@@ -744,18 +746,22 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     named_bar_sync(2, kSoftThreads);
     {
-      const int r = st >> 3, part = st & 7;  // 8 threads per row, 16 key lanes each
-      const float4* src = reinterpret_cast<const float4*>(lbuf + r * 128 + part * 16);
-      float l = 0.f;
+      // softmax warp w sums rows 4w .. 4w+3: 512 contiguous bytes per load
+      const int w = warp - 2;
+      const float4* src = reinterpret_cast<const float4*>(lbuf + w * 4 * 128);
+      float l4[4];
 #pragma unroll
-      for (int q4 = 0; q4 < 4; ++q4) {
-        const float4 x = src[q4];
-        l += (x.x + x.y) + (x.z + x.w);
+      for (int i = 0; i < 4; ++i) {
+        const float4 x = src[i * 32 + lane];
+        l4[i] = (x.x + x.y) + (x.z + x.w);
       }
-      l += __shfl_xor_sync(0xffffffffu, l, 1);
-      l += __shfl_xor_sync(0xffffffffu, l, 2);
-      l += __shfl_xor_sync(0xffffffffu, l, 4);
-      if (part == 0) {
+#pragma unroll
+      for (int sh = 16; sh >= 1; sh >>= 1)
+#pragma unroll
+        for (int i = 0; i < 4; ++i) l4[i] += __shfl_xor_sync(0xffffffffu, l4[i], sh);
+      if (lane < 4) {
+        const int r = 4 * w + lane;
+        const float l = lane == 0 ? l4[0] : lane == 1 ? l4[1] : lane == 2 ? l4[2] : l4[3];
         send[r * kRowF + kD] = n_tiles > 0 ? row_ref[r] : -INFINITY;
         send[r * kRowF + kD + 1] = l;
       }
