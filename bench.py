@@ -86,13 +86,14 @@ def kernel_source_hash():
         return hashlib.sha256(f.read()).hexdigest()
 
 
-def ncu_traffic():
-    """DRAM bytes per verify-attention launch from the committed ncu summary,
-    or None when the kernel source changed since the counters were taken."""
+def ncu_traffic(kernel="verify_layer"):
+    """DRAM bytes per launch of the given kernel from the committed ncu
+    summary, or None when the kernel source changed since the counters were
+    taken."""
     path = os.path.join(ROOT, "profiles", "ncu_traffic.json")
     try:
         with open(path) as f:
-            d = json.load(f)["verify_attention"]
+            d = json.load(f)[kernel]
         if d.get("src_sha256") == kernel_source_hash():
             return float(d["dram_bytes_per_launch"])
     except Exception:

@@ -191,10 +191,12 @@ size_t sd_verify_layer_workspace(int B, int R, int Hq, int Hkv, int D, int capac
  *   overlap on the device -- calls flagged SD_LAYER_PREFIX_EARLY overlap
  *   their predecessor, so give each layer its own workspace.
  *   flags: SD_LAYER_PREFIX_EARLY declares that the kernel issued just before
- *   this call on the stream writes neither this layer's cache nor its len
- *   (true for every layer but the first of a verify pass, when the layers are
- *   issued back to back). The call is then a programmatic dependent launch
- *   that streams the cached prefix while its predecessor still runs.
+ *   this call on the stream writes neither this layer's cache, nor its len,
+ *   nor pos (true for every layer but the first of a verify pass, when the
+ *   layers are issued back to back and the positions were written before the
+ *   pass). The call is then a programmatic dependent launch that reads len and
+ *   pos and streams the cached prefix while its predecessor still runs; q,
+ *   k_new and v_new are read only after the predecessor has completed.
  * For head_dim 128 and G * R <= 32 this is one tcgen05 kernel; other shapes
  * run the three kernels in sequence. A scene whose append would pass the
  * capacity sets SD_DEVERR_KV_OVERFLOW and is left untouched.

@@ -49,3 +49,65 @@ def test_attention_kernel_paths(kernel):
                          text=True, timeout=600)
     assert res.returncode == 0, res.stdout + res.stderr
     assert "OK" in res.stdout
+
+
+def _planted(seed, plants, fused):
+    """B=1, 32 q / 8 KV heads x 128, L=4096 prefix, R=8: key n of KV head h // 4
+    is set to alpha * (rotated) q[i][h], so that row i of head h scores it far
+    above everything in the first tile of its split."""
+    import numpy as np
+    import torch
+    import oracle
+    from paper_2606_31160_gb300 import sd, workloads
+    rng = np.random.default_rng(seed)
+    B, R, Hq, Hkv, D, L = 1, 8, 32, 8, 128, 4096
+    cap = L + R + 8
+    q = workloads.to_bf16(rng.standard_normal((B, R, Hq, D)))
+    k = rng.standard_normal((B, Hkv, cap, D)).astype(np.float32)
+    v = rng.standard_normal((B, Hkv, cap, D)).astype(np.float32)
+    k_new = workloads.to_bf16(rng.standard_normal((B, R, Hkv, D)))
+    v_new = workloads.to_bf16(rng.standard_normal((B, R, Hkv, D)))
+    pos = np.repeat(np.arange(L + 1, L + 1 + R, dtype=np.int32)[None, :, None], 3, axis=2)
+    sections = (16, 24, 24)
+    q64 = q.float().numpy().astype(np.float64)
+    q_rot = oracle.mrope_apply(q64, pos[:, :, None, :], sections, 0, 1e6) if fused else q64
+    for (h, i, n, alpha) in plants:
+        k[0, h // (Hq // Hkv), n] = alpha * q_rot[0, i, h] / np.linalg.norm(q_rot[0, i, h]) * 12.0
+    if fused:
+        k[:, :, L:] = np.nan  # stale rows past the prefix
+        v[:, :, L:] = np.nan
+        cache = sd.KVCache(workloads.to_bf16(k).cuda(), workloads.to_bf16(v).cuda(),
+                           torch.full((B,), L, dtype=torch.int32).cuda())
+        qd, kd = q.cuda(), k_new.cuda()
+        out = sd.verify_layer(qd, kd, v_new.cuda(), torch.from_numpy(pos).cuda(), sections, cache, 0, 1e6)
+        q_ref = qd
+    else:
+        cache = sd.KVCache(workloads.to_bf16(k).cuda(), workloads.to_bf16(v).cuda(),
+                           torch.full((B,), L + R, dtype=torch.int32).cuda())
+        q_ref = q.cuda()
+        out = sd.verify_attention(q_ref, cache)
+    torch.cuda.synchronize()
+    ref = oracle.verify_attention(q_ref.cpu().float().numpy().astype(np.float64),
+                                  cache.k.cpu().float().numpy().astype(np.float64),
+                                  cache.v.cpu().float().numpy().astype(np.float64), cache.len.cpu().numpy())
+    return out.cpu().float().numpy().astype(np.float64), ref, sd.get_device_error()
+
+
+@pytest.mark.parametrize("fused", [False, True])
+def test_fixed_reference_fallback_pass(fused):
+    # a planted key scores ~17 * alpha in log2 units (|k| = 12 alpha along q,
+    # |q| ~ 11.3, scale log2(e) / sqrt(128)): alpha 6 puts it ~100 above the
+    # first tile's maximum (beyond the 64 one pass allows, so its split runs the
+    # fallback pass), alpha 2.5 ~40 above (kept by the single pass), alpha -6
+    # far below; keys in later tiles of splits 0, 3 and 7
+    import numpy as np
+    from tests.helpers import ATTN_ATOL
+    plants = [(0, 0, 300, 6.0), (5, 3, 2000, 6.0), (31, 7, 4000, 6.0), (12, 2, 1700, 2.5),
+              (13, 2, 130, -6.0)]
+    out, ref, err = _planted(7, plants, fused)
+    assert err == 0
+    assert np.isfinite(out).all()
+    e = np.abs(out - ref).max()
+    assert e <= ATTN_ATOL, e
+    # the planted rows are dominated by their key (the output is its value row)
+    assert np.abs(ref[0, 0, 0]).max() > 0.5
