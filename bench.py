@@ -161,16 +161,39 @@ def dist_env():
     return world, rank, local
 
 
+# ------------------------------------------------------------- ranks
+# The verify step shards by scene: every rank runs whole scenes of its own
+# (weak scaling, no data-path collective). These helpers are the only
+# multi-rank logic; tests/test_dist_gloo.py runs them on two gloo ranks.
+def scenes_of_rank(scenes_per_rank, rank):
+    """Global scene indices a rank verifies: a contiguous block of its own."""
+    return list(range(rank * scenes_per_rank, (rank + 1) * scenes_per_rank))
+
+
+def max_over_ranks(value, world, device="cpu"):
+    """The slowest rank's time (the job's time): all-reduce MAX."""
+    t = torch.tensor([float(value)], dtype=torch.float64, device=device)
+    if world > 1:
+        import torch.distributed as dist
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def aggregate_gbs(bytes_per_rank, world, ms_per_step):
+    """Whole-job throughput: the bytes every rank verified / the slowest rank's time."""
+    return bytes_per_rank * world / (ms_per_step * 1e-3) / 1e9
+
+
 # ------------------------------------------------------------- workload
 class Step:
     """Device-resident inputs and outputs of one verify step (one scene)."""
 
-    def __init__(self, device):
+    def __init__(self, device, scene=0):
         from paper_2606_31160_gb300 import sd, workloads
         self.sd = sd
         self.device = device
         gen_t0 = time.time()
-        self.cases = [workloads.target_layer(B=1, layer=l, ell=[3]) for l in range(LAYERS)]
+        self.cases = [workloads.target_layer(B=1, layer=l, ell=[3], scene=scene) for l in range(LAYERS)]
         self.gen_s = time.time() - gen_t0
         c0 = self.cases[0]
         # host copies (pinned) of the per-step inputs, for the end-to-end leg
@@ -362,7 +385,7 @@ def main():
     build.build()
     sd.lib()
 
-    st = Step(device)
+    st = Step(device, scene=scenes_of_rank(1, rank)[0])
     # eager warm-up (sets kernel attributes before any capture), then graphs
     for _ in range(2):
         st.run()
@@ -397,11 +420,7 @@ def main():
     torch.cuda.synchronize()
     if world > 1:
         dist.barrier()
-    ms_total = e0.elapsed_time(e1)
-    t = torch.tensor([ms_total], dtype=torch.float64, device=device)
-    if world > 1:
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-    ms_total = float(t.item())
+    ms_total = max_over_ranks(e0.elapsed_time(e1), world, device)
     ms_step = ms_total / args.steps
 
     # ---- dominant kernel: the fused verify layer, its 36 launches alone
@@ -430,11 +449,7 @@ def main():
         st.d2h()
     a1.record(stream)
     a1.synchronize()
-    ms_e2e = a0.elapsed_time(a1) / e2e_steps
-    te = torch.tensor([ms_e2e], dtype=torch.float64, device=device)
-    if world > 1:
-        dist.all_reduce(te, op=dist.ReduceOp.MAX)
-    ms_e2e = float(te.item())
+    ms_e2e = max_over_ranks(a0.elapsed_time(a1) / e2e_steps, world, device)
     assert sd.get_device_error() == 0
 
     if rank != 0:
@@ -444,8 +459,7 @@ def main():
         return
 
     peak, peak_kind = measured_peaks()
-    bytes_step = step_bytes(1) * world
-    value = bytes_step / (ms_step * 1e-3) / 1e9
+    value = aggregate_gbs(step_bytes(1), world, ms_step)
     achieved = layer_bytes(1) / (ms_layer_launch * 1e-3) / 1e9
     traffic = ncu_traffic()
     cpu_gbs, cpu_layers, cpu_s = time_oracle(args.cpu_budget)
@@ -501,7 +515,7 @@ def main():
                       % (cpu_layers, cpu_s),
         },
         "e2e": {
-            "value": round(bytes_step / (ms_e2e * 1e-3) / 1e9, 2),
+            "value": round(aggregate_gbs(step_bytes(1), world, ms_e2e), 2),
             "unit": "GB/s",
             "ms_per_step": round(ms_e2e, 5),
             "h2d_bytes_per_step": st.h2d_bytes,

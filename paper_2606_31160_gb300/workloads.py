@@ -161,17 +161,19 @@ def tiny(layer=0):
     return case
 
 
-def target_layer(B=1, layer=0, ell=None):
+def target_layer(B=1, layer=0, ell=None, scene=0):
     """8B-class target layer: 32 q / 8 KV heads x 128, sections [16,24,24], base 1e6.
     Prefix L=4096 = 4 cameras x 896 patches (28x32 grid, t = camera) + 512 text
     tokens at 32..543; K=7 query rows at 544..551. Greedy logits bf16 N(0,2) over
-    V=151936 with the matching-prefix length uniform in 0..7."""
+    V=151936 with the matching-prefix length uniform in 0..7. `scene` selects an
+    independent draw (another driving clip): scene 0 is the default stream."""
     K, V, L = 7, 151936, 4096
     R = K + 1
+    off = 10000 * int(scene)
     qpos = np.broadcast_to(text_positions(544, R)[None], (B, R, 3))
     case = verify_case(TARGET_LAYER, B=B, Hq=32, Hkv=8, D=128, prefix=[L] * B, K=K,
-                       sections=(16, 24, 24), base=1e6, query_pos=qpos, layer=layer)
-    rng = philox(TARGET_LAYER, 100 + layer)
+                       sections=(16, 24, 24), base=1e6, query_pos=qpos, layer=layer + off)
+    rng = philox(TARGET_LAYER, 100 + layer + off)
     if ell is None:
         ell = rng.integers(0, K + 1, size=B)
     logits, draft, target = planted_logits(rng, B, R, V, 2.0, "bf16", ell)
