@@ -22,6 +22,7 @@ graph and replayed. Multi-GPU: one independent replica per rank (scenes are
 independent: weak scaling, no data-path collective).
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+    python bench.py --sweep     # sd_verify_attention over the batched sweep grid
 """
 
 import argparse
@@ -362,6 +363,12 @@ def main():
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--cpu-budget", type=float, default=12.0, help="seconds of oracle time (rank 0)")
+    ap.add_argument("--sweep", action="store_true",
+                    help="time sd_verify_attention over the batched sweep grid (B x L x K) and "
+                         "print one JSON line per point; prints no bench line")
+    ap.add_argument("--sweep-b", type=int, nargs="*", default=None, help="restrict the sweep's batch sizes")
+    ap.add_argument("--sweep-l", type=int, nargs="*", default=None, help="restrict the sweep's prefix lengths")
+    ap.add_argument("--sweep-k", type=int, nargs="*", default=None, help="restrict the sweep's draft lengths")
     ap.add_argument("--only", choices=["attention", "layer", "accept", "step"], default=None,
                     help="profiling mode: run one kernel family eagerly `steps` times on the "
                          "target-layer workload (for ncu captures); prints no bench line")
@@ -374,6 +381,8 @@ def main():
         return reference_arm(args, world, rank)
     if args.only:
         return profile_only(args)
+    if args.sweep:
+        return sweep(args)
 
     import torch.distributed as dist
     torch.cuda.set_device(local)
@@ -528,6 +537,60 @@ def main():
     if world > 1:
         dist.barrier()
         dist.destroy_process_group()
+
+
+SWEEP_B, SWEEP_L, SWEEP_K = (1, 8, 32), (2048, 4096, 8192, 16384), (1, 2, 4, 8, 16)
+
+
+def sweep(args):
+    """sd_verify_attention over the batched sweep (B scenes, ragged L_b ~
+    U[0.75 L, L], 32 q / 8 KV x 128, bf16): per point, the rotated rows are
+    appended and the attention launch is timed in a CUDA graph over enough
+    distinct caches that one replay streams > 2 x L2 (inputs larger than L2).
+    Algorithmic bytes: K and V of every key (L_b + R per scene and KV head),
+    plus Q read and O written."""
+    from paper_2606_31160_gb300 import build, sd, workloads
+    build.build()
+    sd.lib()
+    torch.cuda.set_device(0)
+    device = torch.device("cuda", 0)
+    peak, peak_kind = measured_peaks()
+    l2_bytes = 129 * 2 ** 20
+    for B in args.sweep_b or SWEEP_B:
+        for Lp in args.sweep_l or SWEEP_L:
+            for Kp in args.sweep_k or SWEEP_K:
+                R_ = Kp + 1
+                prefix, q, k_new, v_new, pos, kc, vc, cap = workloads.sweep_case_device(B, Lp, Kp, device)
+                nbytes = int(sum(int(p) + R_ for p in prefix)) * HKV * D * 2 * 2 + 2 * B * R_ * HQ * D * 2
+                copies = max(1, min(64, -(-(2 * l2_bytes) // nbytes)))
+                lens = torch.from_numpy(np.asarray(prefix, dtype=np.int32)).to(device)
+                sd.rope_apply(q, k_new, pos, SECTIONS, 0, BASE)
+                caches = []
+                for c in range(copies):
+                    cache = sd.KVCache(kc if c == 0 else kc.clone(), vc if c == 0 else vc.clone(), lens.clone())
+                    sd.kv_append(cache, k_new, v_new)
+                    caches.append(cache)
+                del kc, vc
+                outs = [torch.empty_like(q) for _ in range(copies)]
+                ws = [sd.workspace(sd.attention_workspace_bytes(B, R_, HQ, HKV, D, cap), device)
+                      for _ in range(copies)]
+
+                def launches():
+                    for c in range(copies):
+                        sd.verify_attention(q, caches[c], out=outs[c], ws=ws[c])
+
+                g = capture(launches)
+                ms_one = time_graph(g, 3) / copies
+                reps = max(5, min(2000, int(100.0 / max(ms_one * copies, 1e-3))))
+                ms = time_graph(g, reps) / copies
+                gbs = nbytes / (ms * 1e-3) / 1e9
+                assert sd.get_device_error() == 0
+                print(json.dumps({"sweep": {"B": B, "L": Lp, "K": Kp, "sum_keys": int(sum(prefix)) + B * R_,
+                                            "us": round(ms * 1e3, 3), "gbs": round(gbs, 1),
+                                            "frac": round(gbs / peak, 4), "peak": peak, "peak_kind": peak_kind,
+                                            "bytes": nbytes, "copies": copies}}), flush=True)
+                del caches, outs, ws, g
+                torch.cuda.empty_cache()
 
 
 def profile_only(args):

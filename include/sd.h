@@ -166,6 +166,20 @@ sd_status sd_verify_attention(const void* q, const sd_kv_cache* cache, void* out
                               int R, int Hq, float scale, void* workspace, size_t ws_bytes,
                               sd_stream_t stream);
 
+/*
+ * Cluster size of the tcgen05 verify-attention kernel (sd_verify_attention
+ * and sd_verify_layer, head_dim 128, G*R <= 128): one thread-block cluster of
+ * `cluster_size` CTAs per (scene, KV head) splits that head's keys evenly and
+ * merges the partial softmax states in distributed shared memory (the split-L
+ * form of Eq. verify). 0 (the default) lets every call choose from the
+ * occupancy of each size and the capacity; 1, 2, 4, 6, 8 or 16 forces that
+ * size for later calls on every device (a size of which no cluster fits on
+ * the device falls back to the automatic choice). Process-wide, host-only, no
+ * device work; results are the same for every size up to fp32 rounding order.
+ * Returns SD_ERR_INVALID_ARG for any other value.
+ */
+sd_status sd_set_cluster_size(int cluster_size);
+
 /* sd_verify_layer flag: see below. */
 #define SD_LAYER_PREFIX_EARLY 1
 
@@ -197,8 +211,8 @@ size_t sd_verify_layer_workspace(int B, int R, int Hq, int Hkv, int D, int capac
  *   pass). The call is then a programmatic dependent launch that reads len and
  *   pos and streams the cached prefix while its predecessor still runs; q,
  *   k_new and v_new are read only after the predecessor has completed.
- * For head_dim 128 and G * R <= 32 this is one tcgen05 kernel; other shapes
- * run the three kernels in sequence. A scene whose append would pass the
+ * For head_dim 128, G * R <= 128 and R <= 16 this is one tcgen05 kernel;
+ * other shapes run the three kernels in sequence. A scene whose append would pass the
  * capacity sets SD_DEVERR_KV_OVERFLOW and is left untouched.
  */
 sd_status sd_verify_layer(void* q, void* k_new, const void* v_new, const int32_t* pos,

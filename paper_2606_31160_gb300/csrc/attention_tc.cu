@@ -1,27 +1,35 @@
 // K3 on the 5th-generation tensor cores (tcgen05 + TMEM): verify attention
 // of the K + 1 new rows against the cached prefix (Eq. verify, Sec. 2.2),
-// for head_dim 128 and up to 32 packed query rows per KV head, and the fused
+// for head_dim 128 and up to 128 packed query rows per KV head, and the fused
 // verify layer (M-RoPE of Sec. 2.3 / Sec. 3.2 + the KV append of Eq. commit +
 // the attention) on the same machinery.
 //
 // The packed query tile is small (G*R = 32 rows for 32 q / 8 KV heads and
 // K = 7), so both products run TRANSPOSED, with the 128-wide dimension on the
 // MMA's M side and no padding waste:
-//     S^T[128 keys][32 rows] = K_tile[128 keys][128 d] . Q^T      (K-major A, B)
-//     O^T[128 d][32 rows]   += V_tile^T[128 d][128 keys] . P^T     (MN-major A, B)
-// Both accumulators live in tensor memory (S double-buffered): 96 columns.
+//     S^T[128 keys][kR rows] = K_tile[128 keys][128 d] . Q^T      (K-major A, B)
+//     O^T[128 d][kR rows]   += V_tile^T[128 d][128 keys] . P^T     (MN-major A, B)
+// kR = 32 (G*R <= 32) or 64 (G*R <= 64, and m-blocks of 64 rows up to 128);
+// an N = 64 product costs about what an N = 32 one does. Both accumulators
+// live in tensor memory (S double-buffered): 3 kR columns.
 //
 // Warp roles in a CTA (320 threads):
-//   warp 0      TMA producer: 128-key stages of K and V (128B-swizzled boxes)
+//   warp 0      TMA producer: 128-key tiles of K and V (128B-swizzled boxes)
+//               into a K ring and a V ring of kS slots each. 32 rows: 3 slots,
+//               a tile's K and V load together once the slot's previous PV
+//               is done. 64 rows (less shared memory left): 2 slots, a K slot
+//               is refilled once its S product is done and a V slot once its
+//               PV product is, so S still runs two tiles ahead.
 //   warp 1      allocates tensor memory; one lane issues every tcgen05.mma.
 //               S runs two tiles ahead: per tile it issues PV(t) and commits
-//               "PV(t) done" (stage t is free), then S(t+2) and commits
-//               "S(t+2) ready" (which also implies PV(t) done, so the softmax
-//               needs no other wait). Two commits a tile: each drains the
-//               MMA pipe for ~180 cycles.
+//               "PV(t) done" (V slot free), then S(t+2) and commits
+//               "S(t+2) ready" (K slot free; implies PV(t) done, so the
+//               softmax needs no other wait). Two commits a tile: each drains
+//               the MMA pipe for ~180 cycles.
 //   warps 2..9  softmax: thread (t, h) owns key lane t of S^T and query rows
-//               16h .. 16h+15; P = exp2(S - ref) goes to shared memory as
-//               P^T (64-byte swizzled, MN-major), two 16-byte stores a thread.
+//               h kR/2 .. h kR/2 + kR/2 - 1; P = exp2(S - ref) goes to shared
+//               memory as P^T (MN-major; 64-byte swizzle for 32 rows, 128-byte
+//               for 64), 16-byte stores.
 //
 // Softmax with a fixed reference. The reference of a row is the exact maximum
 // of the CTA's first tile; every later tile uses it unchanged, so the loop has
@@ -44,6 +52,7 @@
 
 #include <math.h>
 #include <stdlib.h>
+#include <atomic>
 #include <mutex>
 
 SD_DEFINE_ERROR_ACCESSOR(sd_take_error_attention_tc)
@@ -51,55 +60,70 @@ SD_DEFINE_ERROR_ACCESSOR(sd_take_error_attention_tc)
 namespace {
 
 constexpr int kD = 128;         // head dim
-constexpr int kRows = 32;       // packed query rows per CTA (N of both MMAs)
 constexpr int kStageKeys = 128; // M of S^T
-constexpr int kStages = 3;
 constexpr int kHalf = kStageKeys * 128;     // one 64-column half of a 128-key tile (16 KB)
-constexpr int kKV = 2 * kHalf;              // K (or V) tile of a stage (32 KB)
-constexpr int kStage = 2 * kKV;             // 64 KB
-constexpr int kRing = kStages * kStage;     // 192 KB
-constexpr int kQHalf = kRows * 128;         // 4 KB
-constexpr int kQ = 2 * kQHalf;              // 8 KB
-constexpr int kPRow = kRows * 2;            // one key of P^T: 32 rows in bf16 (64 B)
-constexpr int kP = kStageKeys * kPRow;      // one P^T buffer (8 KB)
+constexpr int kKV = 2 * kHalf;              // one K (or V) tile of 128 keys (32 KB)
 constexpr int kMaxNew = 16;                 // new rows the fused kernel takes
 constexpr int kNewRow = kD * 2;             // one new key / value row (256 B)
 constexpr int kSoftWarps = 8;
 constexpr int kSoftThreads = 32 * kSoftWarps;
 constexpr int kThreads = 64 + kSoftThreads;
-constexpr int kTmemCols = 128;              // S0 | S1 | O  (32 columns each)
 constexpr uint32_t kSpinLimit = 1u << 20;
 constexpr float kSlack = 64.f;              // log2 units a score may exceed its reference by
-
-// shared memory layout (offsets from the 1024-aligned base)
-constexpr int kOffQ = kRing;
-constexpr int kOffP = kOffQ + kQ;           // also the rotation table before the loop
-constexpr int kOffNewK = kOffP + 2 * kP;
-constexpr int kOffNewV = kOffNewK + kMaxNew * kNewRow;
-constexpr int kOffBar = kOffNewV + kMaxNew * kNewRow;
-// barriers: full[3] p_full[2] s_ready[2] pv_done[3] q_full recv decide
-constexpr int kNumBars = 3 + 2 + 2 + 3 + 1 + 1 + 1;
-constexpr int kOffMisc = (kOffBar + kNumBars * 8 + 15) / 16 * 16;  // tmem slot, excess flag, decision, len
-constexpr int kOffRowA = kOffMisc + 16;           // [32] per-row results (reductions)
-constexpr int kOffRef = kOffRowA + kRows * 4;     // [32] per-row references
-constexpr int kSmemBytes = kOffRef + kRows * 4 + 1024;
-static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
-static_assert(kOffQ % 1024 == 0 && kOffP % 1024 == 0 && kOffNewK % 16 == 0 && kOffNewV % 16 == 0 &&
-                  kOffBar % 8 == 0 && kOffRowA % 16 == 0 && kOffRef % 16 == 0,
-              "alignment of the shared-memory regions (swizzle atoms, vector accesses, mbarriers)");
-static_assert(kMaxNew * 64 * 8 <= 2 * kP, "rotation table fits the P buffers");
-
-// cluster merge buffers (in the ring, free once this CTA's last MMA is done):
-// a partial row is [O(128) | m | l | 2 pad] fp32 = 528 bytes
+// a merged partial row is [O(128) | m | l | 2 pad] fp32 = 528 bytes
 constexpr int kRowF = kD + 4;
 constexpr int kRowBytes = kRowF * 4;
-constexpr int kSend = 0;                            // this CTA's 32 rows
-constexpr int kRecv = 20 * 1024;                    // 32 slots received from the peers
-constexpr int kNewS = 40 * 1024;                    // new-key scores of the merged rows
-constexpr int kWRow = 2 * 16 + 4;                   // merge weights of a row: csize + R, 1 / l
-constexpr int kMergeW = kNewS + kRows * kMaxNew * 4;
-static_assert(kRecv >= kRows * kRowBytes && kRecv + kRows * kRowBytes <= kNewS, "merge buffers");
-static_assert(kMergeW + kRows * kWRow * 4 <= kRing, "merge buffers");
+constexpr int kWRow = 2 * 16 + 4;           // merge weights of a row: csize + R, 1 / l
+constexpr int round_up(int x, int m) { return (x + m - 1) / m * m; }
+
+// Everything that depends on the packed query rows per CTA (kR = 32 or 64:
+// the N of both MMAs). A softmax thread owns kR / 2 rows of one key lane.
+template <int kR>
+struct Cfg {
+  static_assert(kR == 32 || kR == 64, "row tile");
+  static constexpr int kRows = kR;
+  static constexpr int kRpt = kR / 2;                       // rows per softmax thread
+  // K and V rings of kStages tiles each: a K slot is free once its S product
+  // is done, a V slot once its PV product is
+  static constexpr int kStages = kR == 32 ? 3 : 2;
+  static constexpr int kRingV = kStages * kKV;              // V slots follow the K slots
+  static constexpr int kRing = 2 * kStages * kKV;
+  static constexpr int kQHalf = kR * 128;
+  static constexpr int kQ = 2 * kQHalf;
+  static constexpr int kPRow = kR * 2;                      // one key of P^T in bf16
+  static constexpr int kP = kStageKeys * kPRow;             // one P^T buffer
+  // P^T is MN-major: 64-byte swizzle for 32 rows (a 64-byte key row), 128-byte
+  // swizzle for 64 rows; 8-key groups are kPRow * 8 bytes apart
+  static constexpr uint64_t kPLayout = kR == 32 ? 4 : 2;
+  static constexpr int kTmemCols = kR == 32 ? 128 : 256;    // S0 | S1 | O, kR columns each
+  // shared memory layout (offsets from the 1024-aligned base)
+  static constexpr int kOffQ = kRing;
+  static constexpr int kOffP = kOffQ + kQ;                  // also the rotation table before the loop
+  static constexpr int kOffNewK = kOffP + 2 * kP;
+  static constexpr int kOffNewV = kOffNewK + kMaxNew * kNewRow;
+  static constexpr int kOffBar = kOffNewV + kMaxNew * kNewRow;
+  // barriers: full_k[S] full_v[S] p_full[2] s_ready[S] pv_done[S] q_full recv decide
+  static constexpr int kNumBars = 4 * kStages + 5;
+  static constexpr int kOffMisc = round_up(kOffBar + kNumBars * 8, 16);  // tmem slot, excess, decision, len
+  static constexpr int kOffRowA = kOffMisc + 16;            // [kR] per-row results (reductions)
+  static constexpr int kOffRef = kOffRowA + kR * 4;         // [kR] per-row references
+  static constexpr int kOffLim = kOffRef + kR * 4;          // [kR] per-row causal key limits
+  static constexpr int kSmemBytes = kOffLim + kR * 4 + 1024;
+  static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
+  static_assert(kOffQ % 1024 == 0 && kOffP % 1024 == 0 && kP % 1024 == 0 && kOffNewK % 16 == 0 &&
+                    kOffNewV % 16 == 0 && kOffBar % 8 == 0 && kOffRowA % 16 == 0 && kOffRef % 16 == 0,
+                "alignment of the shared-memory regions (swizzle atoms, vector accesses, mbarriers)");
+  static_assert(kMaxNew * 64 * 8 <= 2 * kP, "rotation table fits the P buffers");
+  static_assert(kR * 128 * 4 <= 2 * kP, "row reductions fit the P buffers");
+  // cluster merge buffers (in the rings, free once this CTA's last MMA is done)
+  static constexpr int kSend = 0;                           // this CTA's kR rows
+  static constexpr int kRecv = round_up(kR * kRowBytes, 1024);
+  // slots for ceil(kR / c) rows from each of c ranks, c in {1, 2, 4, 6, 8, 16}
+  static constexpr int kRecvSlots = kR == 32 ? 36 : 66;
+  static constexpr int kNewS = round_up(kRecv + kRecvSlots * kRowBytes, 1024);  // new-key scores
+  static constexpr int kMergeW = kNewS + kR * kMaxNew * 4;
+  static_assert(kMergeW + kR * kWRow * 4 <= kRing, "merge buffers");
+};
 
 __device__ __forceinline__ uint32_t smem_addr(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -198,8 +222,6 @@ constexpr uint32_t umma_idesc(int M, int N, int a_mn_major, int b_mn_major) {
          (static_cast<uint32_t>(b_mn_major) << 16) | (static_cast<uint32_t>(N >> 3) << 17) |
          (static_cast<uint32_t>(M >> 4) << 24);
 }
-constexpr uint32_t kIdescS = umma_idesc(128, kRows, 0, 0);
-constexpr uint32_t kIdescO = umma_idesc(128, kRows, 1, 1);
 
 __device__ __forceinline__ void umma(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc,
                                      int accumulate) {
@@ -234,26 +256,29 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
 }
 
 // Per-row reduction (max or sum) over the 128 key lanes of a CTA, for the 256
-// softmax threads: thread (key lane kl, rows row0 .. row0 + 15) contributes
-// v[j] to row row0 + j. The values pass through buf ([32 rows][128] fp32,
-// 16 KB, free while this runs); the 32 results land in out[32]. Called by
-// all softmax threads; compact on purpose (it runs once or twice a launch).
-template <bool kMax>
-__device__ __forceinline__ void rows_reduce(const float (&v)[16], int kl, int row0, int st, float* buf,
+// softmax threads: thread (key lane kl, rows row0 .. row0 + kN - 1) contributes
+// v[j] to row row0 + j. The values pass through buf ([2 kN rows][128] fp32,
+// free while this runs); the 2 kN results land in out[]. Called by all
+// softmax threads; compact on purpose (it runs once or twice a launch).
+template <bool kMax, int kN>
+__device__ __forceinline__ void rows_reduce(const float (&v)[kN], int kl, int row0, int st, float* buf,
                                             float* out) {
+  constexpr int kRowsAll = 2 * kN;
+  constexpr int kPer = kSoftThreads / kRowsAll;  // threads per row (8 or 4)
+  constexpr int kVals = 128 / kPer;              // values each of them reads (16 or 32)
 #pragma unroll
-  for (int j = 0; j < 16; ++j) buf[(row0 + j) * 128 + kl] = v[j];
+  for (int j = 0; j < kN; ++j) buf[(row0 + j) * 128 + kl] = v[j];
   asm volatile("bar.sync 2, 256;" ::: "memory");
-  const int r = st >> 3, part = st & 7;  // 8 threads per row, 16 values each
-  const float4* src = reinterpret_cast<const float4*>(buf + r * 128 + part * 16);
+  const int r = st / kPer, part = st % kPer;
+  const float4* src = reinterpret_cast<const float4*>(buf + r * 128 + part * kVals);
   float acc = kMax ? -INFINITY : 0.f;
 #pragma unroll
-  for (int q = 0; q < 4; ++q) {
+  for (int q = 0; q < kVals / 4; ++q) {
     const float4 x = src[q];
     acc = kMax ? fmaxf(acc, fmaxf(fmaxf(x.x, x.y), fmaxf(x.z, x.w))) : acc + ((x.x + x.y) + (x.z + x.w));
   }
 #pragma unroll
-  for (int w = 1; w < 8; w <<= 1) {
+  for (int w = 1; w < kPer; w <<= 1) {
     const float o = __shfl_xor_sync(0xffffffffu, acc, w);
     acc = kMax ? fmaxf(acc, o) : acc + o;
   }
@@ -275,7 +300,7 @@ struct TcArgs {
   uint32_t* ticket;         // [B] per-scene CTA tickets (zeroed, re-armed)
   int early;                // prefix, len and pos may be read before the dependency wait
   int R, Hq, Hkv, G, M, cap, n_mblocks;
-  float inv_g;              // 1 / G: p / G == int((p + 0.5) / G) exactly for the p < 32 used here
+  float inv_g;              // 1 / G: p / G == int((p + 0.5) / G) exactly for the p < 128 used here
   float scale_log2;
 };
 
@@ -286,43 +311,56 @@ __device__ __forceinline__ void griddep_launch() {
 
 // ------------------------------------------------------------------ kernel
 // kFused = false: attention over a cache that already holds the R new rows,
-// with the rotated query rows loaded by TMA.
+// with the rotated query rows read from a.q.
 // kFused = true: the whole verify layer -- M-RoPE of the raw query and key
 // rows, the KV append and the attention -- with len[b] the prefix length.
 // Prefix tiles, len and pos are independent of the kernel that precedes this
 // one in the stream (for every layer but the first of a step), so when
 // a.early is set they are read before the programmatic-dependency wait.
-template <bool kFused>
+// Grid: (cluster size, Hkv * n_mblocks, B); m-block mb takes packed query rows
+// mb * kR .. mb * kR + kR - 1.
+template <int kR, bool kFused>
 __global__ void __launch_bounds__(kThreads, 1)
     verify_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k128,
-                          const __grid_constant__ CUtensorMap tm_v128,
-                          const __grid_constant__ CUtensorMap tm_q, const TcArgs a,
+                          const __grid_constant__ CUtensorMap tm_v128, const TcArgs a,
                           const RopeTable tab) {
+  using C = Cfg<kR>;
+  constexpr int kS = C::kStages;
+  constexpr int kRpt = C::kRpt;
+  constexpr uint32_t kIdescS = umma_idesc(128, kR, 0, 0);
+  constexpr uint32_t kIdescO = umma_idesc(128, kR, 1, 1);
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
   const uint32_t base = smem_addr(smem);
-  const uint32_t qs = base + kOffQ;
-  auto bar = [&](int i) { return base + kOffBar + 8u * i; };
-  // barrier indices; T counts tiles over both passes. SREADY(T) (two slots)
-  // and PVDONE(T) (one slot per stage) are tcgen05.commit arrivals. A slot's
-  // next phase cannot complete before its waiter has seen the current one:
-  // S(T + 2) needs PFULL(T), which follows the wait for SREADY(T); PV(T + 3)
-  // needs tile T + 3, loaded only after the wait for PVDONE(T).
-  auto FULL = [&](int s) { return bar(s); };
-  auto PFULL = [&](int b) { return bar(3 + b); };
-  auto SREADY = [&](int T) { return bar(5 + (T & 1)); };
-  auto PVDONE = [&](int T) { return bar(7 + T % kStages); };
-  auto sready_parity = [](int T) { return static_cast<uint32_t>((T >> 1) & 1); };
-  auto pvdone_parity = [](int T) { return static_cast<uint32_t>((T / kStages) & 1); };
-  const uint32_t QFULL = bar(10);
-  const uint32_t RECV = bar(11);    // the cluster merge's incoming partial rows
-  const uint32_t DECIDE = bar(12);  // whether the range runs a second time
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + kOffMisc);
-  int* s_excess = reinterpret_cast<int*>(smem + kOffMisc + 4);
-  int* s_redo = reinterpret_cast<int*>(smem + kOffMisc + 8);
-  float* row_a = reinterpret_cast<float*>(smem + kOffRowA);  // [32] reduction results
-  float* row_ref = reinterpret_cast<float*>(smem + kOffRef); // [32] references
+  const uint32_t qs = base + C::kOffQ;
+  auto bar = [&](int i) { return base + C::kOffBar + 8u * i; };
+  // barrier indices; T counts tiles over both passes. SREADY(T) and PVDONE(T)
+  // (one slot per ring stage) are tcgen05.commit arrivals. A slot's next
+  // phase cannot complete before each of its waiters has seen the current
+  // one: S(T + kS) needs the K tile loaded after the producer's wait for
+  // SREADY(T), and is issued after PV(T + kS - 2), which needs PFULL from the
+  // softmax's tile T + kS - 2 >= T; PV(T + kS) needs the V tile loaded after
+  // the producer's wait for PVDONE(T), and the softmax waits for PVDONE only
+  // once a pass, on its last tile.
+  // With 32 rows (3 slots) a tile's K and V arrive together on FULLK, loaded
+  // once PV(T - 3) is done; with 64 rows (2 slots) each has its own barrier.
+  constexpr bool kSplit = kR == 64;
+  auto FULLK = [&](int s) { return bar(s); };
+  auto FULLV = [&](int s) { return kSplit ? bar(kS + s) : bar(s); };
+  auto PFULL = [&](int b) { return bar(2 * kS + b); };
+  auto SREADY = [&](int T) { return bar(2 * kS + 2 + T % kS); };
+  auto PVDONE = [&](int T) { return bar(3 * kS + 2 + T % kS); };
+  auto ring_parity = [](int T) { return static_cast<uint32_t>((T / kS) & 1); };
+  const uint32_t QFULL = bar(4 * kS + 2);
+  const uint32_t RECV = bar(4 * kS + 3);    // the cluster merge's incoming partial rows
+  const uint32_t DECIDE = bar(4 * kS + 4);  // whether the range runs a second time
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::kOffMisc);
+  int* s_excess = reinterpret_cast<int*>(smem + C::kOffMisc + 4);
+  int* s_redo = reinterpret_cast<int*>(smem + C::kOffMisc + 8);
+  float* row_a = reinterpret_cast<float*>(smem + C::kOffRowA);  // [kR] reduction results
+  float* row_ref = reinterpret_cast<float*>(smem + C::kOffRef); // [kR] references
+  int* row_lim = reinterpret_cast<int*>(smem + C::kOffLim);      // [kR] last key a row sees
 
   auto gdiv = [&](int p) { return __float2int_rz((static_cast<float>(p) + 0.5f) * a.inv_g); };
   const int rank = blockIdx.x;
@@ -334,15 +372,14 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int lane = threadIdx.x & 31;
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kStages; ++s) {
-      mbar_init(FULL(s), 1);
+    for (int s = 0; s < kS; ++s) {
+      mbar_init(FULLK(s), 1);
+      if (kSplit) mbar_init(FULLV(s), 1);
+      mbar_init(SREADY(s), 1);
       mbar_init(PVDONE(s), 1);
     }
-    for (int i = 0; i < 2; ++i) {
-      mbar_init(PFULL(i), kSoftWarps);
-      mbar_init(SREADY(i), 1);
-    }
-    mbar_init(QFULL, kFused ? 1 : 2);  // (producer's expect_tx +) one softmax thread
+    for (int i = 0; i < 2; ++i) mbar_init(PFULL(i), kSoftWarps);
+    mbar_init(QFULL, 1);  // one softmax thread, once the query tile is stored
     mbar_init(RECV, 1);
     mbar_init(DECIDE, 1);
     *s_excess = 0;
@@ -352,12 +389,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 1) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
                      smem_addr(tmem_slot)),
-                 "r"(kTmemCols)
+                 "r"(C::kTmemCols)
                  : "memory");
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
   if (kFused && !a.early) griddep_wait();  // len, pos and the prefix may come from the previous kernel
-  int* s_len = reinterpret_cast<int*>(smem + kOffMisc + 12);
+  int* s_len = reinterpret_cast<int*>(smem + C::kOffMisc + 12);
   if (threadIdx.x == 0) {
     const int len0 = a.len[b];
     *s_len = len0;
@@ -377,8 +414,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  const uint32_t tmem_s = tmem;          // S buffer b at column 32 * b
-  const uint32_t tmem_o = tmem + 64;     // O^T
+  const uint32_t tmem_s = tmem;          // S buffer b at column kR * b
+  const uint32_t tmem_o = tmem + 2 * kR; // O^T
 
   int n_keys, L_pre;
   bool valid;
@@ -405,38 +442,40 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == 0) {
     // -------------------------------------------------------------- producer
-    if (lane == 0) {
-      if (!kFused && n_tiles > 0) {
-        // the packed query tile first: box (64 d, G heads, R rows) lands as
-        // rows p = i * G + g of 128 bytes, the B operand's K-major layout
-        mbar_expect_tx(QFULL, static_cast<uint32_t>(2 * a.M * 128));
-        for (int h = 0; h < 2; ++h)
-          tma_load_3d(qs + h * kQHalf, &tm_q, QFULL, h * 64, kvh * a.G, b * a.R);
-      }
-      if (n_tiles > 0) {
-        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_k128)) : "memory");
-        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_v128)) : "memory");
-        const int z = b * a.Hkv + kvh;
-        for (int pass = 0; pass < 2; ++pass) {
-          if (pass == 1) {
-            // every MMA of pass 0 is done when the decision is out
-            mbar_wait(DECIDE, 0);
-            if (!*reinterpret_cast<volatile int*>(s_redo)) break;
-          }
-          for (int t = 0; t < n_tiles; ++t) {
-            const int T = pass * n_tiles + t;
-            const int s = T % kStages;
-            // stage s last held tile T - 3 (all of pass 0 is done before pass 1 starts)
-            if (t >= kStages) mbar_wait(PVDONE(T - kStages), pvdone_parity(T - kStages));
-            // a whole 128-row box even for a short last tile: keys past the
-            // range are masked, rows past the capacity arrive zero-filled
-            const int y0 = key_begin + t * kStageKeys;
-            const uint32_t kst = base + s * kStage, vst = kst + kKV;
-            mbar_expect_tx(FULL(s), static_cast<uint32_t>(kStage));
+    if (lane == 0 && n_tiles > 0) {
+      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_k128)) : "memory");
+      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_v128)) : "memory");
+      const int z = b * a.Hkv + kvh;
+      for (int pass = 0; pass < 2; ++pass) {
+        if (pass == 1) {
+          // every MMA of pass 0 is done when the decision is out
+          mbar_wait(DECIDE, 0);
+          if (!*reinterpret_cast<volatile int*>(s_redo)) break;
+        }
+        for (int t = 0; t < n_tiles; ++t) {
+          const int T = pass * n_tiles + t;
+          const int s = T % kS;
+          // a whole 128-row box even for a short last tile: keys past the
+          // range are masked, rows past the capacity arrive zero-filled
+          const int y0 = key_begin + t * kStageKeys;
+          // slot s last held tile T - kS (all of pass 0 is done before pass 1)
+          const uint32_t kst = base + s * kKV, vst = base + C::kRingV + s * kKV;
+          if (kSplit) {
+            if (t >= kS) mbar_wait(SREADY(T - kS), ring_parity(T - kS));
+            mbar_expect_tx(FULLK(s), static_cast<uint32_t>(kKV));
+#pragma unroll
+            for (int h = 0; h < 2; ++h) tma_load_3d(kst + h * kHalf, &tm_k128, FULLK(s), h * 64, y0, z);
+            if (t >= kS) mbar_wait(PVDONE(T - kS), ring_parity(T - kS));
+            mbar_expect_tx(FULLV(s), static_cast<uint32_t>(kKV));
+#pragma unroll
+            for (int h = 0; h < 2; ++h) tma_load_3d(vst + h * kHalf, &tm_v128, FULLV(s), h * 64, y0, z);
+          } else {
+            if (t >= kS) mbar_wait(PVDONE(T - kS), ring_parity(T - kS));
+            mbar_expect_tx(FULLK(s), static_cast<uint32_t>(2 * kKV));
 #pragma unroll
             for (int h = 0; h < 2; ++h) {
-              tma_load_3d(kst + h * kHalf, &tm_k128, FULL(s), h * 64, y0, z);
-              tma_load_3d(vst + h * kHalf, &tm_v128, FULL(s), h * 64, y0, z);
+              tma_load_3d(kst + h * kHalf, &tm_k128, FULLK(s), h * 64, y0, z);
+              tma_load_3d(vst + h * kHalf, &tm_v128, FULLK(s), h * 64, y0, z);
             }
           }
         }
@@ -450,10 +489,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0 && n_tiles > 0) {
       mbar_wait(QFULL, 0);
       // base descriptors; a K step only moves the start address (low field, no carry)
-      const uint64_t dK0 = umma_desc(base, 16, 1024);              // K tile: K-major
-      const uint64_t dV0 = umma_desc(base + kKV, kHalf, 1024);     // V^T: MN-major
-      const uint64_t dQ = umma_desc(qs, 16, 1024);                 // Q: K-major
-      const uint64_t dP0 = umma_desc(base + kOffP, 0, 512, 4);     // P^T: MN-major, 64B swizzle
+      const uint64_t dK0 = umma_desc(base, 16, 1024);                     // K tile: K-major
+      const uint64_t dV0 = umma_desc(base + C::kRingV, kHalf, 1024);      // V^T: MN-major
+      const uint64_t dQ = umma_desc(qs, 16, 1024);                        // Q: K-major
+      // P^T: MN-major, one swizzle atom wide (kR rows), 8-key groups 8 * kPRow apart
+      const uint64_t dP0 = umma_desc(base + C::kOffP, 0, 8 * C::kPRow, C::kPLayout);
       // Two issue sites with every K-step offset a compile-time constant (one
       // 64-bit add per descriptor): a rolled or shared issue loop measured
       // ~1.8 us slower per layer.
@@ -468,25 +508,27 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (t >= 0) {
             const int T = T0 + t;
             mbar_wait(PFULL(T & 1), (T >> 1) & 1);
+            if (kSplit) mbar_wait(FULLV(T % kS), ring_parity(T));  // else waited before S(T)
             tc_fence_after();
-            const uint64_t dv = dV0 + static_cast<uint64_t>(((T % kStages) * kStage) >> 4);
-            const uint64_t dp = dP0 + static_cast<uint64_t>(((T & 1) * kP) >> 4);
+            const uint64_t dv = dV0 + static_cast<uint64_t>(((T % kS) * kKV) >> 4);
+            const uint64_t dp = dP0 + static_cast<uint64_t>(((T & 1) * C::kP) >> 4);
 #pragma unroll
             for (int kk = 0; kk < 8; ++kk)
-              umma(tmem_o, dv + (kk * 2048 >> 4), dp + (kk * 1024 >> 4), kIdescO, (t > 0 || kk > 0) ? 1 : 0);
+              umma(tmem_o, dv + (kk * 2048 >> 4), dp + (kk * 16 * C::kPRow >> 4), kIdescO,
+                   (t > 0 || kk > 0) ? 1 : 0);
             umma_commit(PVDONE(T));
           }
           if (t + 2 < n_tiles) {
             // S(T) reuses the S buffer of tile T - 2, read before PFULL(T - 2)
-            const int T = T0 + t + 2, st_ = T % kStages;
-            mbar_wait(FULL(st_), (T / kStages) & 1);
+            const int T = T0 + t + 2, st_ = T % kS;
+            mbar_wait(FULLK(st_), ring_parity(T));
             tc_fence_after();
-            const uint64_t dk = dK0 + static_cast<uint64_t>((st_ * kStage) >> 4);
-            const uint32_t ts = tmem_s + 32 * (T & 1);
+            const uint64_t dk = dK0 + static_cast<uint64_t>((st_ * kKV) >> 4);
+            const uint32_t ts = tmem_s + kR * (T & 1);
 #pragma unroll
             for (int kk = 0; kk < 8; ++kk)
               umma(ts, dk + (((kk >> 2) * kHalf + (kk & 3) * 32) >> 4),
-                   dQ + (((kk >> 2) * kQHalf + (kk & 3) * 32) >> 4), kIdescS, kk > 0 ? 1 : 0);
+                   dQ + (((kk >> 2) * C::kQHalf + (kk & 3) * 32) >> 4), kIdescS, kk > 0 ? 1 : 0);
             umma_commit(SREADY(T));
           }
         }
@@ -498,74 +540,68 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else {
     // -------------------------------------------------------------- softmax
     const int st = threadIdx.x - 64;       // 0..255
-    const int half = (warp - 2) >> 2;      // query rows 16*half .. 16*half + 15
+    const int half = (warp - 2) >> 2;      // query rows kRpt*half .. kRpt*half + kRpt - 1
     const int quarter = warp & 3;          // TMEM lane quarter of this warp
     const int kl = quarter * 32 + lane;    // key lane of S^T / d lane of O^T
     const uint32_t lane_off = static_cast<uint32_t>(quarter * 32) << 16;
-    const int row0 = 16 * half;            // first query row of this thread
-    const float2* cs_tab = reinterpret_cast<const float2*>(smem + kOffP);  // [R][64] (cos, sin)
-    if (!kFused) {
-      // query rows past M stay zero (the TMA box covers rows 0..M-1 only)
-      for (int idx = st; idx < (kRows - a.M) * 16; idx += kSoftThreads) {
-        const int row = a.M + idx / 16, c = idx % 16;
-        st_shared_v4(qs + (c >> 3) * kQHalf + row * 128 + (c & 7) * 16, 0u, 0u, 0u, 0u);
-      }
-      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-      named_bar_sync(2, kSoftThreads);
-      if (st == 0) mbar_arrive(QFULL);
-    } else {
+    const int row0 = kRpt * half;          // first query row of this thread
+    const float2* cs_tab = reinterpret_cast<const float2*>(smem + C::kOffP);  // [R][64] (cos, sin)
+    if (kFused && valid) {
       // rotation table of the R new positions: (cos, sin) per (row, pair)
-      if (valid) {
-        float2* tabw = reinterpret_cast<float2*>(smem + kOffP);
+      float2* tabw = reinterpret_cast<float2*>(smem + C::kOffP);
 #pragma unroll 1
-        for (int idx = st; idx < a.R * 64; idx += kSoftThreads) {
-          const int i = idx >> 6, d = idx & 63;
-          const int32_t pc = a.pos[(static_cast<long long>(b) * a.R + i) * 3 + tab.axis[d]];
-          tabw[idx] = sd_rope_cs(static_cast<float>(pc), d, tab);
-        }
+      for (int idx = st; idx < a.R * 64; idx += kSoftThreads) {
+        const int i = idx >> 6, d = idx & 63;
+        const int32_t pc = a.pos[(static_cast<long long>(b) * a.R + i) * 3 + tab.axis[d]];
+        tabw[idx] = sd_rope_cs(static_cast<float>(pc), d, tab);
       }
-      named_bar_sync(2, kSoftThreads);  // the rotation table is complete
-      // this thread's pieces: query chunks (row, 16-byte chunk c) u = 0, 1 and
-      // one chunk of a new key / value row
-      const __nv_bfloat16* q_src[2];
-      int q_cs[2];
-      bool q_ok[2];
+    }
+    if (kFused) named_bar_sync(2, kSoftThreads);  // the rotation table is complete
+    {
+      // the packed query tile: this thread's 16-byte chunks (row, chunk c),
+      // rows past M zero; in the fused layer also one chunk of a new key and
+      // value row
+      constexpr int kQc = kR * 16 / kSoftThreads;
+      const __nv_bfloat16* q_src[kQc];
+      int q_cs[kQc];
+      bool q_ok[kQc];
 #pragma unroll
-      for (int u = 0; u < 2; ++u) {
-        const int idx = st + u * kSoftThreads, p = mblock * kRows + (idx >> 4), c = idx & 15;
+      for (int u = 0; u < kQc; ++u) {
+        const int idx = st + u * kSoftThreads, p = mblock * kR + (idx >> 4), c = idx & 15;
         const int i = gdiv(p);
         q_ok[u] = valid && p < a.M;
-        q_src[u] = a.qw + ((static_cast<long long>(b) * a.R + i) * a.Hq + kvh * a.G + (p - i * a.G)) * kD + c * 8;
+        q_src[u] = (kFused ? a.qw : a.q) +
+                   ((static_cast<long long>(b) * a.R + i) * a.Hq + kvh * a.G + (p - i * a.G)) * kD + c * 8;
         q_cs[u] = i * 64 + c * 4;
       }
-      const bool has_kv = valid && st < a.R * 16;
+      const bool has_kv = kFused && valid && st < a.R * 16;
       const long long kv_src = ((static_cast<long long>(b) * a.R + (st >> 4)) * a.Hkv + kvh) * kD + (st & 15) * 8;
-      // Iteration 0 runs BEFORE the dependency wait on whatever the rows hold:
-      // it brings this code into the instruction cache and the rows into L2,
-      // and iteration 1 overwrites everything it stored. The loads bypass L1
-      // (.cg) so that iteration 1 cannot hit a line read before the wait.
+      // Fused: iteration 0 runs BEFORE the dependency wait on whatever the
+      // rows hold: it brings this code into the instruction cache and the rows
+      // into L2, and iteration 1 overwrites everything it stored. The loads
+      // bypass L1 (.cg) so that iteration 1 cannot hit a line read before the wait.
 #pragma unroll 1
-      for (int it = 0; it < 2; ++it) {
-        if (it == 1 && a.early) griddep_wait();  // the raw rows come from earlier kernels
-        uint4 qv[2], kv = make_uint4(0, 0, 0, 0), vv = make_uint4(0, 0, 0, 0);
+      for (int it = kFused ? 0 : 1; it < 2; ++it) {
+        if (kFused && it == 1 && a.early) griddep_wait();  // the raw rows come from earlier kernels
+        uint4 qv[kQc], kv = make_uint4(0, 0, 0, 0), vv = make_uint4(0, 0, 0, 0);
 #pragma unroll
-        for (int u = 0; u < 2; ++u)
+        for (int u = 0; u < kQc; ++u)
           qv[u] = q_ok[u] ? __ldcg(reinterpret_cast<const uint4*>(q_src[u])) : make_uint4(0, 0, 0, 0);
         if (has_kv) {
           kv = __ldcg(reinterpret_cast<const uint4*>(a.k_new + kv_src));
           vv = __ldcg(reinterpret_cast<const uint4*>(a.v_new + kv_src));
         }
-        // M-RoPE of the packed query rows, straight into the swizzled tile
+        // (fused: M-RoPE of) the packed query rows, straight into the swizzled tile
 #pragma unroll
-        for (int u = 0; u < 2; ++u) {
+        for (int u = 0; u < kQc; ++u) {
           const int idx = st + u * kSoftThreads, row = idx >> 4, c = idx & 15;
           uint32_t w[4] = {qv[u].x, qv[u].y, qv[u].z, qv[u].w};
-          if (q_ok[u]) {
+          if (kFused && q_ok[u]) {
             const float2* cs = cs_tab + q_cs[u];
 #pragma unroll
             for (int j = 0; j < 4; ++j) w[j] = sd_rope_pair(w[j], cs[j].x, cs[j].y);
           }
-          st_shared_v4(qs + (c >> 3) * kQHalf + row * 128 + (((c & 7) ^ (row & 7)) << 4), w[0], w[1],
+          st_shared_v4(qs + (c >> 3) * C::kQHalf + row * 128 + (((c & 7) ^ (row & 7)) << 4), w[0], w[1],
                        w[2], w[3]);
         }
         // the new key rows (rotated) and value rows of this head
@@ -575,40 +611,49 @@ __global__ void __launch_bounds__(kThreads, 1)
           uint32_t w[4] = {kv.x, kv.y, kv.z, kv.w};
 #pragma unroll
           for (int j = 0; j < 4; ++j) w[j] = sd_rope_pair(w[j], cs[j].x, cs[j].y);
-          st_shared_v4(base + kOffNewK + i * kNewRow + c * 16, w[0], w[1], w[2], w[3]);
-          st_shared_v4(base + kOffNewV + i * kNewRow + c * 16, vv.x, vv.y, vv.z, vv.w);
+          st_shared_v4(base + C::kOffNewK + i * kNewRow + c * 16, w[0], w[1], w[2], w[3]);
+          st_shared_v4(base + C::kOffNewV + i * kNewRow + c * 16, vv.x, vv.y, vv.z, vv.w);
         }
       }
+      // causal limit of each packed row: row p = i * G + g is new row i and
+      // sees keys 0 .. L_prefix + i (Eq. verify's mask)
+      if (!kFused && st < kR) row_lim[st] = min(n_keys - a.R + gdiv(mblock * kR + st), n_keys - 1);
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
       named_bar_sync(2, kSoftThreads);  // Q is complete; the rotation table is no longer read
       if (st == 0) {
         mbar_arrive(QFULL);
         // every older kernel has finished: the next layer may launch
-        griddep_launch();
+        if (kFused) griddep_launch();
       }
     }
 
     const float sl = a.scale_log2;
-    float ref[16];  // reference per query row (log2 units), -inf: no key yet
-    float lp[16];   // per-row partial sums of this thread's key lane
-    float ex[16];   // largest score - reference seen
+    // The reference of a row (log2 units, -inf: no key yet) lives in row_ref;
+    // with 32 rows a thread also keeps its 16 in registers, with 64 rows it
+    // reloads them every tile (broadcast loads) to stay within the registers
+    // that 10 warps leave a thread.
+    constexpr bool kRefRegs = kR == 32;
+    float ref[kRefRegs ? kRpt : 1];
+    float lp[kRpt];   // per-row partial sums of this thread's key lane
+    float ex[kRpt];   // largest score - reference seen
 #pragma unroll
-    for (int j = 0; j < 16; ++j) {
-      ref[j] = -INFINITY;
+    for (int j = 0; j < kRpt; ++j) {
       lp[j] = 0.f;
       ex[j] = -INFINITY;
     }
+    ref[0] = -INFINITY;
     const int L_prefix = n_keys - a.R;
-    // per-key-lane masks of a tile: the key range, and the causal limit of the
-    // new rows that the standalone kernel's range contains
-    auto tile_mask = [&](int key0, bool (&ok)[16]) {
+    // per-key-lane mask of rows row0 + j0 .. row0 + j0 + 15 for a tile: the
+    // key range, and the causal limit of the new rows that the standalone
+    // kernel's range contains
+    auto tile_mask = [&](int key0, int j0, bool (&ok)[16]) {
       const int key = key0 + kl;
       const bool key_ok = key < key_end;
       const bool tail = !kFused && key0 + kStageKeys - 1 > L_prefix;
 #pragma unroll
       for (int j = 0; j < 16; ++j) {
         ok[j] = key_ok;
-        if (tail) ok[j] = ok[j] && key <= min(L_prefix + gdiv(mblock * kRows + row0 + j), n_keys - 1);
+        if (tail) ok[j] = ok[j] && key <= row_lim[row0 + j0 + j];
       }
     };
     if (n_tiles > 0) {
@@ -616,22 +661,27 @@ __global__ void __launch_bounds__(kThreads, 1)
       // which no P has used yet)
       mbar_wait(SREADY(0), 0);
       tc_fence_after();
-      uint32_t r[16];
-      tmem_ld16(tmem_s + row0 + lane_off, r);
-      bool ok[16];
-      tile_mask(key_begin, ok);
-      float v[16];
+      float v[kRpt];
 #pragma unroll
-      for (int j = 0; j < 16; ++j) v[j] = ok[j] ? __uint_as_float(r[j]) * sl : -INFINITY;
-      rows_reduce<true>(v, kl, row0, st, reinterpret_cast<float*>(smem + kOffP), row_ref);
-      const float4* rr4 = reinterpret_cast<const float4*>(row_ref + row0);
+      for (int j0 = 0; j0 < kRpt; j0 += 16) {
+        uint32_t r[16];
+        tmem_ld16(tmem_s + row0 + j0 + lane_off, r);
+        bool ok[16];
+        tile_mask(key_begin, j0, ok);
 #pragma unroll
-      for (int j4 = 0; j4 < 4; ++j4) {
-        const float4 x = rr4[j4];
-        ref[4 * j4 + 0] = x.x;
-        ref[4 * j4 + 1] = x.y;
-        ref[4 * j4 + 2] = x.z;
-        ref[4 * j4 + 3] = x.w;
+        for (int j = 0; j < 16; ++j) v[j0 + j] = ok[j] ? __uint_as_float(r[j]) * sl : -INFINITY;
+      }
+      rows_reduce<true>(v, kl, row0, st, reinterpret_cast<float*>(smem + C::kOffP), row_ref);
+      if (kRefRegs) {
+        const float4* rr4 = reinterpret_cast<const float4*>(row_ref + row0);
+#pragma unroll
+        for (int j4 = 0; j4 < (kRefRegs ? kRpt / 4 : 0); ++j4) {
+          const float4 x = rr4[j4];
+          ref[4 * j4 + 0] = x.x;
+          ref[4 * j4 + 1] = x.y;
+          ref[4 * j4 + 2] = x.z;
+          ref[4 * j4 + 3] = x.w;
+        }
       }
     }
     bool redo = false;
@@ -639,39 +689,60 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (pass == 1 && !redo) break;
       for (int t = 0; t < n_tiles; ++t) {
         const int T = pass * n_tiles + t;
-        const int bb = T & 1, s = T % kStages;
+        const int bb = T & 1, s = T % kS;
         const int key0 = key_begin + t * kStageKeys;
         const int key = key0 + kl;
-        mbar_wait(SREADY(T), sready_parity(T));  // S(T) is ready, and so PV(T - 2) is done
+        mbar_wait(SREADY(T), ring_parity(T));  // S(T) is ready, and so PV(T - 2) is done
         tc_fence_after();
-        uint32_t r[16];
-        tmem_ld16(tmem_s + 32 * bb + row0 + lane_off, r);
         const bool key_ok = key < key_end;
-        bool ok[16];
-        tile_mask(key0, ok);
-        // P = exp2(S * scale - ref) in bf16; l partials from the same rounded weights
-        uint32_t pw[8];
+        // P^T key row kl (its buffer's previous tile, T - 2, is done: see
+        // above): kRpt rows = kRpt / 8 16-byte chunks of 8 query rows, swizzled
+        const uint32_t prow = base + C::kOffP + bb * C::kP + kl * C::kPRow;
+        const int sw = kR == 32 ? (kl >> 1) & 3 : kl & 7;
 #pragma unroll
-        for (int j = 0; j < 16; j += 2) {
-          const float m0 = ref[j] == -INFINITY ? 0.f : ref[j];
-          const float m1 = ref[j + 1] == -INFINITY ? 0.f : ref[j + 1];
-          const float y0 = ok[j] ? fmaf(__uint_as_float(r[j]), sl, -m0) : -INFINITY;
-          const float y1 = ok[j + 1] ? fmaf(__uint_as_float(r[j + 1]), sl, -m1) : -INFINITY;
-          ex[j] = fmaxf(ex[j], y0);
-          ex[j + 1] = fmaxf(ex[j + 1], y1);
-          const uint32_t w = cvt_bf16x2(ex2(y0), ex2(y1));
-          pw[j >> 1] = w;
-          lp[j] += sd_bf16_lo(w);
-          lp[j + 1] += sd_bf16_hi(w);
+        for (int j0 = 0; j0 < kRpt; j0 += 16) {
+          uint32_t r[16];
+          tmem_ld16(tmem_s + kR * bb + row0 + j0 + lane_off, r);
+          bool ok[16];
+          tile_mask(key0, j0, ok);
+          float rc[16];
+#pragma unroll
+          for (int j = 0; j < 16; ++j) rc[j] = kRefRegs ? ref[(j0 + j) % (kRefRegs ? kRpt : 1)] : 0.f;
+          if (!kRefRegs) {
+            const float4* rr4 = reinterpret_cast<const float4*>(row_ref + row0 + j0);
+#pragma unroll
+            for (int j4 = 0; j4 < 4; ++j4) {
+              const float4 x = rr4[j4];
+              rc[4 * j4 + 0] = x.x;
+              rc[4 * j4 + 1] = x.y;
+              rc[4 * j4 + 2] = x.z;
+              rc[4 * j4 + 3] = x.w;
+            }
+          }
+          // P = exp2(S * scale - ref) in bf16; l partials from the same rounded weights
+          uint32_t pw[8];
+#pragma unroll
+          for (int j = 0; j < 16; j += 2) {
+            const float m0 = rc[j] == -INFINITY ? 0.f : rc[j];
+            const float m1 = rc[j + 1] == -INFINITY ? 0.f : rc[j + 1];
+            const float y0 = ok[j] ? fmaf(__uint_as_float(r[j]), sl, -m0) : -INFINITY;
+            const float y1 = ok[j + 1] ? fmaf(__uint_as_float(r[j + 1]), sl, -m1) : -INFINITY;
+            ex[j0 + j] = fmaxf(ex[j0 + j], y0);
+            ex[j0 + j + 1] = fmaxf(ex[j0 + j + 1], y1);
+            const uint32_t w = cvt_bf16x2(ex2(y0), ex2(y1));
+            pw[j >> 1] = w;
+            lp[j0 + j] += sd_bf16_lo(w);
+            lp[j0 + j + 1] += sd_bf16_hi(w);
+          }
+          const int ch = (row0 + j0) >> 3;
+          st_shared_v4(prow + ((ch ^ sw) << 4), pw[0], pw[1], pw[2], pw[3]);
+          st_shared_v4(prow + (((ch + 1) ^ sw) << 4), pw[4], pw[5], pw[6], pw[7]);
         }
-        // P^T key row kl (its buffer's previous tile, T - 2, is done: see above): 64 bytes = 4 chunks of 8 query rows, 64-byte swizzle
-        const uint32_t prow = base + kOffP + bb * kP + kl * kPRow;
-        const int sw = (kl >> 1) & 3;
-        st_shared_v4(prow + (((2 * half) ^ sw) << 4), pw[0], pw[1], pw[2], pw[3]);
-        st_shared_v4(prow + (((2 * half + 1) ^ sw) << 4), pw[4], pw[5], pw[6], pw[7]);
         if (!key_ok) {
-          // stale or foreign key row: zero its V row so 0 * NaN cannot reach O
-          const uint32_t vrow = base + s * kStage + kKV + half * kHalf + kl * 128;
+          // stale or foreign key row: zero its V row (this thread's 64-column
+          // half) so 0 * NaN cannot reach O, once the tile has landed
+          mbar_wait(FULLV(s), ring_parity(T));
+          const uint32_t vrow = base + C::kRingV + s * kKV + half * kHalf + kl * 128;
 #pragma unroll
           for (int c = 0; c < 8; ++c) st_shared_v4(vrow + c * 16, 0u, 0u, 0u, 0u);
         }
@@ -681,16 +752,15 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) mbar_arrive(PFULL(bb));
       }
       if (n_tiles > 0) {
-        // every MMA of the pass is done (the slot's previous phase, PV(Tl - 3),
-        // is implied by SREADY(Tl))
+        // every MMA of the pass is done (PVDONE's phases complete in order)
         const int Tl = pass * n_tiles + n_tiles - 1;
-        mbar_wait(PVDONE(Tl), pvdone_parity(Tl));
+        mbar_wait(PVDONE(Tl), ring_parity(Tl));
       }
       if (pass == 0) {
         // did any score exceed its reference by more than kSlack?
         bool over = false;
 #pragma unroll
-        for (int j = 0; j < 16; ++j) over |= ex[j] > kSlack;
+        for (int j = 0; j < kRpt; ++j) over |= ex[j] > kSlack;
         if (__any_sync(0xffffffffu, over) && lane == 0) atomicOr(s_excess, 1);
         named_bar_sync(2, kSoftThreads);
         redo = *reinterpret_cast<volatile int*>(s_excess) != 0;
@@ -701,104 +771,114 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (redo) {
           // second pass with the exact row maxima of the whole range (every
           // MMA is done: the P buffers are free)
-          rows_reduce<true>(ex, kl, row0, st, reinterpret_cast<float*>(smem + kOffP), row_a);
+          rows_reduce<true>(ex, kl, row0, st, reinterpret_cast<float*>(smem + C::kOffP), row_a);
 #pragma unroll
-          for (int j = 0; j < 16; ++j) {
-            const float e = row_a[row0 + j];
-            const float m0 = ref[j] == -INFINITY ? 0.f : ref[j];
-            ref[j] = e == -INFINITY ? -INFINITY : m0 + e;
+          for (int j = 0; j < kRpt; ++j) {
+            if (kRefRegs) {
+              const float e = row_a[row0 + j];
+              const float m0 = ref[j % (kRefRegs ? kRpt : 1)] == -INFINITY ? 0.f : ref[j % (kRefRegs ? kRpt : 1)];
+              ref[j % (kRefRegs ? kRpt : 1)] = e == -INFINITY ? -INFINITY : m0 + e;
+            }
             lp[j] = 0.f;
           }
-          if (quarter == 0 && lane < 16) {
+          if (quarter == 0 && lane < kRpt) {
             const float e = row_a[row0 + lane];
             const float m0 = row_ref[row0 + lane] == -INFINITY ? 0.f : row_ref[row0 + lane];
             row_ref[row0 + lane] = e == -INFINITY ? -INFINITY : m0 + e;
           }
+          if (!kRefRegs) named_bar_sync(2, kSoftThreads);  // row_ref is read by every thread
         }
       }
     }
 
     // ---- CTA partial: O^T (tensor memory) of this thread's d lane and rows,
     //      and the per-row m (reference) and l (sum over all 128 key lanes)
-    float o_f[16];
-    if (n_tiles > 0) {
-      tc_fence_after();
-      uint32_t o[16];
-      tmem_ld16(tmem_o + row0 + lane_off, o);
-#pragma unroll
-      for (int j = 0; j < 16; ++j) o_f[j] = __uint_as_float(o[j]);
-    } else {
-#pragma unroll
-      for (int j = 0; j < 16; ++j) o_f[j] = 0.f;
-    }
-    // every MMA of this CTA is done: its ring may now receive peers' partials.
+    // every MMA of this CTA is done: its rings may now receive peers' partials.
     // Relaxed: no data passes through this barrier (the tensor core's reads of
-    // the ring are complete, PVDONE was waited), it only orders execution.
-    asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
-    // stage the partial row-major: row j = [O(128) | m | l | pad], 528 bytes;
-    // the l terms of the 128 key lanes go through the (free) P buffers
-    float* send = reinterpret_cast<float*>(smem + kSend);
-    float* lbuf = reinterpret_cast<float*>(smem + kOffP);  // [32 rows][128 key lanes]
+    // the rings are complete, PVDONE was waited), it only orders execution.
+    // The partial is staged row-major: row j = [O(128) | m | l | pad], 528
+    // bytes; the l terms of the 128 key lanes go through the (free) P buffers.
+    float* send = reinterpret_cast<float*>(smem + C::kSend);
+    float* lbuf = reinterpret_cast<float*>(smem + C::kOffP);  // [kR rows][128 key lanes]
+    if (n_tiles > 0) tc_fence_after();
 #pragma unroll
-    for (int j = 0; j < 16; ++j) {
-      send[(row0 + j) * kRowF + kl] = o_f[j];
-      lbuf[(row0 + j) * 128 + kl] = lp[j];
+    for (int j0 = 0; j0 < kRpt; j0 += 16) {
+      uint32_t o[16];
+      if (n_tiles > 0) {
+        tmem_ld16(tmem_o + row0 + j0 + lane_off, o);
+      } else {
+#pragma unroll
+        for (int j = 0; j < 16; ++j) o[j] = 0u;
+      }
+      if (j0 == 0) asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+#pragma unroll
+      for (int j = 0; j < 16; ++j) {
+        send[(row0 + j0 + j) * kRowF + kl] = __uint_as_float(o[j]);
+        lbuf[(row0 + j0 + j) * 128 + kl] = lp[j0 + j];
+      }
     }
     named_bar_sync(2, kSoftThreads);
     {
-      // softmax warp w sums rows 4w .. 4w+3: 512 contiguous bytes per load
+      // softmax warp w sums rows kRw * w .. kRw * w + kRw - 1: 512 contiguous
+      // bytes per load
+      constexpr int kRw = kR / kSoftWarps;
       const int w = warp - 2;
-      const float4* src = reinterpret_cast<const float4*>(lbuf + w * 4 * 128);
-      float l4[4];
+      const float4* src = reinterpret_cast<const float4*>(lbuf + w * kRw * 128);
+      float lw[kRw];
 #pragma unroll
-      for (int i = 0; i < 4; ++i) {
+      for (int i = 0; i < kRw; ++i) {
         const float4 x = src[i * 32 + lane];
-        l4[i] = (x.x + x.y) + (x.z + x.w);
+        lw[i] = (x.x + x.y) + (x.z + x.w);
       }
 #pragma unroll
       for (int sh = 16; sh >= 1; sh >>= 1)
 #pragma unroll
-        for (int i = 0; i < 4; ++i) l4[i] += __shfl_xor_sync(0xffffffffu, l4[i], sh);
-      if (lane < 4) {
-        const int r = 4 * w + lane;
-        const float l = lane == 0 ? l4[0] : lane == 1 ? l4[1] : lane == 2 ? l4[2] : l4[3];
+        for (int i = 0; i < kRw; ++i) lw[i] += __shfl_xor_sync(0xffffffffu, lw[i], sh);
+      float l = lw[0];
+#pragma unroll
+      for (int i = 1; i < kRw; ++i) l = lane == i ? lw[i] : l;
+      if (lane < kRw) {
+        const int r = kRw * w + lane;
         send[r * kRowF + kD] = n_tiles > 0 ? row_ref[r] : -INFINITY;
         send[r * kRowF + kD + 1] = l;
       }
     }
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     named_bar_sync(2, kSoftThreads);
-    const int rpc = kRows / csize;
-    if (st == 0) mbar_expect_tx(RECV, static_cast<uint32_t>(csize * rpc * kRowBytes));
+    // rank c merges rows [c * rpc, c * rpc + rows_of(c)): rpc = ceil(kR / csize)
+    const int rpc = (kR + csize - 1) / csize;
+    auto rows_of = [&](int c) { return max(0, min(rpc, kR - c * rpc)); };
+    const int my_rows = rows_of(rank);
+    if (st == 0) mbar_expect_tx(RECV, static_cast<uint32_t>(csize * my_rows * kRowBytes));
     cluster_wait();  // every peer's ring is free to receive
-    if (st < csize) {
-      // thread c sends rows [c * rpc, (c + 1) * rpc) to rank c, into its slots [rank * rpc, ...)
-      bulk_copy_s2s(cluster_map(base + kRecv + rank * rpc * kRowBytes, st),
-                    base + kSend + st * rpc * kRowBytes, static_cast<uint32_t>(rpc * kRowBytes),
+    if (st < csize && rows_of(st) > 0) {
+      // thread c sends rank c's rows to rank c, into its slots [rank * rpc, ...)
+      bulk_copy_s2s(cluster_map(base + C::kRecv + rank * rpc * kRowBytes, st),
+                    base + C::kSend + st * rpc * kRowBytes, static_cast<uint32_t>(rows_of(st) * kRowBytes),
                     cluster_map(RECV, st));
       asm volatile("cp.async.bulk.commit_group;" ::: "memory");
     }
     const int mrow0 = rank * rpc;  // the rows this CTA merges
-    float* s_new = reinterpret_cast<float*>(smem + kNewS);  // [rpc][R] scores of the new keys
+    float* s_new = reinterpret_cast<float*>(smem + C::kNewS);  // [rpc][R] scores of the new keys
     if (kFused && valid) {
       // new-key scores (log2 units) of the merged rows, 8 threads per dot product;
       // query row p = i * G + g sees new keys 0..i (Eq. verify's causal mask)
       const int sub = lane & 7;
-      const int n_pairs = rpc * a.R;
+      const int n_pairs = my_rows * a.R;
 #pragma unroll 1
       for (int pr0 = (st >> 5) * 4; pr0 < n_pairs; pr0 += kSoftThreads / 8) {  // warp-uniform
         const int pr = min(pr0 + (lane >> 3), n_pairs - 1);
         const bool act = pr0 + (lane >> 3) < n_pairs;
         const int rr = pr / a.R, n = pr % a.R;
         const int row = mrow0 + rr;
-        const int p = mblock * kRows + row;
+        const int p = mblock * kR + row;
         float acc = 0.f;
 #pragma unroll
         for (int u = 0; u < 2; ++u) {
           const int c = 2 * sub + u;
-          const uint4 qw4 = *reinterpret_cast<const uint4*>(smem + kOffQ + (c >> 3) * kQHalf + row * 128 +
+          const uint4 qw4 = *reinterpret_cast<const uint4*>(smem + C::kOffQ + (c >> 3) * C::kQHalf + row * 128 +
                                                              (((c & 7) ^ (row & 7)) << 4));
-          const uint4 kw4 = *reinterpret_cast<const uint4*>(smem + kOffNewK + n * kNewRow + c * 16);
+          const uint4 kw4 = *reinterpret_cast<const uint4*>(smem + C::kOffNewK + n * kNewRow + c * 16);
           const uint32_t qa[4] = {qw4.x, qw4.y, qw4.z, qw4.w};
           const uint32_t ka[4] = {kw4.x, kw4.y, kw4.z, kw4.w};
 #pragma unroll
@@ -818,11 +898,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     // Weights first, one warp per row: lane j < csize takes partial j, lane
     // csize + n new key n; then every output is a sum of independent loads.
     mbar_wait(RECV, 0);
-    const float* recv = reinterpret_cast<const float*>(smem + kRecv);
-    float* s_w = reinterpret_cast<float*>(smem + kMergeW);  // [rpc][kWRow]: weights, then 1 / l
+    const float* recv = reinterpret_cast<const float*>(smem + C::kRecv);
+    float* s_w = reinterpret_cast<float*>(smem + C::kMergeW);  // [rpc][kWRow]: weights, then 1 / l
     const int n_new = (kFused && valid) ? a.R : 0;
 #pragma unroll 1
-    for (int rr = warp - 2; rr < rpc; rr += kSoftWarps) {
+    for (int rr = warp - 2; rr < my_rows; rr += kSoftWarps) {
       float m = -INFINITY, l = 0.f;
       if (lane < csize) {
         m = recv[(lane * rpc + rr) * kRowF + kD];
@@ -843,15 +923,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     named_bar_sync(2, kSoftThreads);
 #pragma unroll 1
-    for (int idx = st; idx < rpc * kD; idx += kSoftThreads) {
+    for (int idx = st; idx < my_rows * kD; idx += kSoftThreads) {
       const int rr = idx / kD, d = idx % kD;
       const int row = mrow0 + rr;
-      const int p = mblock * kRows + row;
+      const int p = mblock * kR + row;
       const float* w = s_w + rr * kWRow;
       float acc = 0.f;
 #pragma unroll 4
       for (int c = 0; c < csize; ++c) acc = fmaf(w[c], recv[(c * rpc + rr) * kRowF + d], acc);
-      const __nv_bfloat16* nv = reinterpret_cast<const __nv_bfloat16*>(smem + kOffNewV) + d;
+      const __nv_bfloat16* nv = reinterpret_cast<const __nv_bfloat16*>(smem + C::kOffNewV) + d;
 #pragma unroll 4
       for (int n = 0; n < n_new; ++n) acc = fmaf(w[csize + n], __bfloat162float(nv[n * kD]), acc);
       const float inv_l = w[kWRow - 1];
@@ -861,35 +941,35 @@ __global__ void __launch_bounds__(kThreads, 1)
             __float2bfloat16_rn(acc * inv_l);
       }
     }
-    if (st < csize) asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+    if (st < csize && rows_of(st) > 0) asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
     if (kFused && valid) {
       // every CTA of the cluster read the raw rows before its main loop (the
       // cluster barrier above is behind all of them): store the rotated query
-      // rows (rank 0), and append the new key / value rows and store the
-      // rotated keys back (last rank)
+      // rows of this m-block (rank 0), and append the new key / value rows
+      // and store the rotated keys back (last rank of m-block 0)
       if (rank == 0) {
 #pragma unroll 1
-        for (int idx = st; idx < kRows * 16; idx += kSoftThreads) {
+        for (int idx = st; idx < kR * 16; idx += kSoftThreads) {
           const int row = idx / 16, c = idx % 16;
-          const int p = mblock * kRows + row;
+          const int p = mblock * kR + row;
           if (p >= a.M) continue;
-          const uint4 v = *reinterpret_cast<const uint4*>(smem + kOffQ + (c >> 3) * kQHalf + row * 128 +
+          const uint4 v = *reinterpret_cast<const uint4*>(smem + C::kOffQ + (c >> 3) * C::kQHalf + row * 128 +
                                                           (((c & 7) ^ (row & 7)) << 4));
           *reinterpret_cast<uint4*>(a.qw + ((static_cast<long long>(b) * a.R + gdiv(p)) * a.Hq + kvh * a.G +
                                             (p - gdiv(p) * a.G)) * kD + c * 8) = v;
         }
       }
-      if (rank == csize - 1) {
+      if (rank == csize - 1 && mblock == 0) {
 #pragma unroll 1
         for (int idx = st; idx < a.R * 16; idx += kSoftThreads) {
           const int i = idx / 16, c = idx % 16;
           const long long src = ((static_cast<long long>(b) * a.R + i) * a.Hkv + kvh) * kD + c * 8;
           const long long dst = ((static_cast<long long>(b) * a.Hkv + kvh) * a.cap + L_pre + i) * kD + c * 8;
-          const uint4 kr = *reinterpret_cast<const uint4*>(smem + kOffNewK + i * kNewRow + c * 16);
+          const uint4 kr = *reinterpret_cast<const uint4*>(smem + C::kOffNewK + i * kNewRow + c * 16);
           *reinterpret_cast<uint4*>(a.kc + dst) = kr;
           *reinterpret_cast<uint4*>(a.k_new + src) = kr;
           *reinterpret_cast<uint4*>(a.vc + dst) =
-              *reinterpret_cast<const uint4*>(smem + kOffNewV + i * kNewRow + c * 16);
+              *reinterpret_cast<const uint4*>(smem + C::kOffNewV + i * kNewRow + c * 16);
         }
       }
     }
@@ -899,7 +979,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 1) {
     tc_fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
-                 "r"(kTmemCols)
+                 "r"(C::kTmemCols)
                  : "memory");
   }
 }
@@ -924,20 +1004,6 @@ EncodeTiledFn encode_fn() {
   return fn;
 }
 
-// q [B][R][Hq][D] as (D, Hq, B*R); box (64, G, R): one KV group's packed rows
-bool make_q_map(CUtensorMap* map, const void* q, int B, int R, int Hq, int G) {
-  EncodeTiledFn fn = encode_fn();
-  if (!fn) return false;
-  cuuint64_t dims[3] = {static_cast<cuuint64_t>(kD), static_cast<cuuint64_t>(Hq),
-                        static_cast<cuuint64_t>(B) * R};
-  cuuint64_t strides[2] = {static_cast<cuuint64_t>(kD) * 2, static_cast<cuuint64_t>(Hq) * kD * 2};
-  cuuint32_t box[3] = {64, static_cast<cuuint32_t>(G), static_cast<cuuint32_t>(R)};
-  cuuint32_t estr[3] = {1, 1, 1};
-  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(q), dims, strides, box, estr,
-            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
 bool make_map(CUtensorMap* map, void* base, int cap, int planes, int box_rows) {
   EncodeTiledFn fn = encode_fn();
   if (!fn) return false;
@@ -952,13 +1018,50 @@ bool make_map(CUtensorMap* map, void* base, int cap, int planes, int box_rows) {
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-constexpr int kClusterSizes[5] = {1, 2, 4, 8, 16};
+constexpr int kNumClusterSizes = 6;
+constexpr int kClusterSizes[kNumClusterSizes] = {1, 2, 4, 6, 8, 16};
 
+// per device: how many clusters of each size fit at once, for each row tile
+// (index 0: 32 rows, 1: 64 rows)
 struct DevState {
   bool ready = false;
   bool ok = false;
-  int active[5] = {0, 0, 0, 0, 0};
+  int active[2][kNumClusterSizes] = {};
 };
+
+template <int kR>
+bool set_attributes(int* active) {
+  auto kern = verify_attn_tc_kernel<kR, false>;
+  auto kern_f = verify_attn_tc_kernel<kR, true>;
+  constexpr int smem = Cfg<kR>::kSmemBytes;
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess ||
+      cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess ||
+      cudaFuncSetAttribute(kern_f, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess ||
+      cudaFuncSetAttribute(kern_f, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess) {
+    (void)cudaGetLastError();
+    return false;
+  }
+  for (int i = 0; i < kNumClusterSizes; ++i) {
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = kClusterSizes[i];
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.gridDim = dim3(kClusterSizes[i], 1, 1);
+    cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.dynamicSmemBytes = smem;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, reinterpret_cast<const void*>(kern), &cfg) != cudaSuccess) {
+      (void)cudaGetLastError();
+      n = 0;
+    }
+    active[i] = n;
+  }
+  return true;
+}
 
 DevState* state() {
   static DevState st[16];
@@ -970,54 +1073,21 @@ DevState* state() {
   DevState& s = st[dev];
   if (!s.ready) {
     s.ready = true;
-    auto kern = verify_attn_tc_kernel<false>;
-    auto kern_f = verify_attn_tc_kernel<true>;
-    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes) !=
-            cudaSuccess ||
-        cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
-            cudaSuccess ||
-        cudaFuncSetAttribute(kern_f, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes) !=
-            cudaSuccess ||
-        cudaFuncSetAttribute(kern_f, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
-            cudaSuccess) {
-      (void)cudaGetLastError();
-      return &s;
-    }
-    for (int i = 0; i < 5; ++i) {
-      cudaLaunchConfig_t cfg = {};
-      cudaLaunchAttribute attr[1];
-      attr[0].id = cudaLaunchAttributeClusterDimension;
-      attr[0].val.clusterDim.x = kClusterSizes[i];
-      attr[0].val.clusterDim.y = 1;
-      attr[0].val.clusterDim.z = 1;
-      cfg.gridDim = dim3(kClusterSizes[i], 1, 1);
-      cfg.blockDim = dim3(kThreads, 1, 1);
-      cfg.dynamicSmemBytes = kSmemBytes;
-      cfg.attrs = attr;
-      cfg.numAttrs = 1;
-      int n = 0;
-      if (cudaOccupancyMaxActiveClusters(&n, reinterpret_cast<const void*>(kern), &cfg) !=
-          cudaSuccess) {
-        (void)cudaGetLastError();
-        n = 0;
-      }
-      s.active[i] = n;
-    }
-    s.ok = true;
+    s.ok = set_attributes<32>(s.active[0]) && set_attributes<64>(s.active[1]);
   }
   return &s;
 }
 
 // Cluster size: minimise waves x (32-key blocks per CTA + a fixed per-CTA cost)
-int pick_cluster(const DevState& s, long long units, int cap) {
+int pick_cluster(const int* active, long long units, int cap) {
   const long long nblk = (cap + 31) / 32;
   long long best_cost = -1;
   int best = 0;
-  for (int i = 0; i < 5; ++i) {
+  for (int i = 0; i < kNumClusterSizes; ++i) {
     const int cs = kClusterSizes[i];
-    if (s.active[i] <= 0) continue;
+    if (active[i] <= 0) continue;
     if (cs > 1 && nblk < 2LL * cs) continue;
-    const long long waves = (units + s.active[i] - 1) / s.active[i];
+    const long long waves = (units + active[i] - 1) / active[i];
     const long long cost = waves * ((nblk + cs - 1) / cs + 6);
     if (best_cost < 0 || cost < best_cost) {
       best_cost = cost;
@@ -1039,58 +1109,92 @@ static bool tc_enabled() {
   return on;
 }
 
-static int serving_cluster(int B, int R, int Hq, int Hkv, int D, int cap);
+// How the tcgen05 path runs a shape: row tile (32 or 64 packed query rows),
+// m-blocks (row tiles per KV head) and cluster size; cs == 0: not served.
+struct TcPlan {
+  int rows = 0, mblocks = 0, cs = 0;
+};
 
-bool sd_internal_tc_serves(int B, int R, int Hq, int Hkv, int D, int cap) {
-  return serving_cluster(B, R, Hq, Hkv, D, cap) > 0;
+// Cluster size forced by sd_set_cluster_size (0: chosen per call).
+static std::atomic<int> g_forced_cluster{0};
+
+extern "C" sd_status sd_set_cluster_size(int cluster_size) {
+  if (cluster_size == 0) {
+    g_forced_cluster.store(0);
+    return SD_OK;
+  }
+  for (int i = 0; i < kNumClusterSizes; ++i)
+    if (kClusterSizes[i] == cluster_size) {
+      g_forced_cluster.store(cluster_size);
+      return SD_OK;
+    }
+  return SD_ERR_INVALID_ARG;
 }
 
-template <bool kFused>
-static sd_status launch_tc(const sd_kv_cache* cache, const void* q_for_map, const TcArgs& a,
-                    const RopeTable& tab, int cs, bool pdl, cudaStream_t stream) {
+static TcPlan tc_plan(int B, int R, int Hq, int Hkv, int D, int cap) {
+  TcPlan p;
+  if (!tc_enabled() || D != kD || Hkv <= 0 || Hq % Hkv || R <= 0) return p;
+  const int M = (Hq / Hkv) * R;
+  if (M > 2 * 64) return p;
+  DevState* s = state();
+  if (!s || !s->ok) return p;
+  p.rows = M <= 32 ? 32 : 64;
+  p.mblocks = (M + p.rows - 1) / p.rows;
+  const int* active = s->active[p.rows == 32 ? 0 : 1];
+  const int forced = g_forced_cluster.load();
+  for (int i = 0; i < kNumClusterSizes && forced > 0; ++i)
+    if (kClusterSizes[i] == forced && active[i] > 0) p.cs = forced;
+  if (p.cs == 0) p.cs = pick_cluster(active, static_cast<long long>(B) * Hkv * p.mblocks, cap);
+  return p;
+}
+
+bool sd_internal_tc_serves(int B, int R, int Hq, int Hkv, int D, int cap) {
+  return tc_plan(B, R, Hq, Hkv, D, cap).cs > 0;
+}
+
+template <int kR, bool kFused>
+static sd_status launch_tc(const sd_kv_cache* cache, const TcArgs& a, const RopeTable& tab,
+                           const TcPlan& plan, bool pdl, cudaStream_t stream) {
   const int B = cache->batch, Hkv = cache->n_kv_heads, cap = cache->capacity;
-  CUtensorMap k128, v128, qm;
-  if (!make_map(&k128, cache->k, cap, B * Hkv, 128) || !make_map(&v128, cache->v, cap, B * Hkv, 128) ||
-      !make_q_map(&qm, q_for_map, B, a.R, a.Hq, a.G))
+  CUtensorMap k128, v128;
+  if (!make_map(&k128, cache->k, cap, B * Hkv, 128) || !make_map(&v128, cache->v, cap, B * Hkv, 128))
     return SD_ERR_CUDA;
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = cs;
+  attr[0].val.clusterDim.x = plan.cs;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
   attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[1].val.programmaticStreamSerializationAllowed = 1;
-  cfg.gridDim = dim3(cs, Hkv, B);
+  cfg.gridDim = dim3(plan.cs, Hkv * plan.mblocks, B);
   cfg.blockDim = dim3(kThreads, 1, 1);
-  cfg.dynamicSmemBytes = kSmemBytes;
+  cfg.dynamicSmemBytes = Cfg<kR>::kSmemBytes;
   cfg.stream = stream;
   cfg.attrs = attr;
   cfg.numAttrs = pdl ? 2 : 1;
-  if (cudaLaunchKernelEx(&cfg, verify_attn_tc_kernel<kFused>, k128, v128, qm, a, tab) !=
-      cudaSuccess) {
+  if (cudaLaunchKernelEx(&cfg, verify_attn_tc_kernel<kR, kFused>, k128, v128, a, tab) != cudaSuccess) {
     (void)cudaGetLastError();
     return SD_ERR_CUDA;
   }
   return SD_OK;
 }
 
-static int serving_cluster(int B, int R, int Hq, int Hkv, int D, int cap) {
-  if (!tc_enabled() || D != kD || Hkv <= 0 || Hq % Hkv) return 0;
-  if ((Hq / Hkv) * R > kRows) return 0;
-  DevState* s = state();
-  if (!s || !s->ok) return 0;
-  return pick_cluster(*s, static_cast<long long>(B) * Hkv, cap);
+template <bool kFused>
+static sd_status launch_plan(const sd_kv_cache* cache, const TcArgs& a, const RopeTable& tab,
+                             const TcPlan& plan, bool pdl, cudaStream_t stream) {
+  return plan.rows == 32 ? launch_tc<32, kFused>(cache, a, tab, plan, pdl, stream)
+                         : launch_tc<64, kFused>(cache, a, tab, plan, pdl, stream);
 }
 
-// Routed here by sd_verify_attention for head_dim 128 and G * R <= 32.
+// Routed here by sd_verify_attention for head_dim 128 and G * R <= 128.
 sd_status sd_internal_verify_attention_tc(const void* q, const sd_kv_cache* cache, void* out,
                                           int R, int Hq, float scale_log2, cudaStream_t stream,
                                           bool* handled) {
   *handled = false;
   const int B = cache->batch, Hkv = cache->n_kv_heads;
-  const int cs = serving_cluster(B, R, Hq, Hkv, cache->head_dim, cache->capacity);
-  if (cs <= 0) return SD_OK;
+  const TcPlan plan = tc_plan(B, R, Hq, Hkv, cache->head_dim, cache->capacity);
+  if (plan.cs <= 0) return SD_OK;
   TcArgs a = {};
   a.q = static_cast<const __nv_bfloat16*>(q);
   a.out = static_cast<__nv_bfloat16*>(out);
@@ -1102,11 +1206,11 @@ sd_status sd_internal_verify_attention_tc(const void* q, const sd_kv_cache* cach
   a.M = a.G * R;
   a.inv_g = 1.0f / static_cast<float>(a.G);
   a.cap = cache->capacity;
-  a.n_mblocks = 1;
+  a.n_mblocks = plan.mblocks;
   a.scale_log2 = scale_log2;
   RopeTable tab = {};
   *handled = true;
-  return launch_tc<false>(cache, q, a, tab, cs, false, stream);
+  return launch_plan<false>(cache, a, tab, plan, false, stream);
 }
 
 // The fused verify layer (rope + append + attention) on the tcgen05 path.
@@ -1117,8 +1221,8 @@ sd_status sd_internal_verify_layer_tc(void* q, void* k_new, const void* v_new, c
   *handled = false;
   const int B = cache->batch, Hkv = cache->n_kv_heads;
   if (R > kMaxNew) return SD_OK;  // the new rows are held in shared memory
-  const int cs = serving_cluster(B, R, Hq, Hkv, cache->head_dim, cache->capacity);
-  if (cs <= 0) return SD_OK;
+  const TcPlan plan = tc_plan(B, R, Hq, Hkv, cache->head_dim, cache->capacity);
+  if (plan.cs <= 0) return SD_OK;
   TcArgs a = {};
   a.q = static_cast<const __nv_bfloat16*>(q);
   a.out = static_cast<__nv_bfloat16*>(out);
@@ -1138,8 +1242,8 @@ sd_status sd_internal_verify_layer_tc(void* q, void* k_new, const void* v_new, c
   a.M = a.G * R;
   a.inv_g = 1.0f / static_cast<float>(a.G);
   a.cap = cache->capacity;
-  a.n_mblocks = 1;
+  a.n_mblocks = plan.mblocks;
   a.scale_log2 = scale_log2;
   *handled = true;
-  return launch_tc<true>(cache, q, a, tab, cs, early != 0, stream);
+  return launch_plan<true>(cache, a, tab, plan, early != 0, stream);
 }

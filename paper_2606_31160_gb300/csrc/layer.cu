@@ -2,7 +2,7 @@
 // Sec. 3.2), the KV append (Eq. commit) and the verify attention (Eq. verify,
 // Sec. 2.2) of one attention layer as one call.
 //
-// On the tcgen05 path (head_dim 128, G * R <= 32) it is one kernel launch that
+// On the tcgen05 path (head_dim 128, G * R <= 128, R <= 16) it is one kernel launch that
 // may overlap the previous layer: the cached prefix of a layer does not
 // depend on the layer before it, so with SD_LAYER_PREFIX_EARLY the kernel is
 // a programmatic dependent launch that starts streaming that prefix while the

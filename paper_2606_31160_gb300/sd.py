@@ -59,6 +59,7 @@ _SIGNATURES = {
     "sd_accept_sample_workspace": ([_i, _i, _i], _sz),
     "sd_accept_sample": ([_vp, _vp, _i, _i, _i, _f, _vp, _vp, _vp, _vp, _vp, _sz, _vp], _i),
     "sd_get_device_error": ([_vp, ctypes.POINTER(ctypes.c_uint32)], _i),
+    "sd_set_cluster_size": ([_i], _i),
 }
 
 
@@ -335,6 +336,11 @@ def accept_sample(z_target, z_draft, draft, u, temperature, ws=None, n_emit=None
                                   _dev(ws, "ws"), ws.numel() * ws.element_size(), _stream()),
            "sd_accept_sample")
     return n_emit, tokens
+
+
+def set_cluster_size(cluster_size=0):
+    """Force the tcgen05 attention cluster size (1, 2, 4, 6, 8, 16); 0 = automatic."""
+    _check(lib().sd_set_cluster_size(int(cluster_size)), "sd_set_cluster_size")
 
 
 def get_device_error():

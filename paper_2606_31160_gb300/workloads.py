@@ -224,6 +224,38 @@ def sweep_case(B, L, K, layer=0):
                        cap=L + 17, layer=1000 * layer + 31 * B + K)
 
 
+def sweep_case_device(B, L, K, device, layer=0):
+    """The batched-sweep recipe at timing sizes, drawn on the device: the same
+    ragged prefix lengths L_b and query positions as sweep_case (same Philox
+    stream), K/V prefix rows, q, k_new and v_new ~ N(0, 1) bf16 from a seeded
+    device generator (torch Philox), cache tails zero. Returns (prefix int64
+    [B], q, k_new, v_new, pos, k_cache, v_cache, cap)."""
+    rng = philox(SWEEP, 7919 * layer + 31 * B + K)
+    lo = -(-3 * L // 4)
+    prefix = rng.integers(lo, L + 1, size=B)
+    R, Hq, Hkv, D, cap = K + 1, 32, 8, 128, L + 17
+    qpos = np.empty((B, R, 3), dtype=np.int32)
+    for b in range(B):
+        n_vis = (7 * int(prefix[b])) // 8
+        start = int(grid_positions(n_vis, 28, 32).max()) + 1 if n_vis else 0
+        qpos[b] = text_positions(start + int(prefix[b]) - n_vis, R)
+    gen = torch.Generator(device=device)
+    gen.manual_seed(1000 * (1000 + SWEEP) + 7919 * layer + 31 * B + K)
+
+    def normal(*shape):
+        return torch.randn(shape, generator=gen, device=device, dtype=torch.float32).to(torch.bfloat16)
+
+    k_cache = torch.zeros((B, Hkv, cap, D), dtype=torch.bfloat16, device=device)
+    v_cache = torch.zeros_like(k_cache)
+    for b in range(B):
+        n = int(prefix[b])
+        k_cache[b, :, :n] = normal(Hkv, n, D)
+        v_cache[b, :, :n] = normal(Hkv, n, D)
+    q, k_new, v_new = normal(B, R, Hq, D), normal(B, R, Hkv, D), normal(B, R, Hkv, D)
+    pos = torch.from_numpy(qpos).to(device)
+    return prefix, q, k_new, v_new, pos, k_cache, v_cache, cap
+
+
 def stochastic(B=8, K=7, V=151936, temperature=0.6, sigma_t=3.0, sigma_noise=0.5, seed_layer=0):
     """Stochastic acceptance inputs: fp32 target logits z_T ~ N(0, sigma_t) [B, K+1, V],
     draft logits z_D = z_T[:, :K] + N(0, sigma_noise) [B, K, V], draft tokens drawn

@@ -9,6 +9,14 @@ from paper_2606_31160_gb300 import build, sd
 ATTN_ATOL = 1e-2
 
 
+def attn_within(out, ref):
+    """True when |out - ref| <= 1e-2 + 2^-8 |ref| everywhere: the 1e-2 bound
+    plus the rounding of an exact result to bf16 (half an ulp is at most
+    2^-8 |x|), which alone exceeds 1e-2 once |x| >= 4 -- rows that see only a
+    few keys (short prefixes) average few values and reach that."""
+    return bool(np.all(np.abs(out - ref) <= ATTN_ATOL + 2.0 ** -8 * np.abs(ref)))
+
+
 def ensure_lib():
     build.build()
     return sd.lib()

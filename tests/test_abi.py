@@ -87,3 +87,12 @@ def test_bad_arguments_return_status_before_launch(lib):
     # empty batches are a no-op success
     cache = sd.KVCacheStruct(0, 0, 0, 0, 8, 64, 128)
     assert lib.sd_verify_attention(null, ctypes.byref(cache), null, 8, 32, 0.0, null, 0, null) == 0
+
+
+def test_cluster_size_override_is_host_only(lib):
+    # accepted sizes and 0 (automatic); no device work, so it runs without a GPU
+    for cs in (1, 2, 4, 6, 8, 16, 0):
+        assert lib.sd_set_cluster_size(cs) == 0
+    for cs in (-1, 3, 5, 7, 12, 32):
+        assert lib.sd_set_cluster_size(cs) == 1
+    assert lib.sd_set_cluster_size(0) == 0
