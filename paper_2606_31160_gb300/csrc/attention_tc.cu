@@ -73,7 +73,6 @@ constexpr float kSlack = 64.f;              // log2 units a score may exceed its
 // a merged partial row is [O(128) | m | l | 2 pad] fp32 = 528 bytes
 constexpr int kRowF = kD + 4;
 constexpr int kRowBytes = kRowF * 4;
-constexpr int kWRow = 2 * 16 + 4;           // merge weights of a row: csize + R, 1 / l
 constexpr int round_up(int x, int m) { return (x + m - 1) / m * m; }
 
 // Everything that depends on the packed query rows per CTA (kR = 32 or 64:
@@ -121,8 +120,7 @@ struct Cfg {
   // slots for ceil(kR / c) rows from each of c ranks, c in {1, 2, 4, 6, 8, 16}
   static constexpr int kRecvSlots = kR == 32 ? 36 : 66;
   static constexpr int kNewS = round_up(kRecv + kRecvSlots * kRowBytes, 1024);  // new-key scores
-  static constexpr int kMergeW = kNewS + kR * kMaxNew * 4;
-  static_assert(kMergeW + kR * kWRow * 4 <= kRing, "merge buffers");
+  static_assert(kNewS + kR * kMaxNew * 4 <= kRing, "merge buffers");
 };
 
 __device__ __forceinline__ uint32_t smem_addr(const void* p) {
@@ -270,11 +268,13 @@ __device__ __forceinline__ void rows_reduce(const float (&v)[kN], int kl, int ro
   for (int j = 0; j < kN; ++j) buf[(row0 + j) * 128 + kl] = v[j];
   asm volatile("bar.sync 2, 256;" ::: "memory");
   const int r = st / kPer, part = st % kPer;
-  const float4* src = reinterpret_cast<const float4*>(buf + r * 128 + part * kVals);
+  // part p reads float4 q * kPer + p of its row: per load, the kPer threads of
+  // a row cover kPer * 16 contiguous bytes (no bank conflicts beyond the rows)
+  const float4* src = reinterpret_cast<const float4*>(buf + r * 128) + part;
   float acc = kMax ? -INFINITY : 0.f;
 #pragma unroll
   for (int q = 0; q < kVals / 4; ++q) {
-    const float4 x = src[q];
+    const float4 x = src[q * kPer];
     acc = kMax ? fmaxf(acc, fmaxf(fmaxf(x.x, x.y), fmaxf(x.z, x.w))) : acc + ((x.x + x.y) + (x.z + x.w));
   }
 #pragma unroll
@@ -875,7 +875,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         float acc = 0.f;
 #pragma unroll
         for (int u = 0; u < 2; ++u) {
-          const int c = 2 * sub + u;
+          const int c = sub + 8 * u;
           const uint4 qw4 = *reinterpret_cast<const uint4*>(smem + C::kOffQ + (c >> 3) * C::kQHalf + row * 128 +
                                                              (((c & 7) ^ (row & 7)) << 4));
           const uint4 kw4 = *reinterpret_cast<const uint4*>(smem + C::kOffNewK + n * kNewRow + c * 16);
@@ -895,50 +895,66 @@ __global__ void __launch_bounds__(kThreads, 1)
       named_bar_sync(2, kSoftThreads);
     }
     // ---- merge of the rows this CTA owns; slot c * rpc + rr came from rank c.
-    // Weights first, one warp per row: lane j < csize takes partial j, lane
-    // csize + n new key n; then every output is a sum of independent loads.
+    // A thread takes one row and two adjacent d: it forms the row's weights
+    // itself (partials c < csize and new keys n < R, all loads issued
+    // together), then its two outputs.
     mbar_wait(RECV, 0);
     const float* recv = reinterpret_cast<const float*>(smem + C::kRecv);
-    float* s_w = reinterpret_cast<float*>(smem + C::kMergeW);  // [rpc][kWRow]: weights, then 1 / l
     const int n_new = (kFused && valid) ? a.R : 0;
 #pragma unroll 1
-    for (int rr = warp - 2; rr < my_rows; rr += kSoftWarps) {
-      float m = -INFINITY, l = 0.f;
-      if (lane < csize) {
-        m = recv[(lane * rpc + rr) * kRowF + kD];
-        l = recv[(lane * rpc + rr) * kRowF + kD + 1];
-      } else if (lane < csize + n_new) {
-        m = s_new[rr * a.R + (lane - csize)];
-        l = 1.f;
-      }
-      float mmax = m;
-#pragma unroll
-      for (int w = 16; w >= 1; w >>= 1) mmax = fmaxf(mmax, __shfl_xor_sync(0xffffffffu, mmax, w));
-      const float f = m == -INFINITY ? 0.f : ex2(m - mmax);
-      float lsum = f * l;
-#pragma unroll
-      for (int w = 16; w >= 1; w >>= 1) lsum += __shfl_xor_sync(0xffffffffu, lsum, w);
-      if (lane < csize + n_new) s_w[rr * kWRow + lane] = f;
-      if (lane == 0) s_w[rr * kWRow + kWRow - 1] = lsum > 0.f ? 1.f / lsum : 0.f;
-    }
-    named_bar_sync(2, kSoftThreads);
-#pragma unroll 1
-    for (int idx = st; idx < my_rows * kD; idx += kSoftThreads) {
-      const int rr = idx / kD, d = idx % kD;
+    for (int idx = st; idx < my_rows * (kD / 2); idx += kSoftThreads) {
+      const int rr = idx / (kD / 2), d = 2 * (idx % (kD / 2));
       const int row = mrow0 + rr;
       const int p = mblock * kR + row;
-      const float* w = s_w + rr * kWRow;
-      float acc = 0.f;
-#pragma unroll 4
-      for (int c = 0; c < csize; ++c) acc = fmaf(w[c], recv[(c * rpc + rr) * kRowF + d], acc);
-      const __nv_bfloat16* nv = reinterpret_cast<const __nv_bfloat16*>(smem + C::kOffNewV) + d;
-#pragma unroll 4
-      for (int n = 0; n < n_new; ++n) acc = fmaf(w[csize + n], __bfloat162float(nv[n * kD]), acc);
-      const float inv_l = w[kWRow - 1];
-      if (valid && p < a.M && inv_l > 0.f) {
+      float mc[16], lc[16], sn[kMaxNew];
+#pragma unroll
+      for (int c = 0; c < 16; ++c) {
+        // slots past the cluster read partial 0 (always present) with weight 0
+        const float* part = recv + ((c < csize ? c : 0) * rpc + rr) * kRowF + kD;
+        mc[c] = c < csize ? part[0] : -INFINITY;
+        lc[c] = c < csize ? part[1] : 0.f;
+      }
+#pragma unroll
+      for (int n = 0; n < kMaxNew; ++n) sn[n] = n < n_new ? s_new[rr * a.R + n] : -INFINITY;
+      float mx = -INFINITY;
+#pragma unroll
+      for (int c = 0; c < 16; ++c) mx = fmaxf(mx, mc[c]);
+#pragma unroll
+      for (int n = 0; n < kMaxNew; ++n) mx = fmaxf(mx, sn[n]);
+      const float msub = mx == -INFINITY ? 0.f : mx;  // no key at all: every weight 0
+      float lsum = 0.f;
+#pragma unroll
+      for (int c = 0; c < 16; ++c) {
+        mc[c] = ex2(mc[c] - msub);  // ex2(-inf) = 0
+        lsum = fmaf(mc[c], lc[c], lsum);
+      }
+#pragma unroll
+      for (int n = 0; n < kMaxNew; ++n) {
+        sn[n] = ex2(sn[n] - msub);
+        lsum += sn[n];
+      }
+      float2 acc = make_float2(0.f, 0.f);
+#pragma unroll
+      for (int c = 0; c < 16; ++c) {
+        if (c < csize) {
+          const float2 o = *reinterpret_cast<const float2*>(recv + ((c < csize ? c : 0) * rpc + rr) * kRowF + d);
+          acc.x = fmaf(mc[c], o.x, acc.x);
+          acc.y = fmaf(mc[c], o.y, acc.y);
+        }
+      }
+#pragma unroll
+      for (int n = 0; n < kMaxNew; ++n) {
+        if (n < n_new) {
+          const uint32_t v2 = *reinterpret_cast<const uint32_t*>(smem + C::kOffNewV + n * kNewRow + d * 2);
+          acc.x = fmaf(sn[n], sd_bf16_lo(v2), acc.x);
+          acc.y = fmaf(sn[n], sd_bf16_hi(v2), acc.y);
+        }
+      }
+      if (valid && p < a.M && lsum > 0.f) {
+        const float inv_l = 1.f / lsum;
         const int i = gdiv(p), gq = (p - gdiv(p) * a.G);
-        a.out[((static_cast<long long>(b) * a.R + i) * a.Hq + kvh * a.G + gq) * kD + d] =
-            __float2bfloat16_rn(acc * inv_l);
+        *reinterpret_cast<uint32_t*>(a.out + ((static_cast<long long>(b) * a.R + i) * a.Hq + kvh * a.G + gq) * kD +
+                                     d) = cvt_bf16x2(acc.x * inv_l, acc.y * inv_l);
       }
     }
     if (st < csize && rows_of(st) > 0) asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
