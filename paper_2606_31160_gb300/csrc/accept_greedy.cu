@@ -5,14 +5,17 @@
 //   l    = number of leading drafts equal to r*   (draft[j] vs r*_j, j < K)
 //   emit draft[0..l-1], r*_l            n_emit = l + 1
 //
-// One launch. The vocabulary of every row is split into chunks; a CTA scans
-// one (scene, row, chunk) with 16-byte vector loads, reduces (value, index)
-// pairs with warp shuffles and shared memory, and writes one partial. The
-// last CTA of each scene (atomic ticket, no spin) reduces the partials of all
-// K + 1 rows, compares with the drafts and writes the outputs, then re-arms
-// its ticket. The (value desc, index asc) order is total, so the result does
-// not depend on the order partials are combined in: bit-exact and
-// deterministic.
+// Cluster kernel (rows whose bytes are 16-byte aligned, the usual case): one
+// thread-block cluster of up to 16 CTAs per (scene, row). CTA c scans the c-th
+// slice of the row with 16-byte loads and sends its (value, index) to rank 0
+// through distributed shared memory; rank 0 writes the row's argmax and takes
+// the scene's ticket (one atomic per row); the scene's last row reads every
+// row's argmax, compares with the drafts (read at kernel start) and writes
+// the outputs. Other shapes take the chunked kernel: a CTA per (scene, row,
+// chunk) writes a partial, and the last CTA of each scene (atomic ticket, no
+// spin) reduces them. The (value desc, index asc) order is total, so both
+// results do not depend on the order candidates are combined in: bit-exact
+// and deterministic.
 #include "common.cuh"
 
 #include <mutex>
@@ -181,6 +184,156 @@ __global__ void __launch_bounds__(kThreads) greedy_kernel(const T* __restrict__ 
   }
 }
 
+// ------------------------------------------------------------ cluster kernel
+constexpr int kCThreads = 512;
+constexpr int kCWarps = kCThreads / 32;
+
+// One cluster of csize CTAs per (scene b, row r): CTA c scans elements
+// [c * slice, (c + 1) * slice) of the row with 16-byte loads, its best goes
+// to rank 0's shared memory; rank 0 writes the row's best to rowbest[b][r]
+// and takes the scene's ticket; the last row of the scene to finish reads
+// every row's best and accepts. R atomics per scene.
+template <typename T>
+__global__ void __launch_bounds__(kCThreads, 1)
+    greedy_cluster_kernel(const T* __restrict__ logits, int R, int V, int slice,
+                          const int32_t* __restrict__ draft, int32_t* __restrict__ n_emit,
+                          int32_t* __restrict__ tokens, int32_t* __restrict__ argmax_out,
+                          float2* __restrict__ rowbest, uint32_t* __restrict__ ticket) {
+  __shared__ float2 s_wbest[kCWarps];
+  __shared__ float2 s_cand[16];
+  __shared__ int s_draft[128];
+  __shared__ int s_star[128];
+  __shared__ bool s_last;
+  const int rank = blockIdx.x, csize = gridDim.x, r = blockIdx.y, b = blockIdx.z;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int K = R - 1;
+  if (rank == 0)  // read early: only the scene's last row uses them
+    for (int j = threadIdx.x; j < K; j += kCThreads) s_draft[j] = __ldg(draft + static_cast<long long>(b) * K + j);
+  const T* row = logits + (static_cast<long long>(b) * R + r) * V;
+  const int lo = rank * slice, hi = min(V, lo + slice);
+  Best best = warp_best(scan_chunk(row, lo, hi, true));
+  if (lane == 0) s_wbest[warp] = make_float2(best.v, __int_as_float(best.i));
+  __syncthreads();
+  if (warp == 0) {
+    Best c{-INFINITY, 0x7fffffff};
+    if (lane < kCWarps) c = Best{s_wbest[lane].x, __float_as_int(s_wbest[lane].y)};
+    c = warp_best(c);
+    if (lane == 0) {
+      uint32_t dst;
+      asm volatile("mapa.shared::cluster.u32 %0, %1, 0;"
+                   : "=r"(dst)
+                   : "r"(static_cast<uint32_t>(__cvta_generic_to_shared(s_cand + rank))));
+      asm volatile("st.shared::cluster.v2.f32 [%0], {%1, %2};" ::"r"(dst), "f"(c.v), "f"(__int_as_float(c.i))
+                   : "memory");
+    }
+  }
+  asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+  asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
+  if (rank != 0 || warp != 0) return;
+  // ---- rank 0, warp 0: the row's best, then the scene's ticket
+  Best w{-INFINITY, 0x7fffffff};
+  if (lane < csize) w = Best{s_cand[lane].x, __float_as_int(s_cand[lane].y)};
+  w = warp_best(w);
+  if (lane == 0) {
+    const int star = w.i == 0x7fffffff ? 0 : w.i;
+    if (argmax_out) argmax_out[static_cast<long long>(b) * R + r] = star;
+    rowbest[static_cast<long long>(b) * R + r] = make_float2(0.f, __int_as_float(star));
+    __threadfence();
+    s_last = atomicAdd(&ticket[b], 1u) == static_cast<uint32_t>(R - 1);
+  }
+  __syncwarp();
+  if (!s_last) return;
+  __threadfence();
+  for (int j = lane; j < R; j += 32) s_star[j] = __float_as_int(__ldcg(rowbest + static_cast<long long>(b) * R + j).y);
+  __syncwarp();
+  // l = first j < K with draft[j] != r*_j (K when none): one ballot per 32 drafts
+  int ell = K;
+  bool range_ok = true;
+  for (int j0 = 0; j0 < K && ell == K; j0 += 32) {
+    const int j = j0 + lane;
+    const bool live = j < K;
+    const int d = live ? s_draft[j] : 0;
+    range_ok &= !live || (d >= 0 && d < V);
+    const uint32_t miss = __ballot_sync(0xffffffffu, live && d != s_star[live ? j : 0]);
+    if (miss) ell = j0 + __ffs(miss) - 1;
+  }
+  for (int j = ell + 1 + lane; j < K; j += 32) {  // drafts past the first mismatch: range only
+    const int d = s_draft[j];
+    range_ok &= d >= 0 && d < V;
+  }
+  if (!__all_sync(0xffffffffu, range_ok) && lane == 0) sd_set_error(SD_DEVERR_TOKEN_RANGE);
+  int32_t* tk = tokens + static_cast<long long>(b) * R;
+  for (int j = lane; j < R; j += 32) tk[j] = j < ell ? s_draft[j] : (j == ell ? s_star[ell] : -1);
+  if (lane == 0) {
+    n_emit[b] = ell + 1;
+    ticket[b] = 0;  // re-arm for the next call
+  }
+}
+
+// Cluster size (rows of about 16 KB per CTA, at most 16) and the slice each
+// CTA scans (a multiple of 16 bytes); 0 when the shape is left to the chunked
+// kernel.
+int max_cluster();
+
+int cluster_slice(int R, int V, int elem_bytes, int* slice) {
+  if ((static_cast<long long>(V) * elem_bytes) % 16 != 0 || R > 128) return 0;
+  const int per = 16 / elem_bytes;
+  long long cs = (static_cast<long long>(V) * elem_bytes + 16383) / 16384;
+  cs = cs < 1 ? 1 : (cs > 16 ? 16 : cs);
+  const int cmax = max_cluster();
+  if (cmax <= 0) return 0;
+  if (cs > cmax) cs = cmax;
+  *slice = static_cast<int>(((V + cs - 1) / cs + per - 1) / per * per);
+  return static_cast<int>(cs);
+}
+
+// Largest cluster size (16 or 8) that can run on this device; 0 when neither
+// (or the attribute calls fail).
+int max_cluster() {
+  static int cache[64];
+  static bool done[64];
+  static std::mutex mu;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) {
+    (void)cudaGetLastError();
+    return 0;
+  }
+  std::lock_guard<std::mutex> lock(mu);
+  if (!done[dev]) {
+    done[dev] = true;
+    const void* kerns[2] = {reinterpret_cast<const void*>(greedy_cluster_kernel<float>),
+                            reinterpret_cast<const void*>(greedy_cluster_kernel<__nv_bfloat16>)};
+    bool ok = true;
+    for (const void* k : kerns)
+      ok = ok && cudaFuncSetAttribute(k, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) == cudaSuccess;
+    int best = 0;
+    if (ok) {
+      for (int cs : {16, 8}) {
+        cudaLaunchConfig_t cfg = {};
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeClusterDimension;
+        attr[0].val.clusterDim.x = cs;
+        attr[0].val.clusterDim.y = 1;
+        attr[0].val.clusterDim.z = 1;
+        cfg.gridDim = dim3(cs, 1, 1);
+        cfg.blockDim = dim3(kCThreads, 1, 1);
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        int nclusters = 0;
+        if (cudaOccupancyMaxActiveClusters(&nclusters, kerns[1], &cfg) == cudaSuccess && nclusters > 0) {
+          best = cs;
+          break;
+        }
+        (void)cudaGetLastError();
+      }
+    } else {
+      (void)cudaGetLastError();
+    }
+    cache[dev] = best;
+  }
+  return cache[dev];
+}
+
 // Chunking depends on V only (never on the device), so the workspace size
 // is the same wherever it is queried: 4096 elements per CTA, more when the
 // row would need over kMaxChunks chunks.
@@ -217,10 +370,52 @@ static sd_status check_args(const void* logits, sd_dtype dtype, int B, int K, in
   return SD_OK;
 }
 
+// The cluster kernel when the shape allows it; true when it was launched (or
+// the launch failed: *status says which). rowbest takes the first B * R
+// entries of the partials.
+static bool launch_cluster(const void* logits, sd_dtype dtype, int B, int K, int V,
+                           const int32_t* draft, int32_t* n_emit, int32_t* tokens, int32_t* argmax,
+                           float2* rowbest, uint32_t* ticket, cudaStream_t st, sd_status* status) {
+  const int R = K + 1;
+  const int eb = dtype == SD_BF16 ? 2 : 4;
+  if ((reinterpret_cast<uintptr_t>(logits) & 15) != 0) return false;
+  int slice = 0;
+  const int cs = cluster_slice(R, V, eb, &slice);
+  if (cs <= 0) return false;
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = cs;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.gridDim = dim3(cs, R, B);
+  cfg.blockDim = dim3(kCThreads, 1, 1);
+  cfg.stream = st;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cudaError_t e;
+  if (dtype == SD_BF16)
+    e = cudaLaunchKernelEx(&cfg, greedy_cluster_kernel<__nv_bfloat16>, static_cast<const __nv_bfloat16*>(logits),
+                           R, V, slice, draft, n_emit, tokens, argmax, rowbest, ticket);
+  else
+    e = cudaLaunchKernelEx(&cfg, greedy_cluster_kernel<float>, static_cast<const float*>(logits), R, V, slice,
+                           draft, n_emit, tokens, argmax, rowbest, ticket);
+  if (e != cudaSuccess) {
+    (void)cudaGetLastError();
+    *status = SD_ERR_CUDA;
+  } else {
+    *status = SD_OK;
+  }
+  return true;
+}
+
 static sd_status launch(const void* logits, sd_dtype dtype, int B, int K, int V,
                         const int32_t* draft, int32_t* n_emit, int32_t* tokens, int32_t* argmax,
                         float2* part, uint32_t* ticket, int chunk, int n_chunks,
                         cudaStream_t st) {
+  sd_status cs_status;
+  if (launch_cluster(logits, dtype, B, K, V, draft, n_emit, tokens, argmax, part, ticket, st, &cs_status))
+    return cs_status;
   const int R = K + 1;
   const dim3 grid(n_chunks, R, B);
   if (dtype == SD_BF16)

@@ -613,6 +613,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int j = 0; j < 4; ++j) w[j] = sd_rope_pair(w[j], cs[j].x, cs[j].y);
           st_shared_v4(base + C::kOffNewK + i * kNewRow + c * 16, w[0], w[1], w[2], w[3]);
           st_shared_v4(base + C::kOffNewV + i * kNewRow + c * 16, vv.x, vv.y, vv.z, vv.w);
+        } else if (kFused && st < kMaxNew * 16) {
+          // value rows past R stay zero: the merge reads all kMaxNew rows
+          st_shared_v4(base + C::kOffNewV + (st >> 4) * kNewRow + (st & 15) * 16, 0u, 0u, 0u, 0u);
         }
       }
       // causal limit of each packed row: row p = i * G + g is new row i and
@@ -895,59 +898,53 @@ __global__ void __launch_bounds__(kThreads, 1)
       named_bar_sync(2, kSoftThreads);
     }
     // ---- merge of the rows this CTA owns; slot c * rpc + rr came from rank c.
-    // A thread takes one row and two adjacent d: it forms the row's weights
-    // itself (partials c < csize and new keys n < R, all loads issued
-    // together), then its two outputs.
+    // A warp takes 64 adjacent outputs of one row (a thread two adjacent d).
+    // The row's weights come lane-parallel: lane c < csize holds partial c's
+    // (m, l), lane csize + n new key n's score; the warp reduces them with
+    // shuffles and broadcasts each weight. The output loads do not depend on
+    // the counts (slots past the cluster read partial 0, value rows past R are
+    // zero; their weights are 0), so they issue together.
     mbar_wait(RECV, 0);
     const float* recv = reinterpret_cast<const float*>(smem + C::kRecv);
     const int n_new = (kFused && valid) ? a.R : 0;
 #pragma unroll 1
-    for (int idx = st; idx < my_rows * (kD / 2); idx += kSoftThreads) {
+    for (int idx = st; idx < my_rows * (kD / 2); idx += kSoftThreads) {  // the row is warp-uniform
       const int rr = idx / (kD / 2), d = 2 * (idx % (kD / 2));
       const int row = mrow0 + rr;
       const int p = mblock * kR + row;
-      float mc[16], lc[16], sn[kMaxNew];
-#pragma unroll
-      for (int c = 0; c < 16; ++c) {
-        // slots past the cluster read partial 0 (always present) with weight 0
-        const float* part = recv + ((c < csize ? c : 0) * rpc + rr) * kRowF + kD;
-        mc[c] = c < csize ? part[0] : -INFINITY;
-        lc[c] = c < csize ? part[1] : 0.f;
+      float m = -INFINITY, l = 0.f;
+      if (lane < csize) {
+        const float2 ml = *reinterpret_cast<const float2*>(recv + (lane * rpc + rr) * kRowF + kD);
+        m = ml.x;
+        l = ml.y;
+      } else if (lane < csize + n_new) {
+        m = s_new[rr * a.R + (lane - csize)];
+        l = 1.f;
       }
+      float mx = m;
 #pragma unroll
-      for (int n = 0; n < kMaxNew; ++n) sn[n] = n < n_new ? s_new[rr * a.R + n] : -INFINITY;
-      float mx = -INFINITY;
+      for (int w = 16; w >= 1; w >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, w));
+      const float f = ex2(m - (mx == -INFINITY ? 0.f : mx));  // ex2(-inf) = 0
+      float lsum = f * l;
 #pragma unroll
-      for (int c = 0; c < 16; ++c) mx = fmaxf(mx, mc[c]);
-#pragma unroll
-      for (int n = 0; n < kMaxNew; ++n) mx = fmaxf(mx, sn[n]);
-      const float msub = mx == -INFINITY ? 0.f : mx;  // no key at all: every weight 0
-      float lsum = 0.f;
-#pragma unroll
-      for (int c = 0; c < 16; ++c) {
-        mc[c] = ex2(mc[c] - msub);  // ex2(-inf) = 0
-        lsum = fmaf(mc[c], lc[c], lsum);
-      }
-#pragma unroll
-      for (int n = 0; n < kMaxNew; ++n) {
-        sn[n] = ex2(sn[n] - msub);
-        lsum += sn[n];
-      }
+      for (int w = 16; w >= 1; w >>= 1) lsum += __shfl_xor_sync(0xffffffffu, lsum, w);
       float2 acc = make_float2(0.f, 0.f);
 #pragma unroll
       for (int c = 0; c < 16; ++c) {
-        if (c < csize) {
-          const float2 o = *reinterpret_cast<const float2*>(recv + ((c < csize ? c : 0) * rpc + rr) * kRowF + d);
-          acc.x = fmaf(mc[c], o.x, acc.x);
-          acc.y = fmaf(mc[c], o.y, acc.y);
-        }
+        const float wc = __shfl_sync(0xffffffffu, f, c);
+        const float2 o = *reinterpret_cast<const float2*>(recv + ((c < csize ? c : 0) * rpc + rr) * kRowF + d);
+        const float wz = c < csize ? wc : 0.f;
+        acc.x = fmaf(wz, o.x, acc.x);
+        acc.y = fmaf(wz, o.y, acc.y);
       }
+      if (kFused) {
 #pragma unroll
-      for (int n = 0; n < kMaxNew; ++n) {
-        if (n < n_new) {
+        for (int n = 0; n < kMaxNew; ++n) {
+          const float wn = __shfl_sync(0xffffffffu, f, min(csize + n, 31));
           const uint32_t v2 = *reinterpret_cast<const uint32_t*>(smem + C::kOffNewV + n * kNewRow + d * 2);
-          acc.x = fmaf(sn[n], sd_bf16_lo(v2), acc.x);
-          acc.y = fmaf(sn[n], sd_bf16_hi(v2), acc.y);
+          const float wz = n < n_new ? wn : 0.f;
+          acc.x = fmaf(wz, sd_bf16_lo(v2), acc.x);
+          acc.y = fmaf(wz, sd_bf16_hi(v2), acc.y);
         }
       }
       if (valid && p < a.M && lsum > 0.f) {
