@@ -9,10 +9,13 @@
 //
 // Two launches:
 //   stats:  grid (chunk, row, scene) over the 2K + 1 rows; each CTA writes
-//           (max, sum exp2((z - max) * log2e / T)) of one chunk. The last CTA
-//           of a scene (atomic ticket, no spin) merges the chunks of every
-//           row in a fixed order, runs the K acceptance tests and records l
-//           and the normalisers of the row to draw from.
+//           (max, sum exp2((z - max) * log2e / T)) of one chunk of 16384
+//           (rows of 16-byte multiples: 32 values per thread from eight
+//           16-byte loads, kept in registers for both) or 4096 elements, and
+//           the CTA whose chunk holds a draft token records its logit. The
+//           last CTA of a scene (atomic ticket, no spin) merges the chunks of
+//           every row in a fixed order, runs the K acceptance tests and
+//           records l and the normalisers of the row to draw from.
 //   draw:   grid (chunk, scene) over that one row; each CTA writes the
 //           chunk sums of the residual weights and of the target weights; the
 //           last CTA of a scene finds the chunk where the running sum passes
@@ -21,6 +24,8 @@
 // uses non-contractible intrinsics so both passes of the draw evaluate
 // identical values, and every spin-free ticket is re-armed after use.
 #include "common.cuh"
+
+#include <mutex>
 
 SD_DEFINE_ERROR_ACCESSOR(sd_take_error_sample)
 
@@ -39,7 +44,9 @@ struct DrawInfo {
 
 // exp2((z - m) * c2) with a fixed rounding sequence
 __device__ __forceinline__ float wexp(float z, float m, float c2) {
-  return exp2f(__fmul_rn(__fsub_rn(z, m), c2));
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(__fmul_rn(__fsub_rn(z, m), c2)));
+  return y;
 }
 
 // (max, sum) pair merge: sum rescaled to the larger max
@@ -64,51 +71,21 @@ __device__ __forceinline__ const float* row_ptr(const float* zt, const float* zd
   return zd + (static_cast<long long>(b) * K + (rr - K - 1)) * V;
 }
 
-// ------------------------------------------------------------------ stats
-__global__ void __launch_bounds__(kThreads)
-    sample_stats_kernel(const float* __restrict__ zt, const float* __restrict__ zd, int K, int V,
-                        float c2, int chunk, int n_chunks, const int32_t* __restrict__ draft,
-                        const float* __restrict__ u, int32_t* __restrict__ n_emit,
-                        int32_t* __restrict__ tokens, float2* __restrict__ part,
-                        uint32_t* __restrict__ ticket, DrawInfo* __restrict__ info) {
-  const int c = blockIdx.x, rr = blockIdx.y, b = blockIdx.z;
+// The last CTA of scene b (all of its chunk partials are in): merge the
+// chunks of every row in a fixed order, run the K acceptance tests, record l
+// and the normalisers of the row to draw from, write n_emit and the accepted
+// tokens, re-arm the ticket. Called by all nthreads threads of that CTA.
+__device__ __noinline__ void accept_tail(const float* __restrict__ zt, const float* __restrict__ zd, int K,
+                                         int V, float c2, int n_chunks, int b, const int* s_x,
+                                         const float* __restrict__ u, int32_t* __restrict__ n_emit,
+                                         int32_t* __restrict__ tokens, const float2* __restrict__ part,
+                                         const float* __restrict__ dlogit, uint32_t* __restrict__ ticket,
+                                         DrawInfo* __restrict__ info, int nthreads) {
   const int rows = 2 * K + 1;
-  const float* row = row_ptr(zt, zd, b, rr, K, V);
-  const int lo = c * chunk, hi = min(V, lo + chunk);
-  // thread max, then thread sum, over a fixed strided subset of the chunk
-  float m = -INFINITY;
-  for (int i = lo + threadIdx.x; i < hi; i += kThreads) m = fmaxf(m, __ldg(row + i));
-  float s = 0.f;
-  if (m != -INFINITY)
-    for (int i = lo + threadIdx.x; i < hi; i += kThreads) s = __fadd_rn(s, wexp(__ldg(row + i), m, c2));
-  // warp then block merge, fixed tree
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    const float m2 = __shfl_xor_sync(0xffffffffu, m, o);
-    const float s2 = __shfl_xor_sync(0xffffffffu, s, o);
-    merge_ms(m, s, m2, s2, c2);
-  }
-  __shared__ float sm[kThreads / 32], ss[kThreads / 32];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  if (lane == 0) {
-    sm[warp] = m;
-    ss[warp] = s;
-  }
-  __syncthreads();
-  __shared__ bool s_last;
-  if (threadIdx.x == 0) {
-    float bm = sm[0], bs = ss[0];
-    for (int w = 1; w < kThreads / 32; ++w) merge_ms(bm, bs, sm[w], ss[w], c2);
-    part[(static_cast<long long>(b) * rows + rr) * n_chunks + c] = make_float2(bm, bs);
-    __threadfence();
-    s_last = atomicAdd(&ticket[b], 1u) == static_cast<uint32_t>(rows * n_chunks - 1);
-  }
-  __syncthreads();
-  if (!s_last) return;
-  __threadfence();
-  // ---- last CTA of scene b: merge chunks per row, then the acceptance tests
+  const int kT = nthreads;
   __shared__ float row_m[2 * 128 + 1], row_s[2 * 128 + 1];
-  for (int r = warp; r < rows; r += kThreads / 32) {
+  for (int r = warp; r < rows; r += kT / 32) {
     float rm = -INFINITY, rs = 0.f;
     const float2* pr = part + (static_cast<long long>(b) * rows + r) * n_chunks;
     for (int k = lane; k < n_chunks; k += 32) {
@@ -127,15 +104,13 @@ __global__ void __launch_bounds__(kThreads)
     }
   }
   __syncthreads();
-  // the K draft tokens and their two logits, fetched in parallel
-  __shared__ int s_x[128];
+  // the K draft tokens' two logits, recorded by the CTAs holding them
   __shared__ float s_zt[128], s_zd[128];
-  for (int j = threadIdx.x; j < K; j += kThreads) {
-    const int x = draft[static_cast<long long>(b) * K + j];
-    s_x[j] = x;
+  for (int j = threadIdx.x; j < K; j += kT) {
+    const int x = s_x[j];
     const bool ok = x >= 0 && x < V;
-    s_zt[j] = ok ? row_ptr(zt, zd, b, j, K, V)[x] : 0.f;
-    s_zd[j] = ok ? row_ptr(zt, zd, b, K + 1 + j, K, V)[x] : 0.f;
+    s_zt[j] = ok ? __ldcg(dlogit + static_cast<long long>(b) * rows + j) : 0.f;
+    s_zd[j] = ok ? __ldcg(dlogit + static_cast<long long>(b) * rows + K + 1 + j) : 0.f;
   }
   __syncthreads();
   if (threadIdx.x == 0) {
@@ -169,6 +144,239 @@ __global__ void __launch_bounds__(kThreads)
     n_emit[b] = ell + 1;
     ticket[b] = 0;
   }
+}
+
+// ------------------------------------------------------------------ stats
+constexpr int kVecThreads = 512;       // threads of the vectorised stats kernel
+constexpr int kVecPer = 32;            // values per thread (eight 16-byte loads)
+constexpr int kVecChunk = kVecThreads * kVecPer;
+
+template <bool kVec>
+__global__ void __launch_bounds__(kVec ? kVecThreads : kThreads)
+    sample_stats_kernel(const float* __restrict__ zt, const float* __restrict__ zd, int K, int V,
+                        float c2, int chunk, int n_chunks, const int32_t* __restrict__ draft,
+                        const float* __restrict__ u, int32_t* __restrict__ n_emit,
+                        int32_t* __restrict__ tokens, float2* __restrict__ part,
+                        float* __restrict__ dlogit, uint32_t* __restrict__ ticket,
+                        DrawInfo* __restrict__ info) {
+  constexpr int kT = kVec ? kVecThreads : kThreads;
+  const int c = blockIdx.x, rr = blockIdx.y, b = blockIdx.z;
+  const int rows = 2 * K + 1;
+  const float* row = row_ptr(zt, zd, b, rr, K, V);
+  const int lo = c * chunk, hi = min(V, lo + chunk);
+  // the drafts, read early (only the scene's last CTA needs them all); the
+  // CTA whose chunk holds the draft token of its row records that logit
+  __shared__ int s_x[128];
+  for (int j = threadIdx.x; j < K; j += kT) s_x[j] = __ldg(draft + static_cast<long long>(b) * K + j);
+  if (threadIdx.x == 0 && rr != K) {
+    const int j = rr < K ? rr : rr - K - 1;
+    const int x = __ldg(draft + static_cast<long long>(b) * K + j);
+    if (x >= lo && x < hi) dlogit[static_cast<long long>(b) * rows + rr] = __ldg(row + x);
+  }
+  float m = -INFINITY, s = 0.f;
+  if (kVec) {
+    // values lo + 4 (t + kT k) + e, k < 8, e < 4: one fixed order for both passes
+    float x[kVecPer];
+#pragma unroll
+    for (int k = 0; k < kVecPer / 4; ++k) {
+      const int i = lo + 4 * (threadIdx.x + kT * k);
+      const float4 v = i < hi ? __ldg(reinterpret_cast<const float4*>(row + i))
+                              : make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
+      x[4 * k + 0] = v.x;
+      x[4 * k + 1] = v.y;
+      x[4 * k + 2] = v.z;
+      x[4 * k + 3] = v.w;
+    }
+#pragma unroll
+    for (int e = 0; e < kVecPer; ++e) m = fmaxf(m, x[e]);
+    if (m != -INFINITY)
+#pragma unroll
+      for (int e = 0; e < kVecPer; ++e) s = __fadd_rn(s, x[e] == -INFINITY ? 0.f : wexp(x[e], m, c2));
+  } else {
+    // thread max, then thread sum, over a fixed strided subset of the chunk
+    for (int i = lo + threadIdx.x; i < hi; i += kT) m = fmaxf(m, __ldg(row + i));
+    if (m != -INFINITY)
+      for (int i = lo + threadIdx.x; i < hi; i += kT) s = __fadd_rn(s, wexp(__ldg(row + i), m, c2));
+  }
+  // warp then block merge, fixed tree
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float m2 = __shfl_xor_sync(0xffffffffu, m, o);
+    const float s2 = __shfl_xor_sync(0xffffffffu, s, o);
+    merge_ms(m, s, m2, s2, c2);
+  }
+  __shared__ float sm[kT / 32], ss[kT / 32];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (lane == 0) {
+    sm[warp] = m;
+    ss[warp] = s;
+  }
+  __syncthreads();
+  __shared__ bool s_last;
+  if (threadIdx.x == 0) {
+    float bm = sm[0], bs = ss[0];
+    for (int w = 1; w < kT / 32; ++w) merge_ms(bm, bs, sm[w], ss[w], c2);
+    part[(static_cast<long long>(b) * rows + rr) * n_chunks + c] = make_float2(bm, bs);
+    __threadfence();
+    s_last = atomicAdd(&ticket[b], 1u) == static_cast<uint32_t>(rows * n_chunks - 1);
+  }
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  accept_tail(zt, zd, K, V, c2, n_chunks, b, s_x, u, n_emit, tokens, part, dlogit, ticket, info, kT);
+}
+
+// Streaming stats: one CTA per (segment, row, scene) moves its segment of the
+// row through a ring of kStages 16 KB shared-memory stages with bulk copies
+// (warp 8 produces, warps 0-7 consume); a consumer thread keeps an online
+// (max, sum) over its 16 values of every stage in a fixed order. Rows must
+// start on 16-byte boundaries (V % 4 == 0, aligned bases).
+constexpr int kStreamConsumers = 256;
+constexpr int kStreamThreads = kStreamConsumers + 32;
+constexpr int kStageFloats = 4096;
+constexpr int kStreamStages = 4;
+constexpr uint32_t kStreamSpin = 1u << 22;
+
+__device__ __forceinline__ bool st_try_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\tmbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// bounded wait; false after the limit (the caller records a timeout)
+__device__ __forceinline__ bool st_wait(uint32_t bar, uint32_t parity) {
+#pragma unroll 1
+  for (uint32_t i = 0; i < kStreamSpin; ++i)
+    if (st_try_wait(bar, parity)) return true;
+  return false;
+}
+
+__global__ void __launch_bounds__(kStreamThreads)
+    sample_stats_stream_kernel(const float* __restrict__ zt, const float* __restrict__ zd, int K, int V,
+                               float c2, int seg, int n_seg, const int32_t* __restrict__ draft,
+                               const float* __restrict__ u, int32_t* __restrict__ n_emit,
+                               int32_t* __restrict__ tokens, float2* __restrict__ part,
+                               float* __restrict__ dlogit, uint32_t* __restrict__ ticket,
+                               DrawInfo* __restrict__ info) {
+  extern __shared__ __align__(128) float stage_raw[];  // [kStreamStages][kStageFloats]
+  float (*stage)[kStageFloats] = reinterpret_cast<float (*)[kStageFloats]>(stage_raw);
+  __shared__ __align__(8) uint64_t full[kStreamStages], empty[kStreamStages];
+  __shared__ int s_x[128];
+  __shared__ int s_timeout;
+  const int c = blockIdx.x, rr = blockIdx.y, b = blockIdx.z;
+  const int rows = 2 * K + 1;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const float* row = row_ptr(zt, zd, b, rr, K, V);
+  const int lo = c * seg, hi = min(V, lo + seg);
+  const int n_st = hi > lo ? (hi - lo + kStageFloats - 1) / kStageFloats : 0;
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < kStreamStages; ++i) {
+      asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(static_cast<uint32_t>(__cvta_generic_to_shared(&full[i]))));
+      asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(static_cast<uint32_t>(__cvta_generic_to_shared(&empty[i]))),
+                   "r"(kStreamConsumers / 32));
+    }
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    s_timeout = 0;
+  }
+  for (int j = threadIdx.x; j < K; j += kStreamThreads) s_x[j] = __ldg(draft + static_cast<long long>(b) * K + j);
+  __syncthreads();
+  float m = -INFINITY, s = 0.f;
+  if (warp == kStreamConsumers / 32) {
+    // ---- producer: thread 0 of warp 8; also records the draft token's logit
+    if (lane == 0) {
+      if (rr != K) {
+        const int j = rr < K ? rr : rr - K - 1;
+        const int x = s_x[j];
+        if (x >= lo && x < hi) dlogit[static_cast<long long>(b) * rows + rr] = __ldg(row + x);
+      }
+      for (int t = 0; t < n_st; ++t) {
+        const int st = t % kStreamStages;
+        if (t >= kStreamStages &&
+            !st_wait(static_cast<uint32_t>(__cvta_generic_to_shared(&empty[st])),
+                     static_cast<uint32_t>(((t / kStreamStages) - 1) & 1))) {
+          s_timeout = 1;
+          break;
+        }
+        const int p0 = lo + t * kStageFloats;
+        const uint32_t bytes = static_cast<uint32_t>(min(kStageFloats, hi - p0) * 4);
+        const uint32_t fb = static_cast<uint32_t>(__cvta_generic_to_shared(&full[st]));
+        asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(fb), "r"(bytes) : "memory");
+        asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                         static_cast<uint32_t>(__cvta_generic_to_shared(&stage[st][0]))),
+                     "l"(row + p0), "r"(bytes), "r"(fb)
+                     : "memory");
+      }
+    }
+  } else {
+    // ---- consumers: thread t takes float4 t + 256 k (k < 4) of every stage
+    for (int t = 0; t < n_st; ++t) {
+      const int st = t % kStreamStages;
+      if (!st_wait(static_cast<uint32_t>(__cvta_generic_to_shared(&full[st])),
+                   static_cast<uint32_t>((t / kStreamStages) & 1))) {
+        s_timeout = 1;
+        break;
+      }
+      const int p0 = lo + t * kStageFloats;
+      const int nv = min(kStageFloats, hi - p0) / 4;  // float4s in this stage
+      float x[16];
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const int v = threadIdx.x + kStreamConsumers * k;
+        const float4 f = v < nv ? reinterpret_cast<const float4*>(stage[st])[v]
+                                : make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
+        x[4 * k + 0] = f.x;
+        x[4 * k + 1] = f.y;
+        x[4 * k + 2] = f.z;
+        x[4 * k + 3] = f.w;
+      }
+      __syncwarp();
+      if (lane == 0)
+        asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(static_cast<uint32_t>(__cvta_generic_to_shared(&empty[st])))
+                     : "memory");
+      float mx = x[0];
+#pragma unroll
+      for (int e = 1; e < 16; ++e) mx = fmaxf(mx, x[e]);
+      if (mx != -INFINITY) {
+        if (mx > m) {
+          if (m != -INFINITY) s = __fmul_rn(s, wexp(m, mx, c2));
+          m = mx;
+        }
+#pragma unroll
+        for (int e = 0; e < 16; ++e) s = __fadd_rn(s, wexp(x[e], m, c2));
+      }
+    }
+  }
+  // warp then block merge (consumer warps), fixed tree
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float m2 = __shfl_xor_sync(0xffffffffu, m, o);
+    const float s2 = __shfl_xor_sync(0xffffffffu, s, o);
+    merge_ms(m, s, m2, s2, c2);
+  }
+  __shared__ float sm[kStreamConsumers / 32], ss[kStreamConsumers / 32];
+  if (lane == 0 && warp < kStreamConsumers / 32) {
+    sm[warp] = m;
+    ss[warp] = s;
+  }
+  __syncthreads();
+  __shared__ bool s_last;
+  if (threadIdx.x == 0) {
+    if (s_timeout) sd_set_error(SD_DEVERR_TIMEOUT);
+    float bm = sm[0], bs = ss[0];
+    for (int w = 1; w < kStreamConsumers / 32; ++w) merge_ms(bm, bs, sm[w], ss[w], c2);
+    part[(static_cast<long long>(b) * rows + rr) * n_seg + c] = make_float2(bm, bs);
+    __threadfence();
+    s_last = atomicAdd(&ticket[b], 1u) == static_cast<uint32_t>(rows * n_seg - 1);
+  }
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  accept_tail(zt, zd, K, V, c2, n_seg, b, s_x, u, n_emit, tokens, part, dlogit, ticket, info,
+              kStreamThreads);
 }
 
 // ------------------------------------------------------------------ draw
@@ -363,13 +571,21 @@ __global__ void __launch_bounds__(kThreads)
 
 struct Plan {
   int chunk1, n1, chunk2, n2;
+  bool vec;
+  int chunk_scalar, n_scalar;  // the scalar stats kernel's chunking (unaligned rows)
 };
 
+// Vectorised stats when every row starts on a 16-byte boundary (V a multiple
+// of 4 and a 16-byte-aligned base, checked at the call).
 Plan plan(int V) {
   Plan p;
-  p.chunk1 = 4096;
+  p.vec = V % 4 == 0;
+  p.chunk1 = p.vec ? kVecChunk : 4096;
   while ((V + p.chunk1 - 1) / p.chunk1 > kMaxChunks) p.chunk1 *= 2;
   p.n1 = (V + p.chunk1 - 1) / p.chunk1;
+  p.chunk_scalar = 4096;
+  while ((V + p.chunk_scalar - 1) / p.chunk_scalar > kMaxChunks) p.chunk_scalar *= 2;
+  p.n_scalar = (V + p.chunk_scalar - 1) / p.chunk_scalar;
   p.chunk2 = 2048;
   while ((V + p.chunk2 - 1) / p.chunk2 > kMaxChunks) p.chunk2 *= 2;
   p.n2 = (V + p.chunk2 - 1) / p.chunk2;
@@ -377,7 +593,7 @@ Plan plan(int V) {
 }
 
 struct Layout {
-  size_t part, ticket1, info, sums, ticket2, total;
+  size_t part, dlogit, ticket1, info, sums, ticket2, total;
 };
 
 Layout layout(int B, int K, const Plan& p) {
@@ -388,13 +604,43 @@ Layout layout(int B, int K, const Plan& p) {
     off += (bytes + 255) / 256 * 256;
     return at;
   };
-  l.part = take(static_cast<size_t>(B) * (2 * K + 1) * p.n1 * sizeof(float2));
+  // room for the scalar chunking's partials too (rows found unaligned at the call)
+  l.part = take(static_cast<size_t>(B) * (2 * K + 1) * (p.n_scalar > p.n1 ? p.n_scalar : p.n1) * sizeof(float2));
+  l.dlogit = take(static_cast<size_t>(B) * (2 * K + 1) * sizeof(float));
   l.ticket1 = take(static_cast<size_t>(B) * 4);
   l.info = take(static_cast<size_t>(B) * sizeof(DrawInfo));
   l.sums = take(static_cast<size_t>(B) * p.n2 * sizeof(float2));
   l.ticket2 = take(static_cast<size_t>(B) * 4);
   l.total = off;
   return l;
+}
+
+constexpr int kStreamSmem = kStreamStages * kStageFloats * 4;
+
+// SMs of the current device, once the streaming kernel's shared-memory
+// attribute is set there; 0 when either call fails (the one-shot kernel runs).
+int stream_sms() {
+  static int cache[64];
+  static bool done[64];
+  static std::mutex mu;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) {
+    (void)cudaGetLastError();
+    return 0;
+  }
+  std::lock_guard<std::mutex> lock(mu);
+  if (!done[dev]) {
+    done[dev] = true;
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+        cudaFuncSetAttribute(sample_stats_stream_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             kStreamSmem) != cudaSuccess) {
+      (void)cudaGetLastError();
+      n = 0;
+    }
+    cache[dev] = n;
+  }
+  return cache[dev];
 }
 
 }  // namespace
@@ -414,19 +660,40 @@ extern "C" sd_status sd_accept_sample(const float* z_target, const float* z_draf
   if (B == 0) return SD_OK;
   if (!z_target || !u || !n_emit || !tokens || (K > 0 && (!z_draft || !draft)))
     return SD_ERR_INVALID_ARG;
-  const Plan p = plan(V);
+  Plan p = plan(V);
   const Layout l = layout(B, K, p);
+  // the vectorised stats also need 16-byte-aligned rows (same workspace either way)
+  if ((reinterpret_cast<uintptr_t>(z_target) & 15) || (K > 0 && (reinterpret_cast<uintptr_t>(z_draft) & 15))) {
+    p.vec = false;
+    p.chunk1 = p.chunk_scalar;
+    p.n1 = p.n_scalar;
+  }
   if (!ws || ws_bytes < l.total || !sd_aligned16(ws)) return SD_ERR_WORKSPACE;
   char* w = static_cast<char*>(ws);
   auto* part = reinterpret_cast<float2*>(w + l.part);
+  auto* dlogit = reinterpret_cast<float*>(w + l.dlogit);
   auto* ticket1 = reinterpret_cast<uint32_t*>(w + l.ticket1);
   auto* info = reinterpret_cast<DrawInfo*>(w + l.info);
   auto* sums = reinterpret_cast<float2*>(w + l.sums);
   auto* ticket2 = reinterpret_cast<uint32_t*>(w + l.ticket2);
   const float c2 = static_cast<float>(kLog2e / static_cast<double>(temperature));
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-  sample_stats_kernel<<<dim3(p.n1, 2 * K + 1, B), kThreads, 0, st>>>(
-      z_target, z_draft, K, V, c2, p.chunk1, p.n1, draft, u, n_emit, tokens, part, ticket1, info);
+  const int n_sm = stream_sms();
+  if (p.vec && n_sm > 0) {
+    // segments of whole stages, about two CTAs per SM over all (row, scene) pairs
+    const long long rows_all = static_cast<long long>(2 * K + 1) * B;
+    long long n_seg = (2LL * n_sm + rows_all - 1) / rows_all;
+    n_seg = n_seg < 1 ? 1 : (n_seg > p.n1 ? p.n1 : n_seg);
+    const int seg = static_cast<int>(((V + n_seg - 1) / n_seg + kStageFloats - 1) / kStageFloats * kStageFloats);
+    const int ns = (V + seg - 1) / seg;
+    sample_stats_stream_kernel<<<dim3(ns, 2 * K + 1, B), kStreamThreads, kStreamSmem, st>>>(
+        z_target, z_draft, K, V, c2, seg, ns, draft, u, n_emit, tokens, part, dlogit, ticket1, info);
+  } else if (p.vec)
+    sample_stats_kernel<true><<<dim3(p.n1, 2 * K + 1, B), kVecThreads, 0, st>>>(
+        z_target, z_draft, K, V, c2, p.chunk1, p.n1, draft, u, n_emit, tokens, part, dlogit, ticket1, info);
+  else
+    sample_stats_kernel<false><<<dim3(p.n1, 2 * K + 1, B), kThreads, 0, st>>>(
+        z_target, z_draft, K, V, c2, p.chunk1, p.n1, draft, u, n_emit, tokens, part, dlogit, ticket1, info);
   SD_CHECK_LAUNCH();
   sample_draw_kernel<<<dim3(p.n2, B), kThreads, 0, st>>>(z_target, z_draft, K, V, c2, p.chunk2,
                                                           p.n2, u, tokens, info, sums, ticket2);
