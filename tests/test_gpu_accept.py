@@ -139,11 +139,13 @@ def test_sample_equal_distributions_always_accept():
     assert torch.equal(t[:, :K].cpu(), draft)
 
 
-def test_sample_output_law_by_enumeration_on_gpu():
-    # Leviathan/Chen on a 5-token vocabulary through the kernel: every draft
+# V = 5 takes the scalar stats kernel, V = 8 (a multiple of 4) the streaming one
+@pytest.mark.parametrize("V", [5, 8])
+def test_sample_output_law_by_enumeration_on_gpu(V):
+    # Leviathan/Chen on a small vocabulary through the kernel: every draft
     # token x (weight q(x)) times an N x N grid of uniforms, in one batch.
     rng = np.random.default_rng(81)
-    V, T, N = 5, 0.8, 64
+    T, N = 0.8, 64
     z_t = (rng.standard_normal((2, V)) * 1.5).astype(np.float32)
     z_d = (rng.standard_normal((1, V)) * 1.5).astype(np.float32)
     grid = (np.arange(N) + 0.5) / N
