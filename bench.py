@@ -351,6 +351,92 @@ def time_sample_accept(device, reps=20):
     return ms * 1e3, nbytes
 
 
+def time_draft_steps(device, reps=20):
+    """The draft's propose loop for one attention layer (16 q / 4 KV heads x 128,
+    L = 4096, FlatRoPE = M-RoPE at (m, m, m)): 7 single-row decode steps, each one
+    sd_verify_layer call (rotation at m = L + s, append, attention over
+    L + s + 1 keys), then the rollback to the committed length and the reset
+    to L, in a graph. Returns us per step."""
+    from paper_2606_31160_gb300 import sd, workloads
+    w = workloads.draft_flat()
+    L_, steps = w["L"], w["steps"]
+    lens = torch.full((1,), L_, dtype=torch.int32, device=device)
+    lens0 = lens.clone()
+    cache = sd.KVCache(w["k_cache"].to(device), w["v_cache"].to(device), lens)
+    q = [w["q"][s].to(device) for s in range(steps)]
+    k = [w["k_new"][s].to(device) for s in range(steps)]
+    v = [w["v_new"][s].to(device) for s in range(steps)]
+    pos = [torch.full((1, 1, 3), L_ + s, dtype=torch.int32, device=device) for s in range(steps)]
+    out = [torch.empty_like(x) for x in q]
+    ws = sd.workspace(sd.layer_workspace_bytes(1, 1, 16, 4, 128, cache.shape[2]), device)
+    committed = torch.tensor([w["committed"]], dtype=torch.int32, device=device)
+
+    def loop():
+        for s in range(steps):
+            sd.verify_layer(q[s], k[s], v[s], pos[s], SECTIONS, cache, 0, w["base"], out=out[s], ws=ws)
+        sd.kv_rollback(lens, committed, steps)
+        lens.copy_(lens0, non_blocking=True)
+
+    g = capture(loop)
+    ms = time_graph(g, reps)
+    assert sd.get_device_error() == 0
+    return ms * 1e3 / steps
+
+
+def time_stochastic_step(device, layers=LAYERS):
+    """The stochastic-acceptance step: 36 fused target layers at B = 8 (L = 4096,
+    R = 8, 32 q / 8 KV x 128, one cache per layer: 4.84 GB streamed from HBM),
+    then rejection sampling over fp32 logits [8][8][151936] (T = 0.6) and the
+    rollback of all 36 lengths to the sampled commits, in a graph. Caches and
+    rows ~ N(0, 1) bf16 from a seeded device generator. Returns (us per step,
+    algorithmic bytes per step)."""
+    from paper_2606_31160_gb300 import sd, workloads
+    B_ = 8
+    gen = torch.Generator(device=device)
+    gen.manual_seed(5000)
+    cap = L + R
+
+    def normal(*shape):
+        return torch.randn(shape, generator=gen, device=device, dtype=torch.float32).to(torch.bfloat16)
+
+    lens = torch.full((layers, B_), L, dtype=torch.int32, device=device)
+    lens0 = lens.clone()
+    caches, qs, ks, vs, outs, wss = [], [], [], [], [], []
+    for l in range(layers):
+        kc = torch.zeros((B_, HKV, cap, D), dtype=torch.bfloat16, device=device)
+        vc = torch.zeros_like(kc)
+        kc[:, :, :L] = normal(B_, HKV, L, D)
+        vc[:, :, :L] = normal(B_, HKV, L, D)
+        caches.append(sd.KVCache(kc, vc, lens[l]))
+        qs.append(normal(B_, R, HQ, D))
+        ks.append(normal(B_, R, HKV, D))
+        vs.append(normal(B_, R, HKV, D))
+        outs.append(torch.empty_like(qs[-1]))
+        wss.append(sd.workspace(sd.layer_workspace_bytes(B_, R, HQ, HKV, D, cap), device))
+    qpos = torch.from_numpy(np.stack([workloads.text_positions(544, R)] * B_)).to(device)
+    w = workloads.stochastic()
+    zt, zd, dr, u = (w["z_target"].to(device), w["z_draft"].to(device), w["draft"].to(device), w["u"].to(device))
+    ws_s = sd.workspace(sd.sample_workspace_bytes(B_, K, V), device)
+    n_emit = torch.zeros(B_, dtype=torch.int32, device=device)
+    tokens = torch.zeros((B_, R), dtype=torch.int32, device=device)
+
+    def step():
+        for l in range(layers):
+            sd.verify_layer(qs[l], ks[l], vs[l], qpos, SECTIONS, caches[l], 0, BASE, out=outs[l], ws=wss[l],
+                            early=l > 0)
+        sd.accept_sample(zt, zd, dr, u, w["temperature"], ws=ws_s, n_emit=n_emit, tokens=tokens)
+        sd.kv_rollback(lens, n_emit, R)
+        lens.copy_(lens0, non_blocking=True)
+
+    g = capture(step)
+    ms = time_graph(g, 10)
+    assert sd.get_device_error() == 0
+    logits = (B_ * R * V + B_ * K * V) * 4
+    del caches, qs, ks, vs, outs, wss
+    torch.cuda.empty_cache()
+    return ms * 1e3, layers * layer_bytes(B_) + logits  # the same accounting as the main step
+
+
 def oracle_layer_sample(case, logits, draft):
     """The float64 oracle on one layer of the step plus the acceptance:
     returns bytes of the workload it covered (same accounting as the GPU)."""
@@ -496,8 +582,11 @@ def main():
     a1.synchronize()
     ms_e2e = max_over_ranks(a0.elapsed_time(a1) / e2e_steps, world, device)
     assert sd.get_device_error() == 0
-    # the stochastic-acceptance workload (rejection sampling over B = 8 scenes)
+    # the stochastic-acceptance workload (rejection sampling over B = 8 scenes),
+    # its whole step (36 layers at B = 8 + sampling), and the draft's propose loop
     sample_us, sample_bytes = time_sample_accept(device) if rank == 0 else (None, None)
+    draft_us = time_draft_steps(device) if rank == 0 else None
+    stoch_us, stoch_bytes = time_stochastic_step(device) if rank == 0 else (None, None)
     assert sd.get_device_error() == 0
 
     if rank != 0:
@@ -542,6 +631,9 @@ def main():
         "accept_us": round(ms_accept * 1e3, 3),
         "sample_accept_us": round(sample_us, 3),
         "sample_accept_gbs": round(sample_bytes / (sample_us * 1e-6) / 1e9, 1),
+        "draft_step_us": round(draft_us, 3),
+        "stochastic_step_us": round(stoch_us, 2),
+        "stochastic_step_gbs": round(stoch_bytes / (stoch_us * 1e-6) / 1e9, 1),
         "bytes_per_step": step_bytes(1),
         "roofline": {
             "kernel": "sd_verify_layer -> verify_attn_tc_kernel<fused> (M-RoPE + append + attention, tcgen05)",

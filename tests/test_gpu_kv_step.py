@@ -121,3 +121,27 @@ def test_k_zero_is_plain_decode():
     qq = torch.from_numpy(to64(q)[0]).permute(1, 0, 2)
     ref = torch.nn.functional.scaled_dot_product_attention(qq, kk, vv).permute(1, 0, 2).numpy()
     assert np.abs(to64(out)[0] - ref).max() <= ATTN_ATOL
+
+
+def test_draft_step_as_one_fused_layer_call():
+    # FlatRoPE is M-RoPE with (m, m, m): the draft's single-row decode step
+    # (rotation at m = L + s, append, attention over L + s + 1 keys) as one
+    # sd_verify_layer call per step, against the oracle's 1D rotation and attention
+    w = workloads.draft_flat()
+    L, steps = w["L"], w["steps"]
+    cache = sd.KVCache(w["k_cache"].cuda(), w["v_cache"].cuda(), torch.tensor([L], dtype=torch.int32).cuda())
+    for s in range(steps):
+        q, k = w["q"][s].cuda(), w["k_new"][s].cuda()
+        pos = torch.full((1, 1, 3), L + s, dtype=torch.int32, device="cuda")
+        out = sd.verify_layer(q, k, w["v_new"][s].cuda(), pos, (16, 24, 24), cache, 0, w["base"])
+        ref_q = oracle.rope_1d(to64(w["q"][s]), L + s, w["base"])
+        ref_k = oracle.rope_1d(to64(w["k_new"][s]), L + s, w["base"])
+        assert np.all(np.abs(to64(q) - ref_q) <= rope_bound(ref_q, pair_magnitude(to64(w["q"][s]))))
+        assert np.all(np.abs(to64(k) - ref_k) <= rope_bound(ref_k, pair_magnitude(to64(w["k_new"][s]))))
+        assert torch.equal(cache.k[0, :, L + s], k[0, 0]) and torch.equal(cache.v[0, :, L + s], w["v_new"][s][0, 0].cuda())
+        ref_o = oracle.verify_attention(to64(q), to64(cache.k), to64(cache.v), cache.len.cpu().numpy())
+        assert np.abs(to64(out) - ref_o).max() <= ATTN_ATOL
+    assert cache.len.item() == L + steps
+    sd.kv_rollback(cache.len, torch.tensor([w["committed"]], dtype=torch.int32, device="cuda"), steps)
+    assert cache.len.item() == L + w["committed"]
+    assert sd.get_device_error() == 0
