@@ -11,6 +11,8 @@ Driving", arxiv 2606.31160):
   accept.py     greedy longest-prefix acceptance + bonus (Eqs. accept, commit)
                 and Leviathan/Chen rejection sampling (cited in Sec. 1 and 2)
   kv.py         KV-cache append and rollback to the committed length (Eq. commit)
+  budget.py     per-segment attention mass and normalised entropy of the verify
+                rows (Sec. 3.2, Table tab:attn-budget)
 
 Only tests/, __graft_entry__.smoke() and bench.py (its cpu_baseline leg and
 its --impl reference arm) may import it. The CUDA library and its Python
@@ -28,10 +30,11 @@ from .rope import (rope_frequencies, axis_assignment, mrope_apply, rope_1d,
 from .attention import verify_attention
 from .accept import accept_greedy, accept_sample, argmax_lowest
 from .kv import kv_append, kv_rollback
+from .budget import attention_budget
 
 __all__ = [
     "rope_frequencies", "axis_assignment", "mrope_apply", "rope_1d",
     "rope_1d_matrix", "flatrope_positions", "verify_attention",
     "accept_greedy", "accept_sample", "argmax_lowest", "kv_append",
-    "kv_rollback",
+    "kv_rollback", "attention_budget",
 ]
