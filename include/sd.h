@@ -180,6 +180,30 @@ sd_status sd_verify_attention(const void* q, const sd_kv_cache* cache, void* out
  */
 sd_status sd_set_cluster_size(int cluster_size);
 
+/*
+ * Attention budget of the verify rows (Sec. 3.2 "Empirical confirmation",
+ * Table tab:attn-budget), a diagnostic beside the verify path. For scene b,
+ * query head h and row i, with p the softmax of q . k * scale over the keys
+ * row i sees (0 .. len[b] - R + i, as in sd_verify_attention) and
+ * L_b = len[b] - R:
+ *   mass[b][i][h][0] = sum of p over the visual keys [0, n_visual[b])
+ *   mass[b][i][h][1] = over the trajectory / prompt-text keys [n_visual[b], L_b)
+ *   mass[b][i][h][2] = over the rows generated in this step [L_b, L_b + i]
+ *   entropy[b][i][h] = entropy (nats) of p over the keys from n_visual[b] on,
+ *                      renormalised, divided by the log of their number
+ *                      (0 when there is at most one such key)
+ *   q: [B][R][Hq][D] bf16 (rotated), cache: keys appended (len includes R),
+ *   n_visual: int32 [B] device, mass: fp32 [B][R][Hq][3] device,
+ *   entropy: fp32 [B][R][Hq] device; scale: 0 selects 1/sqrt(D).
+ * Exact rather than fast: two fp32 passes over the keys on the CUDA cores.
+ * D in {64, 128}, Hq % Hkv == 0. A scene with len[b] < R or len[b] >
+ * capacity sets SD_DEVERR_LENGTH and is left unwritten; n_visual[b] outside
+ * [0, L_b] sets it too and is clamped.
+ */
+sd_status sd_attention_budget(const void* q, const sd_kv_cache* cache, int R, int Hq, float scale,
+                              const int32_t* n_visual, float* mass, float* entropy,
+                              sd_stream_t stream);
+
 /* sd_verify_layer flag: see below. */
 #define SD_LAYER_PREFIX_EARLY 1
 

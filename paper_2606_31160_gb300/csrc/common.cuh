@@ -35,6 +35,7 @@ cudaError_t sd_take_error_attention(uint32_t* bits);
 cudaError_t sd_take_error_attention_tc(uint32_t* bits);
 cudaError_t sd_take_error_greedy(uint32_t* bits);
 cudaError_t sd_take_error_sample(uint32_t* bits);
+cudaError_t sd_take_error_budget(uint32_t* bits);
 
 // Verify attention on the tcgen05 path (attention_tc.cu). Sets *handled when
 // the shape is one it serves (head_dim 128, G * R <= 32) and it launched.

@@ -60,6 +60,7 @@ _SIGNATURES = {
     "sd_accept_sample": ([_vp, _vp, _i, _i, _i, _f, _vp, _vp, _vp, _vp, _vp, _sz, _vp], _i),
     "sd_get_device_error": ([_vp, ctypes.POINTER(ctypes.c_uint32)], _i),
     "sd_set_cluster_size": ([_i], _i),
+    "sd_attention_budget": ([_vp, ctypes.POINTER(KVCacheStruct), _i, _i, _f, _vp, _vp, _vp, _vp], _i),
 }
 
 
@@ -226,6 +227,23 @@ def verify_attention(q, cache, out=None, scale=0.0, ws=None):
                                      _dev(out, "out", torch.bfloat16), R, Hq, float(scale), wp, nbytes,
                                      _stream()), "sd_verify_attention")
     return out
+
+
+def attention_budget(q, cache, n_visual, scale=0.0, mass=None, entropy=None):
+    """Per (scene, row, head): attention mass on the visual, trajectory / text and
+    generated keys, and the normalised entropy over the non-visual keys.
+    q [B,R,Hq,D] (rotated), cache appended, n_visual int32 [B] -> (mass [B,R,Hq,3],
+    entropy [B,R,Hq]) float32."""
+    B, R, Hq, D = q.shape
+    if mass is None:
+        mass = torch.empty((B, R, Hq, 3), dtype=torch.float32, device=q.device)
+    if entropy is None:
+        entropy = torch.empty((B, R, Hq), dtype=torch.float32, device=q.device)
+    _check(lib().sd_attention_budget(_dev(q, "q", torch.bfloat16), cache.struct, R, Hq, float(scale),
+                                     _dev(n_visual, "n_visual", torch.int32), _dev(mass, "mass", torch.float32),
+                                     _dev(entropy, "entropy", torch.float32), _stream()),
+           "sd_attention_budget")
+    return mass, entropy
 
 
 SD_LAYER_PREFIX_EARLY = 1
