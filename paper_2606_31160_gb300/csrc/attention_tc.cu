@@ -63,7 +63,6 @@ constexpr int kD = 128;         // head dim
 constexpr int kStageKeys = 128; // M of S^T
 constexpr int kHalf = kStageKeys * 128;     // one 64-column half of a 128-key tile (16 KB)
 constexpr int kKV = 2 * kHalf;              // one K (or V) tile of 128 keys (32 KB)
-constexpr int kMaxNew = 16;                 // new rows the fused kernel takes
 constexpr int kNewRow = kD * 2;             // one new key / value row (256 B)
 constexpr int kSoftWarps = 8;
 constexpr int kSoftThreads = 32 * kSoftWarps;
@@ -82,6 +81,7 @@ struct Cfg {
   static_assert(kR == 32 || kR == 64, "row tile");
   static constexpr int kRows = kR;
   static constexpr int kRpt = kR / 2;                       // rows per softmax thread
+  static constexpr int kMaxNew = kR == 32 ? 16 : 32;        // new rows the fused kernel takes
   // K and V rings of kStages tiles each: a K slot is free once its S product
   // is done, a V slot once its PV product is
   static constexpr int kStages = kR == 32 ? 3 : 2;
@@ -103,8 +103,9 @@ struct Cfg {
   static constexpr int kOffBar = kOffNewV + kMaxNew * kNewRow;
   // barriers: full_k[S] full_v[S] p_full[2] s_ready[S] pv_done[S] q_full recv decide
   static constexpr int kNumBars = 4 * kStages + 5;
-  static constexpr int kOffMisc = round_up(kOffBar + kNumBars * 8, 16);  // tmem slot, excess, decision, len
-  static constexpr int kOffRowA = kOffMisc + 16;            // [kR] per-row results (reductions)
+  // tmem slot, excess, decision, len (and, 64 rows, the last reader of the new key rows)
+  static constexpr int kOffMisc = round_up(kOffBar + kNumBars * 8, 16);
+  static constexpr int kOffRowA = kOffMisc + (kR == 32 ? 16 : 32);  // [kR] per-row results (reductions)
   static constexpr int kOffRef = kOffRowA + kR * 4;         // [kR] per-row references
   static constexpr int kOffLim = kOffRef + kR * 4;          // [kR] per-row causal key limits
   static constexpr int kSmemBytes = kOffLim + kR * 4 + 1024;
@@ -298,6 +299,7 @@ struct TcArgs {
   __nv_bfloat16* vc;
   const int32_t* pos;       // [B][R][3]
   uint32_t* ticket;         // [B] per-scene CTA tickets (zeroed, re-armed)
+  uint32_t* kv_ticket;      // [B][Hkv] read-before-write-back tickets (several m-blocks)
   int early;                // prefix, len and pos may be read before the dependency wait
   int R, Hq, Hkv, G, M, cap, n_mblocks;
   float inv_g;              // 1 / G: p / G == int((p + 0.5) / G) exactly for the p < 128 used here
@@ -358,6 +360,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::kOffMisc);
   int* s_excess = reinterpret_cast<int*>(smem + C::kOffMisc + 4);
   int* s_redo = reinterpret_cast<int*>(smem + C::kOffMisc + 8);
+  int* s_kvlast = reinterpret_cast<int*>(smem + C::kOffMisc + 16);  // 64 rows only
   float* row_a = reinterpret_cast<float*>(smem + C::kOffRowA);  // [kR] reduction results
   float* row_ref = reinterpret_cast<float*>(smem + C::kOffRef); // [kR] references
   int* row_lim = reinterpret_cast<int*>(smem + C::kOffLim);      // [kR] last key a row sees
@@ -574,8 +577,17 @@ __global__ void __launch_bounds__(kThreads, 1)
                    ((static_cast<long long>(b) * a.R + i) * a.Hq + kvh * a.G + (p - i * a.G)) * kD + c * 8;
         q_cs[u] = i * 64 + c * 4;
       }
-      const bool has_kv = kFused && valid && st < a.R * 16;
-      const long long kv_src = ((static_cast<long long>(b) * a.R + (st >> 4)) * a.Hkv + kvh) * kD + (st & 15) * 8;
+      // new key / value rows: chunk st + u * 256 (row >> 4, 16-byte chunk & 15);
+      // one chunk a thread with 32 rows (16 new rows), two with 64 (32)
+      constexpr int kKvc = C::kMaxNew * 16 / kSoftThreads;
+      bool has_kv[kKvc];
+      long long kv_src[kKvc];
+#pragma unroll
+      for (int u = 0; u < kKvc; ++u) {
+        const int idx = st + u * kSoftThreads;
+        has_kv[u] = kFused && valid && idx < a.R * 16;
+        kv_src[u] = ((static_cast<long long>(b) * a.R + (idx >> 4)) * a.Hkv + kvh) * kD + (idx & 15) * 8;
+      }
       // Fused: iteration 0 runs BEFORE the dependency wait on whatever the
       // rows hold: it brings this code into the instruction cache and the rows
       // into L2, and iteration 1 overwrites everything it stored. The loads
@@ -583,13 +595,14 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll 1
       for (int it = kFused ? 0 : 1; it < 2; ++it) {
         if (kFused && it == 1 && a.early) griddep_wait();  // the raw rows come from earlier kernels
-        uint4 qv[kQc], kv = make_uint4(0, 0, 0, 0), vv = make_uint4(0, 0, 0, 0);
+        uint4 qv[kQc], kv[kKvc], vv[kKvc];
 #pragma unroll
         for (int u = 0; u < kQc; ++u)
           qv[u] = q_ok[u] ? __ldcg(reinterpret_cast<const uint4*>(q_src[u])) : make_uint4(0, 0, 0, 0);
-        if (has_kv) {
-          kv = __ldcg(reinterpret_cast<const uint4*>(a.k_new + kv_src));
-          vv = __ldcg(reinterpret_cast<const uint4*>(a.v_new + kv_src));
+#pragma unroll
+        for (int u = 0; u < kKvc; ++u) {
+          kv[u] = has_kv[u] ? __ldcg(reinterpret_cast<const uint4*>(a.k_new + kv_src[u])) : make_uint4(0, 0, 0, 0);
+          vv[u] = has_kv[u] ? __ldcg(reinterpret_cast<const uint4*>(a.v_new + kv_src[u])) : make_uint4(0, 0, 0, 0);
         }
         // (fused: M-RoPE of) the packed query rows, straight into the swizzled tile
 #pragma unroll
@@ -604,18 +617,22 @@ __global__ void __launch_bounds__(kThreads, 1)
           st_shared_v4(qs + (c >> 3) * C::kQHalf + row * 128 + (((c & 7) ^ (row & 7)) << 4), w[0], w[1],
                        w[2], w[3]);
         }
-        // the new key rows (rotated) and value rows of this head
-        if (has_kv) {
-          const int i = st >> 4, c = st & 15;
-          const float2* cs = cs_tab + i * 64 + c * 4;
-          uint32_t w[4] = {kv.x, kv.y, kv.z, kv.w};
+        // the new key rows (rotated) and value rows of this head; value rows
+        // past R stay zero (the merge reads all kMaxNew rows)
 #pragma unroll
-          for (int j = 0; j < 4; ++j) w[j] = sd_rope_pair(w[j], cs[j].x, cs[j].y);
-          st_shared_v4(base + C::kOffNewK + i * kNewRow + c * 16, w[0], w[1], w[2], w[3]);
-          st_shared_v4(base + C::kOffNewV + i * kNewRow + c * 16, vv.x, vv.y, vv.z, vv.w);
-        } else if (kFused && st < kMaxNew * 16) {
-          // value rows past R stay zero: the merge reads all kMaxNew rows
-          st_shared_v4(base + C::kOffNewV + (st >> 4) * kNewRow + (st & 15) * 16, 0u, 0u, 0u, 0u);
+        for (int u = 0; u < kKvc; ++u) {
+          if (!kFused) break;
+          const int idx = st + u * kSoftThreads, i = idx >> 4, c = idx & 15;
+          if (has_kv[u]) {
+            const float2* cs = cs_tab + i * 64 + c * 4;
+            uint32_t w[4] = {kv[u].x, kv[u].y, kv[u].z, kv[u].w};
+#pragma unroll
+            for (int j = 0; j < 4; ++j) w[j] = sd_rope_pair(w[j], cs[j].x, cs[j].y);
+            st_shared_v4(base + C::kOffNewK + i * kNewRow + c * 16, w[0], w[1], w[2], w[3]);
+            st_shared_v4(base + C::kOffNewV + i * kNewRow + c * 16, vv[u].x, vv[u].y, vv[u].z, vv[u].w);
+          } else {
+            st_shared_v4(base + C::kOffNewV + i * kNewRow + c * 16, 0u, 0u, 0u, 0u);
+          }
         }
       }
       // causal limit of each packed row: row p = i * G + g is new row i and
@@ -627,6 +644,20 @@ __global__ void __launch_bounds__(kThreads, 1)
         mbar_arrive(QFULL);
         // every older kernel has finished: the next layer may launch
         if (kFused) griddep_launch();
+        // with several m-blocks the head's raw key rows are read by several
+        // clusters: the last of the head's CTAs to have read them writes the
+        // rotated rows back (the fence orders this CTA's reads before its ticket)
+        if constexpr (kR == 64) {
+          if (kFused && valid) {
+            if (a.n_mblocks > 1) {
+              __threadfence();
+              *s_kvlast = atomicAdd(&a.kv_ticket[b * a.Hkv + kvh], 1u) ==
+                          static_cast<uint32_t>(csize * a.n_mblocks - 1);
+            } else {
+              *s_kvlast = rank == csize - 1;
+            }
+          }
+        }
       }
     }
 
@@ -898,53 +929,59 @@ __global__ void __launch_bounds__(kThreads, 1)
       named_bar_sync(2, kSoftThreads);
     }
     // ---- merge of the rows this CTA owns; slot c * rpc + rr came from rank c.
-    // A warp takes 64 adjacent outputs of one row (a thread two adjacent d).
-    // The row's weights come lane-parallel: lane c < csize holds partial c's
-    // (m, l), lane csize + n new key n's score; the warp reduces them with
-    // shuffles and broadcasts each weight. The output loads do not depend on
-    // the counts (slots past the cluster read partial 0, value rows past R are
-    // zero; their weights are 0), so they issue together.
+    // A thread takes one row and two adjacent d: it forms the row's weights
+    // itself (partials c < csize and new keys n < R, all loads issued
+    // together), then its two outputs.
     mbar_wait(RECV, 0);
     const float* recv = reinterpret_cast<const float*>(smem + C::kRecv);
     const int n_new = (kFused && valid) ? a.R : 0;
 #pragma unroll 1
-    for (int idx = st; idx < my_rows * (kD / 2); idx += kSoftThreads) {  // the row is warp-uniform
+    for (int idx = st; idx < my_rows * (kD / 2); idx += kSoftThreads) {
       const int rr = idx / (kD / 2), d = 2 * (idx % (kD / 2));
       const int row = mrow0 + rr;
       const int p = mblock * kR + row;
-      float m = -INFINITY, l = 0.f;
-      if (lane < csize) {
-        const float2 ml = *reinterpret_cast<const float2*>(recv + (lane * rpc + rr) * kRowF + kD);
-        m = ml.x;
-        l = ml.y;
-      } else if (lane < csize + n_new) {
-        m = s_new[rr * a.R + (lane - csize)];
-        l = 1.f;
+      float mc[16], lc[16], sn[C::kMaxNew];
+#pragma unroll
+      for (int c = 0; c < 16; ++c) {
+        // slots past the cluster read partial 0 (always present) with weight 0
+        const float* part = recv + ((c < csize ? c : 0) * rpc + rr) * kRowF + kD;
+        mc[c] = c < csize ? part[0] : -INFINITY;
+        lc[c] = c < csize ? part[1] : 0.f;
       }
-      float mx = m;
 #pragma unroll
-      for (int w = 16; w >= 1; w >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, w));
-      const float f = ex2(m - (mx == -INFINITY ? 0.f : mx));  // ex2(-inf) = 0
-      float lsum = f * l;
+      for (int n = 0; n < C::kMaxNew; ++n) sn[n] = n < n_new ? s_new[rr * a.R + n] : -INFINITY;
+      float mx = -INFINITY;
 #pragma unroll
-      for (int w = 16; w >= 1; w >>= 1) lsum += __shfl_xor_sync(0xffffffffu, lsum, w);
+      for (int c = 0; c < 16; ++c) mx = fmaxf(mx, mc[c]);
+#pragma unroll
+      for (int n = 0; n < C::kMaxNew; ++n) mx = fmaxf(mx, sn[n]);
+      const float msub = mx == -INFINITY ? 0.f : mx;  // no key at all: every weight 0
+      float lsum = 0.f;
+#pragma unroll
+      for (int c = 0; c < 16; ++c) {
+        mc[c] = ex2(mc[c] - msub);  // ex2(-inf) = 0
+        lsum = fmaf(mc[c], lc[c], lsum);
+      }
+#pragma unroll
+      for (int n = 0; n < C::kMaxNew; ++n) {
+        sn[n] = ex2(sn[n] - msub);
+        lsum += sn[n];
+      }
       float2 acc = make_float2(0.f, 0.f);
 #pragma unroll
       for (int c = 0; c < 16; ++c) {
-        const float wc = __shfl_sync(0xffffffffu, f, c);
-        const float2 o = *reinterpret_cast<const float2*>(recv + ((c < csize ? c : 0) * rpc + rr) * kRowF + d);
-        const float wz = c < csize ? wc : 0.f;
-        acc.x = fmaf(wz, o.x, acc.x);
-        acc.y = fmaf(wz, o.y, acc.y);
+        if (c < csize) {
+          const float2 o = *reinterpret_cast<const float2*>(recv + ((c < csize ? c : 0) * rpc + rr) * kRowF + d);
+          acc.x = fmaf(mc[c], o.x, acc.x);
+          acc.y = fmaf(mc[c], o.y, acc.y);
+        }
       }
-      if (kFused) {
 #pragma unroll
-        for (int n = 0; n < kMaxNew; ++n) {
-          const float wn = __shfl_sync(0xffffffffu, f, min(csize + n, 31));
+      for (int n = 0; n < C::kMaxNew; ++n) {
+        if (n < n_new) {
           const uint32_t v2 = *reinterpret_cast<const uint32_t*>(smem + C::kOffNewV + n * kNewRow + d * 2);
-          const float wz = n < n_new ? wn : 0.f;
-          acc.x = fmaf(wz, sd_bf16_lo(v2), acc.x);
-          acc.y = fmaf(wz, sd_bf16_hi(v2), acc.y);
+          acc.x = fmaf(sn[n], sd_bf16_lo(v2), acc.x);
+          acc.y = fmaf(sn[n], sd_bf16_hi(v2), acc.y);
         }
       }
       if (valid && p < a.M && lsum > 0.f) {
@@ -972,18 +1009,25 @@ __global__ void __launch_bounds__(kThreads, 1)
                                             (p - gdiv(p) * a.G)) * kD + c * 8) = v;
         }
       }
-      if (rank == csize - 1 && mblock == 0) {
+      const bool append = rank == csize - 1 && mblock == 0;
+      // the head's last reader of the raw key rows (32 rows: one m-block, one cluster)
+      bool write_k = append;
+      if constexpr (kR == 64) write_k = *s_kvlast != 0;
+      if (append || write_k) {
 #pragma unroll 1
         for (int idx = st; idx < a.R * 16; idx += kSoftThreads) {
           const int i = idx / 16, c = idx % 16;
           const long long src = ((static_cast<long long>(b) * a.R + i) * a.Hkv + kvh) * kD + c * 8;
           const long long dst = ((static_cast<long long>(b) * a.Hkv + kvh) * a.cap + L_pre + i) * kD + c * 8;
           const uint4 kr = *reinterpret_cast<const uint4*>(smem + C::kOffNewK + i * kNewRow + c * 16);
-          *reinterpret_cast<uint4*>(a.kc + dst) = kr;
-          *reinterpret_cast<uint4*>(a.k_new + src) = kr;
-          *reinterpret_cast<uint4*>(a.vc + dst) =
-              *reinterpret_cast<const uint4*>(smem + C::kOffNewV + i * kNewRow + c * 16);
+          if (append) {
+            *reinterpret_cast<uint4*>(a.kc + dst) = kr;
+            *reinterpret_cast<uint4*>(a.vc + dst) =
+                *reinterpret_cast<const uint4*>(smem + C::kOffNewV + i * kNewRow + c * 16);
+          }
+          if (write_k) *reinterpret_cast<uint4*>(a.k_new + src) = kr;
         }
+        if (kR == 64 && write_k && a.n_mblocks > 1 && st == 0) a.kv_ticket[b * a.Hkv + kvh] = 0;  // re-armed
       }
     }
   }
@@ -1144,7 +1188,7 @@ extern "C" sd_status sd_set_cluster_size(int cluster_size) {
   return SD_ERR_INVALID_ARG;
 }
 
-static TcPlan tc_plan(int B, int R, int Hq, int Hkv, int D, int cap) {
+static TcPlan tc_plan(int B, int R, int Hq, int Hkv, int D, int cap, int max_cs = 16) {
   TcPlan p;
   if (!tc_enabled() || D != kD || Hkv <= 0 || Hq % Hkv || R <= 0) return p;
   const int M = (Hq / Hkv) * R;
@@ -1154,10 +1198,14 @@ static TcPlan tc_plan(int B, int R, int Hq, int Hkv, int D, int cap) {
   p.rows = M <= 32 ? 32 : 64;
   p.mblocks = (M + p.rows - 1) / p.rows;
   const int* active = s->active[p.rows == 32 ? 0 : 1];
+  // sizes above max_cs are not used (the fused merge holds csize partials and
+  // R new keys in the lanes of one warp)
+  int capped[kNumClusterSizes];
+  for (int i = 0; i < kNumClusterSizes; ++i) capped[i] = kClusterSizes[i] <= max_cs ? active[i] : 0;
   const int forced = g_forced_cluster.load();
   for (int i = 0; i < kNumClusterSizes && forced > 0; ++i)
-    if (kClusterSizes[i] == forced && active[i] > 0) p.cs = forced;
-  if (p.cs == 0) p.cs = pick_cluster(active, static_cast<long long>(B) * Hkv * p.mblocks, cap);
+    if (kClusterSizes[i] == forced && capped[i] > 0) p.cs = forced;
+  if (p.cs == 0) p.cs = pick_cluster(capped, static_cast<long long>(B) * Hkv * p.mblocks, cap);
   return p;
 }
 
@@ -1233,9 +1281,12 @@ sd_status sd_internal_verify_layer_tc(void* q, void* k_new, const void* v_new, c
                                       cudaStream_t stream, bool* handled) {
   *handled = false;
   const int B = cache->batch, Hkv = cache->n_kv_heads;
-  if (R > kMaxNew) return SD_OK;  // the new rows are held in shared memory
-  const TcPlan plan = tc_plan(B, R, Hq, Hkv, cache->head_dim, cache->capacity);
+  // the new rows are held in shared memory (16 with the 32-row tile, 32 with
+  // the 64-row tile) and merged in the lanes of one warp with the partials
+  if (R > 32) return SD_OK;
+  const TcPlan plan = tc_plan(B, R, Hq, Hkv, cache->head_dim, cache->capacity, 32 - R);
   if (plan.cs <= 0) return SD_OK;
+  if (R > (plan.rows == 32 ? Cfg<32>::kMaxNew : Cfg<64>::kMaxNew)) return SD_OK;
   TcArgs a = {};
   a.q = static_cast<const __nv_bfloat16*>(q);
   a.out = static_cast<__nv_bfloat16*>(out);
@@ -1247,6 +1298,7 @@ sd_status sd_internal_verify_layer_tc(void* q, void* k_new, const void* v_new, c
   a.vc = static_cast<__nv_bfloat16*>(cache->v);
   a.pos = pos;
   a.ticket = ticket;
+  a.kv_ticket = ticket + B;
   a.early = early ? 1 : 0;
   a.R = R;
   a.Hq = Hq;

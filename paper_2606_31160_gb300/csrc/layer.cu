@@ -13,13 +13,18 @@
 #include <math.h>
 
 namespace {
-constexpr size_t kTicketBytes(int B) { return (static_cast<size_t>(B) * 4 + 255) / 256 * 256; }
+// per-scene tickets [B], then per-(scene, KV head) tickets [B][Hkv] (the
+// tcgen05 kernel's read-before-write-back count when a head spans several
+// clusters)
+constexpr size_t kTicketBytes(int B, int Hkv) {
+  return (static_cast<size_t>(B) * (1 + static_cast<size_t>(Hkv)) * 4 + 255) / 256 * 256;
+}
 }  // namespace
 
 extern "C" size_t sd_verify_layer_workspace(int B, int R, int Hq, int Hkv, int D, int capacity) {
   if (B <= 0) return 0;
   const size_t attn = sd_verify_attention_workspace(B, R, Hq, Hkv, D, capacity);
-  return kTicketBytes(B) + attn;
+  return kTicketBytes(B, Hkv) + attn;
 }
 
 extern "C" sd_status sd_verify_layer(void* q, void* k_new, const void* v_new, const int32_t* pos,
@@ -58,6 +63,6 @@ extern "C" sd_status sd_verify_layer(void* q, void* k_new, const void* v_new, co
   if (r != SD_OK) return r;
   r = sd_kv_append(cache, k_new, v_new, R, stream);
   if (r != SD_OK) return r;
-  return sd_verify_attention(q, cache, out, R, Hq, scale, static_cast<char*>(workspace) + kTicketBytes(B),
-                             ws_bytes - kTicketBytes(B), stream);
+  return sd_verify_attention(q, cache, out, R, Hq, scale, static_cast<char*>(workspace) + kTicketBytes(B, Hkv),
+                             ws_bytes - kTicketBytes(B, Hkv), stream);
 }

@@ -102,3 +102,26 @@ def test_fused_overflow_sets_error_and_leaves_scene():
     assert sd.get_device_error() & sd.SD_DEVERR_KV_OVERFLOW
     assert cache.len.item() == case.cap - 3
     assert torch.all(out == 5.0)
+
+
+@pytest.mark.parametrize("K", [15, 16, 23])
+def test_fused_layer_long_drafts(K):
+    # block-diffusion drafts propose K = 16 tokens at once: R = K + 1 new rows
+    # (68 packed rows for K = 16: two 64-row m-blocks) in one fused call
+    R = K + 1
+    prefix = [4096, 1500]
+    qpos = np.stack([workloads.text_positions(int(p) + 1, R) for p in prefix])
+    case = workloads.verify_case(workloads.TARGET_LAYER, B=2, Hq=32, Hkv=8, D=128, prefix=prefix, K=K,
+                                 sections=(16, 24, 24), base=1e6, query_pos=qpos, cap=max(prefix) + R + 8,
+                                 layer=300 + K, tail_fill=float("nan"))
+    qa, ka, ca, oa = _unfused(case)
+    qb, kb, cb, ob = _fused(case)
+
+    def same(x, y):  # stale cache rows hold NaN on both sides
+        return bool(((x == y) | (x.isnan() & y.isnan())).all())
+
+    assert torch.equal(qa, qb) and torch.equal(ka, kb)
+    assert same(ca.k, cb.k) and same(ca.v, cb.v) and torch.equal(ca.len, cb.len)
+    _check_against_oracle(case, qb, cb, ob)
+    assert (ob.float() - oa.float()).abs().max().item() <= 2 * ATTN_ATOL
+    assert sd.get_device_error() == 0
