@@ -15,18 +15,24 @@ Readings taken where the paper is silent:
   * Softmax scale 1/sqrt(D) unless the caller gives one.
   * Grouped-query attention with contiguous groups: q head h reads KV head
     floor(h / G), G = Hq / Hkv.
+  * Block mask (block=True): the variant of the block-diffusion drafts
+    (Sec. 4, "Targets and drafts": a block of K = 16 tokens proposed at
+    once), where every new row also sees the new rows after it: row i sees
+    keys 0 .. L_b + R - 1.
 
 Parity: pinned (tests/test_oracle_attention.py) against torch's float64
 scaled_dot_product_attention with an explicitly built causal mask, and by the
 special cases one key -> v, identical keys -> mean of V, R = 1 -> plain
-decode, and the per-scene independence of a ragged batch.
+decode, and the per-scene independence of a ragged batch; the block mask
+against scaled_dot_product_attention without a mask.
 """
 
 import numpy as np
 
 
-def verify_attention(q, k_cache, v_cache, lens, scale=None):
-    """o[b, i, h] = softmax_n(q[b, i, h] . k[b, g, n] * scale) v[b, g, n], n <= L_b + i.
+def verify_attention(q, k_cache, v_cache, lens, scale=None, block=False):
+    """o[b, i, h] = softmax_n(q[b, i, h] . k[b, g, n] * scale) v[b, g, n], n <= L_b + i
+    (n < L_b + R with block=True).
 
     q:        [B, R, Hq, D]        float64 (rotated query rows)
     k_cache:  [B, Hkv, cap, D]     float64
@@ -53,7 +59,7 @@ def verify_attention(q, k_cache, v_cache, lens, scale=None):
         # visible[i, n]: row i (position prefix + i) sees key n <= prefix + i
         rows = np.arange(r_n)[:, None]
         keys = np.arange(n_keys)[None, :]
-        visible = keys <= prefix + rows
+        visible = keys <= prefix + rows if not block else np.ones((r_n, n_keys), dtype=bool)
         for h in range(hq):
             g = h // group
             k = k_cache[b, g, :n_keys]

@@ -115,3 +115,23 @@ def test_explicit_scale_is_used():
     a = oracle.verify_attention(q, k, v, lens, scale=0.5)
     b = oracle.verify_attention(q * (0.5 * 4.0), k, v, lens)   # default 1/sqrt(16) = 1/4
     np.testing.assert_allclose(a, b, rtol=0, atol=1e-13)
+
+
+def test_block_mask_is_unmasked_attention_over_all_rows():
+    # the block mask: every new row sees the prefix and all R new rows
+    rng = np.random.default_rng(21)
+    q, k, v, lens = _random_case(rng, 2, 6, 4, 2, 16, [13, 0], 24)
+    out = oracle.verify_attention(q, k, v, lens, block=True)
+    B, R, Hq, D = q.shape
+    G = Hq // k.shape[1]
+    for b in range(B):
+        n = int(lens[b])
+        qt = torch.from_numpy(q[b]).permute(1, 0, 2)
+        kt = torch.from_numpy(k[b, :, :n]).repeat_interleave(G, dim=0)
+        vt = torch.from_numpy(v[b, :, :n]).repeat_interleave(G, dim=0)
+        ref = torch.nn.functional.scaled_dot_product_attention(qt, kt, vt).permute(1, 0, 2).numpy()
+        assert np.allclose(out[b], ref, atol=1e-12)
+    # the last row sees the same keys under both masks
+    causal = oracle.verify_attention(q, k, v, lens)
+    assert np.allclose(out[:, -1], causal[:, -1], atol=1e-12)
+    assert not np.allclose(out[:, 0], causal[:, 0])
