@@ -166,6 +166,21 @@ sd_status sd_verify_attention(const void* q, const sd_kv_cache* cache, void* out
                               int R, int Hq, float scale, void* workspace, size_t ws_bytes,
                               sd_stream_t stream);
 
+/* sd_verify_attention_ex flag: the block mask. */
+#define SD_ATTN_BLOCK_MASK 1
+
+/*
+ * sd_verify_attention with flags. SD_ATTN_BLOCK_MASK selects the block mask of
+ * the block-diffusion drafts (Sec. 4 "Targets and drafts": a block of K = 16
+ * tokens proposed at once): every new row sees the prefix and all R new rows,
+ * n = 0 .. len[b] - 1, instead of n <= len[b] - R + i. Other bits:
+ * SD_ERR_INVALID_ARG. Everything else as sd_verify_attention (which is this
+ * call with flags 0).
+ */
+sd_status sd_verify_attention_ex(const void* q, const sd_kv_cache* cache, void* out,
+                                 int R, int Hq, float scale, int flags, void* workspace,
+                                 size_t ws_bytes, sd_stream_t stream);
+
 /*
  * Cluster size of the tcgen05 verify-attention kernel (sd_verify_attention
  * and sd_verify_layer, head_dim 128, G*R <= 128): one thread-block cluster of
@@ -204,8 +219,9 @@ sd_status sd_attention_budget(const void* q, const sd_kv_cache* cache, int R, in
                               const int32_t* n_visual, float* mass, float* entropy,
                               sd_stream_t stream);
 
-/* sd_verify_layer flag: see below. */
+/* sd_verify_layer flags: see below. */
 #define SD_LAYER_PREFIX_EARLY 1
+#define SD_LAYER_BLOCK_MASK 2
 
 /*
  * Workspace bytes sd_verify_layer needs on the CURRENT device for this shape.
@@ -235,6 +251,8 @@ size_t sd_verify_layer_workspace(int B, int R, int Hq, int Hkv, int D, int capac
  *   pass). The call is then a programmatic dependent launch that reads len and
  *   pos and streams the cached prefix while its predecessor still runs; q,
  *   k_new and v_new are read only after the predecessor has completed.
+ *   SD_LAYER_BLOCK_MASK: the attention uses the block mask (as
+ *   SD_ATTN_BLOCK_MASK of sd_verify_attention_ex).
  * For head_dim 128, G * R <= 128 and R <= 16 this is one tcgen05 kernel;
  * other shapes run the three kernels in sequence. A scene whose append would pass the
  * capacity sets SD_DEVERR_KV_OVERFLOW and is left untouched.

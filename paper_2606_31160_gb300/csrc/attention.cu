@@ -184,6 +184,7 @@ struct AttnArgs {
   float* part;    // [units][n_sp][kPartFloats] split partials (n_sp > 1)
   uint32_t* cnt;  // [units][2] arrival / departure counters (n_sp > 1)
   int R, Hq, Hkv, G, M, cap, n_sp;
+  int block;         // block mask: every new row sees all R new rows
   float scale_log2;  // softmax scale * log2(e)
 };
 
@@ -296,7 +297,7 @@ __global__ void __launch_bounds__(Cfg<D, MT, NMG>::kThreads, 1)
 #pragma unroll
       for (int hh = 0; hh < 2; ++hh) {
         const int p = mblock * C::kRows + mg * C::kRowsW + mt * 16 + g8 + 8 * hh;
-        lim[mt][hh] = min(L_prefix + p / a.G, n_keys - 1);
+        lim[mt][hh] = a.block ? n_keys - 1 : min(L_prefix + p / a.G, n_keys - 1);
       }
 
     float o[MT][D / 8][4];
@@ -790,7 +791,15 @@ extern "C" size_t sd_verify_attention_workspace(int B, int R, int Hq, int Hkv, i
 extern "C" sd_status sd_verify_attention(const void* q, const sd_kv_cache* cache, void* out,
                                          int R, int Hq, float scale, void* workspace,
                                          size_t ws_bytes, sd_stream_t stream) {
+  return sd_verify_attention_ex(q, cache, out, R, Hq, scale, 0, workspace, ws_bytes, stream);
+}
+
+extern "C" sd_status sd_verify_attention_ex(const void* q, const sd_kv_cache* cache, void* out,
+                                            int R, int Hq, float scale, int flags, void* workspace,
+                                            size_t ws_bytes, sd_stream_t stream) {
   if (!cache) return SD_ERR_INVALID_ARG;
+  if (flags & ~SD_ATTN_BLOCK_MASK) return SD_ERR_INVALID_ARG;
+  const int block = (flags & SD_ATTN_BLOCK_MASK) ? 1 : 0;
   const int B = cache->batch, Hkv = cache->n_kv_heads, cap = cache->capacity, D = cache->head_dim;
   const sd_status shape = check_shape(B, R, Hq, Hkv, D, cap);
   if (shape != SD_OK) return shape;
@@ -804,7 +813,7 @@ extern "C" sd_status sd_verify_attention(const void* q, const sd_kv_cache* cache
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   {
     bool handled = false;
-    const sd_status s = sd_internal_verify_attention_tc(q, cache, out, R, Hq, scale_log2, st, &handled);
+    const sd_status s = sd_internal_verify_attention_tc(q, cache, out, R, Hq, scale_log2, block, st, &handled);
     if (handled) return s;
   }
   Plan p;
@@ -827,6 +836,7 @@ extern "C" sd_status sd_verify_attention(const void* q, const sd_kv_cache* cache
   a.M = a.G * R;
   a.cap = cap;
   a.n_sp = 1;
+  a.block = block;
   a.scale_log2 = scale_log2;
   return D == 64 ? run_rows<64>(tk, tv, a, B, p, workspace, st)
                  : run_rows<128>(tk, tv, a, B, p, workspace, st);

@@ -300,7 +300,9 @@ struct TcArgs {
   const int32_t* pos;       // [B][R][3]
   uint32_t* ticket;         // [B] per-scene CTA tickets (zeroed, re-armed)
   uint32_t* kv_ticket;      // [B][Hkv] read-before-write-back tickets (several m-blocks)
-  int early;                // prefix, len and pos may be read before the dependency wait
+  // fused kernel: prefix, len and pos may be read before the dependency wait;
+  // standalone kernel: the block mask (every new row sees all R new rows)
+  int early;
   int R, Hq, Hkv, G, M, cap, n_mblocks;
   float inv_g;              // 1 / G: p / G == int((p + 0.5) / G) exactly for the p < 128 used here
   float scale_log2;
@@ -637,7 +639,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       // causal limit of each packed row: row p = i * G + g is new row i and
       // sees keys 0 .. L_prefix + i (Eq. verify's mask)
-      if (!kFused && st < kR) row_lim[st] = min(n_keys - a.R + gdiv(mblock * kR + st), n_keys - 1);
+      if (!kFused && st < kR)
+        row_lim[st] = a.early ? n_keys - 1 : min(n_keys - a.R + gdiv(mblock * kR + st), n_keys - 1);
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
       named_bar_sync(2, kSoftThreads);  // Q is complete; the rotation table is no longer read
       if (st == 0) {
@@ -1250,7 +1253,7 @@ static sd_status launch_plan(const sd_kv_cache* cache, const TcArgs& a, const Ro
 
 // Routed here by sd_verify_attention for head_dim 128 and G * R <= 128.
 sd_status sd_internal_verify_attention_tc(const void* q, const sd_kv_cache* cache, void* out,
-                                          int R, int Hq, float scale_log2, cudaStream_t stream,
+                                          int R, int Hq, float scale_log2, int block, cudaStream_t stream,
                                           bool* handled) {
   *handled = false;
   const int B = cache->batch, Hkv = cache->n_kv_heads;
@@ -1268,6 +1271,7 @@ sd_status sd_internal_verify_attention_tc(const void* q, const sd_kv_cache* cach
   a.inv_g = 1.0f / static_cast<float>(a.G);
   a.cap = cache->capacity;
   a.n_mblocks = plan.mblocks;
+  a.early = block;  // the standalone kernel's block mask
   a.scale_log2 = scale_log2;
   RopeTable tab = {};
   *handled = true;
@@ -1278,9 +1282,12 @@ sd_status sd_internal_verify_attention_tc(const void* q, const sd_kv_cache* cach
 sd_status sd_internal_verify_layer_tc(void* q, void* k_new, const void* v_new, const int32_t* pos,
                                       const RopeTable& tab, const sd_kv_cache* cache, void* out,
                                       int R, int Hq, float scale_log2, uint32_t* ticket, int early,
-                                      cudaStream_t stream, bool* handled) {
+                                      int block, cudaStream_t stream, bool* handled) {
   *handled = false;
   const int B = cache->batch, Hkv = cache->n_kv_heads;
+  // the block mask (a draft's pattern, not the target's verify) takes the
+  // three separate kernels: the fused kernel's new-key merge stays causal
+  if (block) return SD_OK;
   // the new rows are held in shared memory (16 with the 32-row tile, 32 with
   // the 64-row tile) and merged in the lanes of one warp with the partials
   if (R > 32) return SD_OK;

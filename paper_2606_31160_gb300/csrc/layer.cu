@@ -37,7 +37,8 @@ extern "C" sd_status sd_verify_layer(void* q, void* k_new, const void* v_new, co
   if (B < 0 || R <= 0 || Hq <= 0 || Hkv <= 0 || cap <= 0 || Hq % Hkv) return SD_ERR_INVALID_ARG;
   if (D != 64 && D != 128) return SD_ERR_UNSUPPORTED;
   if (interleaved != 0 && interleaved != 1) return SD_ERR_INVALID_ARG;
-  if (flags & ~SD_LAYER_PREFIX_EARLY) return SD_ERR_INVALID_ARG;
+  if (flags & ~(SD_LAYER_PREFIX_EARLY | SD_LAYER_BLOCK_MASK)) return SD_ERR_INVALID_ARG;
+  const int block = (flags & SD_LAYER_BLOCK_MASK) ? 1 : 0;
   if (B == 0) return SD_OK;
   if (!q || !k_new || !v_new || !pos || !sections || !out || !cache->k || !cache->v || !cache->len)
     return SD_ERR_INVALID_ARG;
@@ -56,13 +57,14 @@ extern "C" sd_status sd_verify_layer(void* q, void* k_new, const void* v_new, co
   bool handled = false;
   const sd_status s = sd_internal_verify_layer_tc(q, k_new, v_new, pos, tab, cache, out, R, Hq,
                                                   scale_log2, ticket, flags & SD_LAYER_PREFIX_EARLY,
-                                                  st, &handled);
+                                                  block, st, &handled);
   if (handled) return s;
   // other shapes: the same three steps as separate kernels
   sd_status r = sd_rope_apply(q, k_new, B, R, Hq, Hkv, D, pos, sections, interleaved, base, stream);
   if (r != SD_OK) return r;
   r = sd_kv_append(cache, k_new, v_new, R, stream);
   if (r != SD_OK) return r;
-  return sd_verify_attention(q, cache, out, R, Hq, scale, static_cast<char*>(workspace) + kTicketBytes(B, Hkv),
-                             ws_bytes - kTicketBytes(B, Hkv), stream);
+  return sd_verify_attention_ex(q, cache, out, R, Hq, scale, block ? SD_ATTN_BLOCK_MASK : 0,
+                                static_cast<char*>(workspace) + kTicketBytes(B, Hkv),
+                                ws_bytes - kTicketBytes(B, Hkv), stream);
 }

@@ -49,6 +49,7 @@ _SIGNATURES = {
     "sd_kv_rollback": ([_vp, _i, _i, _vp, _i, _vp], _i),
     "sd_verify_attention_workspace": ([_i, _i, _i, _i, _i, _i], _sz),
     "sd_verify_attention": ([_vp, ctypes.POINTER(KVCacheStruct), _vp, _i, _i, _f, _vp, _sz, _vp], _i),
+    "sd_verify_attention_ex": ([_vp, ctypes.POINTER(KVCacheStruct), _vp, _i, _i, _f, _i, _vp, _sz, _vp], _i),
     "sd_verify_layer_workspace": ([_i, _i, _i, _i, _i, _i], _sz),
     "sd_verify_layer": ([_vp, _vp, _vp, _vp, ctypes.POINTER(ctypes.c_int32), _i, _f,
                          ctypes.POINTER(KVCacheStruct), _vp, _i, _i, _f, _vp, _sz, _i, _vp], _i),
@@ -206,7 +207,11 @@ def attention_workspace_bytes(B, R, Hq, Hkv, D, capacity):
 _attn_ws = {}
 
 
-def verify_attention(q, cache, out=None, scale=0.0, ws=None):
+SD_ATTN_BLOCK_MASK = 1
+SD_LAYER_BLOCK_MASK = 2
+
+
+def verify_attention(q, cache, out=None, scale=0.0, ws=None, block=False):
     """Causal GQA verify attention of q [B,R,Hq,D] (rotated) over the cache (appended).
     ws: the split-merge workspace (see sd_verify_attention_workspace); when None a
     zero-filled one is kept per (device, shape) and reused by later calls."""
@@ -223,9 +228,10 @@ def verify_attention(q, cache, out=None, scale=0.0, ws=None):
         ws = _attn_ws.get(key)
     wp = _dev(ws, "ws") if ws is not None else ctypes.c_void_p(0)
     nbytes = ws.numel() * ws.element_size() if ws is not None else 0
-    _check(lib().sd_verify_attention(_dev(q, "q", torch.bfloat16), cache.struct,
-                                     _dev(out, "out", torch.bfloat16), R, Hq, float(scale), wp, nbytes,
-                                     _stream()), "sd_verify_attention")
+    _check(lib().sd_verify_attention_ex(_dev(q, "q", torch.bfloat16), cache.struct,
+                                        _dev(out, "out", torch.bfloat16), R, Hq, float(scale),
+                                        SD_ATTN_BLOCK_MASK if block else 0, wp, nbytes, _stream()),
+           "sd_verify_attention")
     return out
 
 
@@ -254,11 +260,11 @@ def layer_workspace_bytes(B, R, Hq, Hkv, D, capacity):
 
 
 def verify_layer(q, k_new, v_new, pos, sections, cache, interleaved=0, base=1e6, out=None, scale=0.0,
-                 ws=None, early=False):
+                 ws=None, early=False, block=False):
     """sd_verify_layer: M-RoPE of q / k_new (in place), append of k_new / v_new at
     len[b] (the prefix length on entry; len += R) and the verify attention; returns out.
     early=True sets SD_LAYER_PREFIX_EARLY (the previous kernel on the stream writes
-    neither this layer's cache nor its len)."""
+    neither this layer's cache nor its len); block=True sets SD_LAYER_BLOCK_MASK."""
     B, R, Hq, D = q.shape
     Hkv = k_new.shape[2]
     if tuple(k_new.shape) != (B, R, Hkv, D) or k_new.shape != v_new.shape or tuple(pos.shape) != (B, R, 3):
@@ -280,7 +286,8 @@ def verify_layer(q, k_new, v_new, pos, sections, cache, interleaved=0, base=1e6,
                                  _dev(v_new, "v_new", torch.bfloat16), _dev(pos, "pos", torch.int32), sec,
                                  int(interleaved), float(base), cache.struct, _dev(out, "out", torch.bfloat16),
                                  R, Hq, float(scale), _dev(ws, "ws"), ws.numel() * ws.element_size(),
-                                 SD_LAYER_PREFIX_EARLY if early else 0, _stream()), "sd_verify_layer")
+                                 (SD_LAYER_PREFIX_EARLY if early else 0) | (SD_LAYER_BLOCK_MASK if block else 0),
+                                 _stream()), "sd_verify_layer")
     return out
 
 

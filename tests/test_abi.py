@@ -96,3 +96,13 @@ def test_cluster_size_override_is_host_only(lib):
     for cs in (-1, 3, 5, 7, 12, 32):
         assert lib.sd_set_cluster_size(cs) == 1
     assert lib.sd_set_cluster_size(0) == 0
+
+
+def test_unknown_mask_flags_are_rejected_before_launch(lib):
+    null = ctypes.c_void_p(0)
+    cache = sd.KVCacheStruct(16, 16, 16, 1, 8, 64, 128)
+    assert lib.sd_verify_attention_ex(ctypes.c_void_p(16), ctypes.byref(cache), ctypes.c_void_p(16), 8, 32, 0.0,
+                                      4, null, 0, null) == 1
+    assert lib.sd_verify_layer(ctypes.c_void_p(16), ctypes.c_void_p(16), ctypes.c_void_p(16), ctypes.c_void_p(16),
+                               (ctypes.c_int32 * 3)(16, 24, 24), 0, 1e6, ctypes.byref(cache), ctypes.c_void_p(16),
+                               8, 32, 0.0, null, 0, 4, null) == 1
