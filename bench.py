@@ -437,6 +437,61 @@ def time_stochastic_step(device, layers=LAYERS):
     return ms * 1e3, layers * layer_bytes(B_) + logits  # the same accounting as the main step
 
 
+def time_long_draft_step(device, K_=16, layers=LAYERS):
+    """The verify step of a block-diffusion draft (Sec. 4: blocks of K = 16
+    tokens): 36 fused target layers at B = 1, L = 4096, R = 17 (68 packed rows
+    per KV head: two 64-row m-blocks), one cache per layer, then the greedy
+    accept over bf16 logits [1][17][151936] and the rollback, in a graph.
+    Returns (us per step, algorithmic bytes per step)."""
+    from paper_2606_31160_gb300 import sd, workloads
+    R_ = K_ + 1
+    gen = torch.Generator(device=device)
+    gen.manual_seed(6000)
+    cap = L + R_
+
+    def normal(*shape):
+        return torch.randn(shape, generator=gen, device=device, dtype=torch.float32).to(torch.bfloat16)
+
+    lens = torch.full((layers, 1), L, dtype=torch.int32, device=device)
+    lens0 = lens.clone()
+    caches, qs, ks, vs, outs, wss = [], [], [], [], [], []
+    for l in range(layers):
+        kc = torch.zeros((1, HKV, cap, D), dtype=torch.bfloat16, device=device)
+        vc = torch.zeros_like(kc)
+        kc[:, :, :L] = normal(1, HKV, L, D)
+        vc[:, :, :L] = normal(1, HKV, L, D)
+        caches.append(sd.KVCache(kc, vc, lens[l]))
+        qs.append(normal(1, R_, HQ, D))
+        ks.append(normal(1, R_, HKV, D))
+        vs.append(normal(1, R_, HKV, D))
+        outs.append(torch.empty_like(qs[-1]))
+        wss.append(sd.workspace(sd.layer_workspace_bytes(1, R_, HQ, HKV, D, cap), device))
+    qpos = torch.from_numpy(workloads.text_positions(544, R_)[None]).to(device)
+    logits = normal(1, R_, V)
+    draft = torch.randint(0, V, (1, K_), generator=gen, device=device, dtype=torch.int32)
+    ws_g = sd.workspace(sd.greedy_workspace_bytes(1, K_, V), device)
+    n_emit = torch.zeros(1, dtype=torch.int32, device=device)
+    tokens = torch.zeros((1, R_), dtype=torch.int32, device=device)
+    argmax = torch.zeros((1, R_), dtype=torch.int32, device=device)
+
+    def step():
+        for l in range(layers):
+            sd.verify_layer(qs[l], ks[l], vs[l], qpos, SECTIONS, caches[l], 0, BASE, out=outs[l], ws=wss[l],
+                            early=l > 0)
+        sd.accept_greedy(logits, draft, ws=ws_g, n_emit=n_emit, tokens=tokens, argmax=argmax)
+        sd.kv_rollback(lens, n_emit, R_)
+        lens.copy_(lens0, non_blocking=True)
+
+    g = capture(step)
+    ms = time_graph(g, 20)
+    assert sd.get_device_error() == 0
+    rows = 2 * R_ * (2 * HQ + 3 * HKV) * D  # q in / out, rotated q, new k / v rows, out (as layer_bytes)
+    nbytes = layers * (L * HKV * D * 2 * 2 + rows) + R_ * V * 2
+    del caches, qs, ks, vs, outs, wss
+    torch.cuda.empty_cache()
+    return ms * 1e3, nbytes
+
+
 def oracle_layer_sample(case, logits, draft):
     """The float64 oracle on one layer of the step plus the acceptance:
     returns bytes of the workload it covered (same accounting as the GPU)."""
@@ -587,6 +642,7 @@ def main():
     sample_us, sample_bytes = time_sample_accept(device) if rank == 0 else (None, None)
     draft_us = time_draft_steps(device) if rank == 0 else None
     stoch_us, stoch_bytes = time_stochastic_step(device) if rank == 0 else (None, None)
+    long_us, long_bytes = time_long_draft_step(device) if rank == 0 else (None, None)
     assert sd.get_device_error() == 0
 
     if rank != 0:
@@ -634,6 +690,8 @@ def main():
         "draft_step_us": round(draft_us, 3),
         "stochastic_step_us": round(stoch_us, 2),
         "stochastic_step_gbs": round(stoch_bytes / (stoch_us * 1e-6) / 1e9, 1),
+        "block_draft_step_us": round(long_us, 2),
+        "block_draft_step_gbs": round(long_bytes / (long_us * 1e-6) / 1e9, 1),
         "bytes_per_step": step_bytes(1),
         "roofline": {
             "kernel": "sd_verify_layer -> verify_attn_tc_kernel<fused> (M-RoPE + append + attention, tcgen05)",
