@@ -166,6 +166,12 @@ __device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap* map
       "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(x), "r"(y), "r"(z)
       : "memory");
 }
+__device__ __forceinline__ void tma_prefetch_3d(const CUtensorMap* map, int x, int y, int z) {
+  asm volatile("cp.async.bulk.prefetch.tensor.3d.L2.global.tile [%0, {%1, %2, %3}];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(x), "r"(y), "r"(z)
+               : "memory");
+}
 __device__ __forceinline__ float ex2(float x) {
   float y;
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
@@ -451,6 +457,19 @@ __global__ void __launch_bounds__(kThreads, 1)
       asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_k128)) : "memory");
       asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_v128)) : "memory");
       const int z = b * a.Hkv + kvh;
+      // chained layers: the cluster launched last (the last KV head of the
+      // last scene) starts only when the previous layer frees its SMs; the
+      // first head's CTAs bring that head's tiles of their own key range
+      // into L2 meanwhile
+      if (kFused && a.early && kvh == 0 && b == static_cast<int>(gridDim.z) - 1 && a.Hkv > 1) {
+        const int zl = b * a.Hkv + a.Hkv - 1;
+        for (int t = 0; t < n_tiles; ++t)
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            tma_prefetch_3d(&tm_k128, h * 64, key_begin + t * kStageKeys, zl);
+            tma_prefetch_3d(&tm_v128, h * 64, key_begin + t * kStageKeys, zl);
+          }
+      }
       for (int pass = 0; pass < 2; ++pass) {
         if (pass == 1) {
           // every MMA of pass 0 is done when the decision is out
