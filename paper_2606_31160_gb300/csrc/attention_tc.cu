@@ -66,7 +66,8 @@ constexpr int kKV = 2 * kHalf;              // one K (or V) tile of 128 keys (32
 constexpr int kNewRow = kD * 2;             // one new key / value row (256 B)
 constexpr int kSoftWarps = 8;
 constexpr int kSoftThreads = 32 * kSoftWarps;
-constexpr int kThreads = 64 + kSoftThreads;
+constexpr int kPvWarp = 2 + kSoftWarps;        // the warp after the softmax warps issues PV
+constexpr int kThreads = 96 + kSoftThreads;
 constexpr uint32_t kSpinLimit = 1u << 20;
 constexpr float kSlack = 64.f;              // log2 units a score may exceed its reference by
 // a merged partial row is [O(128) | m | l | 2 pad] fp32 = 528 bytes
@@ -170,6 +171,10 @@ __device__ __forceinline__ void tma_prefetch_3d(const CUtensorMap* map, int x, i
   asm volatile("cp.async.bulk.prefetch.tensor.3d.L2.global.tile [%0, {%1, %2, %3}];" ::"l"(
                    reinterpret_cast<uint64_t>(map)),
                "r"(x), "r"(y), "r"(z)
+               : "memory");
+}
+__device__ __forceinline__ void bulk_prefetch_l2(const void* p, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(reinterpret_cast<uint64_t>(p)), "r"(bytes)
                : "memory");
 }
 __device__ __forceinline__ float ex2(float x) {
@@ -293,6 +298,36 @@ __device__ __forceinline__ void rows_reduce(const float (&v)[kN], int kl, int ro
   asm volatile("bar.sync 2, 256;" ::: "memory");
 }
 
+// Second pass (fixed references exceeded): row r's reference moves to
+// ref + max over the range of (score - ref); buf holds every thread's 16 or 32
+// per-row maxima at [row][key lane]. Out of line: it runs only when a score
+// exceeded its reference by more than the slack.
+template <int kN>
+__device__ __noinline__ void redo_references(int kl, int row0, int st, int quarter, int lane, float* buf,
+                                             float* row_a, float* row_ref) {
+  constexpr int kRowsAll = 2 * kN;
+  constexpr int kPer = kSoftThreads / kRowsAll;
+  constexpr int kVals = 128 / kPer;
+  asm volatile("bar.sync 2, 256;" ::: "memory");
+  const int r = st / kPer, part = st % kPer;
+  const float4* src = reinterpret_cast<const float4*>(buf + r * 128) + part;
+  float acc = -INFINITY;
+#pragma unroll 1
+  for (int q = 0; q < kVals / 4; ++q) {
+    const float4 x = src[q * kPer];
+    acc = fmaxf(acc, fmaxf(fmaxf(x.x, x.y), fmaxf(x.z, x.w)));
+  }
+  for (int w = 1; w < kPer; w <<= 1) acc = fmaxf(acc, __shfl_xor_sync(0xffffffffu, acc, w));
+  if (part == 0) row_a[r] = acc;
+  asm volatile("bar.sync 2, 256;" ::: "memory");
+  if (quarter == 0 && lane < kN) {
+    const float e = row_a[row0 + lane];
+    const float m0 = row_ref[row0 + lane] == -INFINITY ? 0.f : row_ref[row0 + lane];
+    row_ref[row0 + lane] = e == -INFINITY ? -INFINITY : m0 + e;
+  }
+  asm volatile("bar.sync 2, 256;" ::: "memory");
+}
+
 struct TcArgs {
   const __nv_bfloat16* q;   // rotated q rows (standalone attention)
   __nv_bfloat16* out;
@@ -353,9 +388,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   // softmax's tile T + kS - 2 >= T; PV(T + kS) needs the V tile loaded after
   // the producer's wait for PVDONE(T), and the softmax waits for PVDONE only
   // once a pass, on its last tile.
-  // With 32 rows (3 slots) a tile's K and V arrive together on FULLK, loaded
-  // once PV(T - 3) is done; with 64 rows (2 slots) each has its own barrier.
-  constexpr bool kSplit = kR == 64;
+  // K and V of a tile have their own barriers: a K slot refills once its S
+  // product is done, a V slot once its PV product is.
+  constexpr bool kSplit = true;
   auto FULLK = [&](int s) { return bar(s); };
   auto FULLV = [&](int s) { return kSplit ? bar(kS + s) : bar(s); };
   auto PFULL = [&](int b) { return bar(2 * kS + b); };
@@ -421,6 +456,17 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
   }
+  if (kFused && threadIdx.x >= 64 && threadIdx.x < 64 + kSoftThreads) {
+    // rotation table of the R new positions: (cos, sin) per (row, pair),
+    // built while thread 0 takes the scene's length
+    float2* tabw = reinterpret_cast<float2*>(smem + C::kOffP);
+#pragma unroll 1
+    for (int idx = threadIdx.x - 64; idx < a.R * 64; idx += kSoftThreads) {
+      const int i = idx >> 6, d = idx & 63;
+      const int32_t pc = a.pos[(static_cast<long long>(blockIdx.z) * a.R + i) * 3 + tab.axis[d]];
+      tabw[idx] = sd_rope_cs(static_cast<float>(pc), d, tab);
+    }
+  }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -469,6 +515,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             tma_prefetch_3d(&tm_k128, h * 64, key_begin + t * kStageKeys, zl);
             tma_prefetch_3d(&tm_v128, h * 64, key_begin + t * kStageKeys, zl);
           }
+        // and that head's query and new key / value rows
+        if (rank == 0)
+          for (int i = 0; i < a.R; ++i) {
+            const long long row = static_cast<long long>(b) * a.R + i;
+            bulk_prefetch_l2(a.qw + (row * a.Hq + (a.Hkv - 1) * a.G) * kD, a.G * kD * 2);
+            bulk_prefetch_l2(a.k_new + (row * a.Hkv + a.Hkv - 1) * kD, kD * 2);
+            bulk_prefetch_l2(a.v_new + (row * a.Hkv + a.Hkv - 1) * kD, kD * 2);
+          }
       }
       for (int pass = 0; pass < 2; ++pass) {
         if (pass == 1) {
@@ -509,52 +563,64 @@ __global__ void __launch_bounds__(kThreads, 1)
     cluster_arrive();  // the cluster's rings are free (see the softmax branch)
     cluster_wait();
   } else if (warp == 1) {
-    // -------------------------------------------------------------- MMA issue
+    // -------------------------------------------------------------- S issue
+    // S(T) and PV(T) come from two threads (this one and the PV warp's), so
+    // that one batch is issued while the other executes.
     if (lane == 0 && n_tiles > 0) {
       mbar_wait(QFULL, 0);
       // base descriptors; a K step only moves the start address (low field, no carry)
-      const uint64_t dK0 = umma_desc(base, 16, 1024);                     // K tile: K-major
-      const uint64_t dV0 = umma_desc(base + C::kRingV, kHalf, 1024);      // V^T: MN-major
-      const uint64_t dQ = umma_desc(qs, 16, 1024);                        // Q: K-major
-      // P^T: MN-major, one swizzle atom wide (kR rows), 8-key groups 8 * kPRow apart
-      const uint64_t dP0 = umma_desc(base + C::kOffP, 0, 8 * C::kPRow, C::kPLayout);
-      // Two issue sites with every K-step offset a compile-time constant (one
-      // 64-bit add per descriptor): a rolled or shared issue loop measured
-      // ~1.8 us slower per layer.
+      const uint64_t dK0 = umma_desc(base, 16, 1024);  // K tile: K-major
+      const uint64_t dQ = umma_desc(qs, 16, 1024);     // Q: K-major
       for (int pass = 0; pass < 2; ++pass) {
         if (pass == 1) {
           mbar_wait(DECIDE, 0);
           if (!*reinterpret_cast<volatile int*>(s_redo)) break;
         }
         const int T0 = pass * n_tiles;
-        // S(0), S(1) first; then per tile PV(t) and S(t + 2)
-        for (int t = -2; t < n_tiles; ++t) {
-          if (t >= 0) {
-            const int T = T0 + t;
-            mbar_wait(PFULL(T & 1), (T >> 1) & 1);
-            if (kSplit) mbar_wait(FULLV(T % kS), ring_parity(T));  // else waited before S(T)
-            tc_fence_after();
-            const uint64_t dv = dV0 + static_cast<uint64_t>(((T % kS) * kKV) >> 4);
-            const uint64_t dp = dP0 + static_cast<uint64_t>(((T & 1) * C::kP) >> 4);
+        for (int t = 0; t < n_tiles; ++t) {
+          // S(T) reuses the S buffer of tile T - 2: the softmax has read it
+          // once PFULL(T - 2) is out (pass 1 starts after all of pass 0)
+          const int T = T0 + t, st_ = T % kS;
+          if (t >= 2) mbar_wait(PFULL(T & 1), ((T - 2) >> 1) & 1);
+          mbar_wait(FULLK(st_), ring_parity(T));
+          tc_fence_after();
+          const uint64_t dk = dK0 + static_cast<uint64_t>((st_ * kKV) >> 4);
+          const uint32_t ts = tmem_s + kR * (T & 1);
 #pragma unroll
-            for (int kk = 0; kk < 8; ++kk)
-              umma(tmem_o, dv + (kk * 2048 >> 4), dp + (kk * 16 * C::kPRow >> 4), kIdescO,
-                   (t > 0 || kk > 0) ? 1 : 0);
-            umma_commit(PVDONE(T));
-          }
-          if (t + 2 < n_tiles) {
-            // S(T) reuses the S buffer of tile T - 2, read before PFULL(T - 2)
-            const int T = T0 + t + 2, st_ = T % kS;
-            mbar_wait(FULLK(st_), ring_parity(T));
-            tc_fence_after();
-            const uint64_t dk = dK0 + static_cast<uint64_t>((st_ * kKV) >> 4);
-            const uint32_t ts = tmem_s + kR * (T & 1);
+          for (int kk = 0; kk < 8; ++kk)
+            umma(ts, dk + (((kk >> 2) * kHalf + (kk & 3) * 32) >> 4),
+                 dQ + (((kk >> 2) * C::kQHalf + (kk & 3) * 32) >> 4), kIdescS, kk > 0 ? 1 : 0);
+          umma_commit(SREADY(T));
+        }
+      }
+    }
+    __syncwarp();
+    cluster_arrive();
+    cluster_wait();
+  } else if (warp == kPvWarp) {
+    // -------------------------------------------------------------- PV issue
+    if (lane == 0 && n_tiles > 0) {
+      const uint64_t dV0 = umma_desc(base + C::kRingV, kHalf, 1024);  // V^T: MN-major
+      // P^T: MN-major, one swizzle atom wide (kR rows), 8-key groups 8 * kPRow apart
+      const uint64_t dP0 = umma_desc(base + C::kOffP, 0, 8 * C::kPRow, C::kPLayout);
+      for (int pass = 0; pass < 2; ++pass) {
+        if (pass == 1) {
+          mbar_wait(DECIDE, 0);
+          if (!*reinterpret_cast<volatile int*>(s_redo)) break;
+        }
+        const int T0 = pass * n_tiles;
+        for (int t = 0; t < n_tiles; ++t) {
+          const int T = T0 + t;
+          mbar_wait(PFULL(T & 1), (T >> 1) & 1);
+          mbar_wait(FULLV(T % kS), ring_parity(T));  // (FULLK when K and V share a barrier)
+          tc_fence_after();
+          const uint64_t dv = dV0 + static_cast<uint64_t>(((T % kS) * kKV) >> 4);
+          const uint64_t dp = dP0 + static_cast<uint64_t>(((T & 1) * C::kP) >> 4);
 #pragma unroll
-            for (int kk = 0; kk < 8; ++kk)
-              umma(ts, dk + (((kk >> 2) * kHalf + (kk & 3) * 32) >> 4),
-                   dQ + (((kk >> 2) * C::kQHalf + (kk & 3) * 32) >> 4), kIdescS, kk > 0 ? 1 : 0);
-            umma_commit(SREADY(T));
-          }
+          for (int kk = 0; kk < 8; ++kk)
+            umma(tmem_o, dv + (kk * 2048 >> 4), dp + (kk * 16 * C::kPRow >> 4), kIdescO,
+                 (t > 0 || kk > 0) ? 1 : 0);
+          umma_commit(PVDONE(T));
         }
       }
     }
@@ -570,17 +636,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t lane_off = static_cast<uint32_t>(quarter * 32) << 16;
     const int row0 = kRpt * half;          // first query row of this thread
     const float2* cs_tab = reinterpret_cast<const float2*>(smem + C::kOffP);  // [R][64] (cos, sin)
-    if (kFused && valid) {
-      // rotation table of the R new positions: (cos, sin) per (row, pair)
-      float2* tabw = reinterpret_cast<float2*>(smem + C::kOffP);
-#pragma unroll 1
-      for (int idx = st; idx < a.R * 64; idx += kSoftThreads) {
-        const int i = idx >> 6, d = idx & 63;
-        const int32_t pc = a.pos[(static_cast<long long>(b) * a.R + i) * 3 + tab.axis[d]];
-        tabw[idx] = sd_rope_cs(static_cast<float>(pc), d, tab);
-      }
-    }
-    if (kFused) named_bar_sync(2, kSoftThreads);  // the rotation table is complete
     {
       // the packed query tile: this thread's 16-byte chunks (row, chunk c),
       // rows past M zero; in the fused layer also one chunk of a new key and
@@ -613,8 +668,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       // rows hold: it brings this code into the instruction cache and the rows
       // into L2, and iteration 1 overwrites everything it stored. The loads
       // bypass L1 (.cg) so that iteration 1 cannot hit a line read before the wait.
+      // the cluster launched last starts when the previous kernel is done or
+      // nearly so: no warm-up pass, its rows are read once, after the wait
+      const bool last_cluster = blockIdx.y == gridDim.y - 1 && blockIdx.z == gridDim.z - 1;
 #pragma unroll 1
-      for (int it = kFused ? 0 : 1; it < 2; ++it) {
+      for (int it = (kFused && !(a.early && last_cluster)) ? 0 : 1; it < 2; ++it) {
         if (kFused && it == 1 && a.early) griddep_wait();  // the raw rows come from earlier kernels
         uint4 qv[kQc], kv[kKvc], vv[kKvc];
 #pragma unroll
@@ -748,12 +806,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int bb = T & 1, s = T % kS;
         const int key0 = key_begin + t * kStageKeys;
         const int key = key0 + kl;
-        mbar_wait(SREADY(T), ring_parity(T));  // S(T) is ready, and so PV(T - 2) is done
+        mbar_wait(SREADY(T), ring_parity(T));  // S(T) is ready
         tc_fence_after();
         const bool key_ok = key < key_end;
         // P^T key row kl (its buffer's previous tile, T - 2, is done: see
         // above): kRpt rows = kRpt / 8 16-byte chunks of 8 query rows, swizzled
         const uint32_t prow = base + C::kOffP + bb * C::kP + kl * C::kPRow;
+        if (T >= 2) mbar_wait(PVDONE(T - 2), ring_parity(T - 2));  // PV(T - 2) has read P buffer bb
         const int sw = kR == 32 ? (kl >> 1) & 3 : kl & 7;
 #pragma unroll
         for (int j0 = 0; j0 < kRpt; j0 += 16) {
@@ -827,22 +886,24 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (redo) {
           // second pass with the exact row maxima of the whole range (every
           // MMA is done: the P buffers are free)
-          rows_reduce<true>(ex, kl, row0, st, reinterpret_cast<float*>(smem + C::kOffP), row_a);
+          float* rb = reinterpret_cast<float*>(smem + C::kOffP);
 #pragma unroll
           for (int j = 0; j < kRpt; ++j) {
-            if (kRefRegs) {
-              const float e = row_a[row0 + j];
-              const float m0 = ref[j % (kRefRegs ? kRpt : 1)] == -INFINITY ? 0.f : ref[j % (kRefRegs ? kRpt : 1)];
-              ref[j % (kRefRegs ? kRpt : 1)] = e == -INFINITY ? -INFINITY : m0 + e;
-            }
+            rb[(row0 + j) * 128 + kl] = ex[j];
             lp[j] = 0.f;
           }
-          if (quarter == 0 && lane < kRpt) {
-            const float e = row_a[row0 + lane];
-            const float m0 = row_ref[row0 + lane] == -INFINITY ? 0.f : row_ref[row0 + lane];
-            row_ref[row0 + lane] = e == -INFINITY ? -INFINITY : m0 + e;
+          redo_references<kRpt>(kl, row0, st, quarter, lane, rb, row_a, row_ref);
+          if (kRefRegs) {
+            const float4* rr4 = reinterpret_cast<const float4*>(row_ref + row0);
+#pragma unroll
+            for (int j4 = 0; j4 < (kRefRegs ? kRpt / 4 : 0); ++j4) {
+              const float4 x = rr4[j4];
+              ref[(4 * j4 + 0) % (kRefRegs ? kRpt : 1)] = x.x;
+              ref[(4 * j4 + 1) % (kRefRegs ? kRpt : 1)] = x.y;
+              ref[(4 * j4 + 2) % (kRefRegs ? kRpt : 1)] = x.z;
+              ref[(4 * j4 + 3) % (kRefRegs ? kRpt : 1)] = x.w;
+            }
           }
-          if (!kRefRegs) named_bar_sync(2, kSoftThreads);  // row_ref is read by every thread
         }
       }
     }
@@ -951,59 +1012,48 @@ __global__ void __launch_bounds__(kThreads, 1)
       named_bar_sync(2, kSoftThreads);
     }
     // ---- merge of the rows this CTA owns; slot c * rpc + rr came from rank c.
-    // A thread takes one row and two adjacent d: it forms the row's weights
-    // itself (partials c < csize and new keys n < R, all loads issued
-    // together), then its two outputs.
+    // A warp takes one row (kD / 2 = 64 items a row, so a row is two whole
+    // warps) and a thread two adjacent d. Lane c forms the weight of partial c
+    // (c < csize) and of new key c (c < R) once for the warp; the weights are
+    // broadcast by shuffles to the FMAs of every lane.
     mbar_wait(RECV, 0);
     const float* recv = reinterpret_cast<const float*>(smem + C::kRecv);
     const int n_new = (kFused && valid) ? a.R : 0;
+    static_assert(C::kMaxNew <= 32, "one new key a lane");
 #pragma unroll 1
-    for (int idx = st; idx < my_rows * (kD / 2); idx += kSoftThreads) {
+    for (int idx = st; idx < my_rows * (kD / 2); idx += kSoftThreads) {  // warp-uniform
       const int rr = idx / (kD / 2), d = 2 * (idx % (kD / 2));
       const int row = mrow0 + rr;
       const int p = mblock * kR + row;
-      float mc[16], lc[16], sn[C::kMaxNew];
+      float2 ml = make_float2(-INFINITY, 0.f);  // (m, l) of partial `lane`
+      if (lane < csize) ml = *reinterpret_cast<const float2*>(recv + (lane * rpc + rr) * kRowF + kD);
+      const float sn = lane < n_new ? s_new[rr * a.R + lane] : -INFINITY;
+      float mx = fmaxf(ml.x, sn);
 #pragma unroll
-      for (int c = 0; c < 16; ++c) {
-        // slots past the cluster read partial 0 (always present) with weight 0
-        const float* part = recv + ((c < csize ? c : 0) * rpc + rr) * kRowF + kD;
-        mc[c] = c < csize ? part[0] : -INFINITY;
-        lc[c] = c < csize ? part[1] : 0.f;
-      }
-#pragma unroll
-      for (int n = 0; n < C::kMaxNew; ++n) sn[n] = n < n_new ? s_new[rr * a.R + n] : -INFINITY;
-      float mx = -INFINITY;
-#pragma unroll
-      for (int c = 0; c < 16; ++c) mx = fmaxf(mx, mc[c]);
-#pragma unroll
-      for (int n = 0; n < C::kMaxNew; ++n) mx = fmaxf(mx, sn[n]);
+      for (int sh = 16; sh >= 1; sh >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, sh));
       const float msub = mx == -INFINITY ? 0.f : mx;  // no key at all: every weight 0
-      float lsum = 0.f;
+      const float wp = ex2(ml.x - msub);              // ex2(-inf) = 0
+      const float wn = ex2(sn - msub);
+      float lsum = fmaf(wp, ml.y, wn);
 #pragma unroll
-      for (int c = 0; c < 16; ++c) {
-        mc[c] = ex2(mc[c] - msub);  // ex2(-inf) = 0
-        lsum = fmaf(mc[c], lc[c], lsum);
-      }
-#pragma unroll
-      for (int n = 0; n < C::kMaxNew; ++n) {
-        sn[n] = ex2(sn[n] - msub);
-        lsum += sn[n];
-      }
+      for (int sh = 16; sh >= 1; sh >>= 1) lsum += __shfl_xor_sync(0xffffffffu, lsum, sh);
       float2 acc = make_float2(0.f, 0.f);
-#pragma unroll
-      for (int c = 0; c < 16; ++c) {
-        if (c < csize) {
-          const float2 o = *reinterpret_cast<const float2*>(recv + ((c < csize ? c : 0) * rpc + rr) * kRowF + d);
-          acc.x = fmaf(mc[c], o.x, acc.x);
-          acc.y = fmaf(mc[c], o.y, acc.y);
+#pragma unroll 1
+      for (int c = 0; c < csize; ++c) {
+        {
+          const float w = __shfl_sync(0xffffffffu, wp, c);
+          const float2 o = *reinterpret_cast<const float2*>(recv + (c * rpc + rr) * kRowF + d);
+          acc.x = fmaf(w, o.x, acc.x);
+          acc.y = fmaf(w, o.y, acc.y);
         }
       }
-#pragma unroll
-      for (int n = 0; n < C::kMaxNew; ++n) {
-        if (n < n_new) {
+#pragma unroll 1
+      for (int n = 0; n < n_new; ++n) {
+        {
+          const float w = __shfl_sync(0xffffffffu, wn, n);
           const uint32_t v2 = *reinterpret_cast<const uint32_t*>(smem + C::kOffNewV + n * kNewRow + d * 2);
-          acc.x = fmaf(sn[n], sd_bf16_lo(v2), acc.x);
-          acc.y = fmaf(sn[n], sd_bf16_hi(v2), acc.y);
+          acc.x = fmaf(w, sd_bf16_lo(v2), acc.x);
+          acc.y = fmaf(w, sd_bf16_hi(v2), acc.y);
         }
       }
       if (valid && p < a.M && lsum > 0.f) {
