@@ -241,6 +241,14 @@ __device__ __forceinline__ void umma(uint32_t d_tmem, uint64_t a, uint64_t b, ui
       "l"(a), "l"(b), "r"(idesc), "r"(accumulate)
       : "memory");
 }
+// one lane of the (converged) warp
+__device__ __forceinline__ bool elect_one() {
+  uint32_t pred = 0;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\telect.sync _|p, 0xffffffff;\n\tselp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(pred));
+  return pred != 0;
+}
 __device__ __forceinline__ void umma_commit(uint32_t bar) {
   asm volatile(
       "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
@@ -499,31 +507,35 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == 0) {
     // -------------------------------------------------------------- producer
-    if (lane == 0 && n_tiles > 0) {
-      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_k128)) : "memory");
-      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_v128)) : "memory");
+    // the whole warp waits, one elected lane issues the copies
+    if (n_tiles > 0) {
       const int z = b * a.Hkv + kvh;
-      // chained layers: the cluster launched last (the last KV head of the
-      // last scene) starts only when the previous layer frees its SMs; the
-      // first head's CTAs bring that head's tiles of their own key range
-      // into L2 meanwhile
-      if (kFused && a.early && kvh == 0 && b == static_cast<int>(gridDim.z) - 1 && a.Hkv > 1) {
-        const int zl = b * a.Hkv + a.Hkv - 1;
-        for (int t = 0; t < n_tiles; ++t)
+      if (elect_one()) {
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_k128)) : "memory");
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_v128)) : "memory");
+        // chained layers: the cluster launched last (the last KV head of the
+        // last scene) starts only when the previous layer frees its SMs; the
+        // first head's CTAs bring that head's tiles of their own key range
+        // into L2 meanwhile
+        if (kFused && a.early && kvh == 0 && b == static_cast<int>(gridDim.z) - 1 && a.Hkv > 1) {
+          const int zl = b * a.Hkv + a.Hkv - 1;
+          for (int t = 0; t < n_tiles; ++t)
 #pragma unroll
-          for (int h = 0; h < 2; ++h) {
-            tma_prefetch_3d(&tm_k128, h * 64, key_begin + t * kStageKeys, zl);
-            tma_prefetch_3d(&tm_v128, h * 64, key_begin + t * kStageKeys, zl);
-          }
-        // and that head's query and new key / value rows
-        if (rank == 0)
-          for (int i = 0; i < a.R; ++i) {
-            const long long row = static_cast<long long>(b) * a.R + i;
-            bulk_prefetch_l2(a.qw + (row * a.Hq + (a.Hkv - 1) * a.G) * kD, a.G * kD * 2);
-            bulk_prefetch_l2(a.k_new + (row * a.Hkv + a.Hkv - 1) * kD, kD * 2);
-            bulk_prefetch_l2(a.v_new + (row * a.Hkv + a.Hkv - 1) * kD, kD * 2);
-          }
+            for (int h = 0; h < 2; ++h) {
+              tma_prefetch_3d(&tm_k128, h * 64, key_begin + t * kStageKeys, zl);
+              tma_prefetch_3d(&tm_v128, h * 64, key_begin + t * kStageKeys, zl);
+            }
+          // and that head's query and new key / value rows
+          if (rank == 0)
+            for (int i = 0; i < a.R; ++i) {
+              const long long row = static_cast<long long>(b) * a.R + i;
+              bulk_prefetch_l2(a.qw + (row * a.Hq + (a.Hkv - 1) * a.G) * kD, a.G * kD * 2);
+              bulk_prefetch_l2(a.k_new + (row * a.Hkv + a.Hkv - 1) * kD, kD * 2);
+              bulk_prefetch_l2(a.v_new + (row * a.Hkv + a.Hkv - 1) * kD, kD * 2);
+            }
+        }
       }
+      __syncwarp();
       for (int pass = 0; pass < 2; ++pass) {
         if (pass == 1) {
           // every MMA of pass 0 is done when the decision is out
@@ -540,13 +552,19 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint32_t kst = base + s * kKV, vst = base + C::kRingV + s * kKV;
           if (kSplit) {
             if (t >= kS) mbar_wait(SREADY(T - kS), ring_parity(T - kS));
-            mbar_expect_tx(FULLK(s), static_cast<uint32_t>(kKV));
+            if (elect_one()) {
+              mbar_expect_tx(FULLK(s), static_cast<uint32_t>(kKV));
 #pragma unroll
-            for (int h = 0; h < 2; ++h) tma_load_3d(kst + h * kHalf, &tm_k128, FULLK(s), h * 64, y0, z);
+              for (int h = 0; h < 2; ++h) tma_load_3d(kst + h * kHalf, &tm_k128, FULLK(s), h * 64, y0, z);
+            }
+            __syncwarp();
             if (t >= kS) mbar_wait(PVDONE(T - kS), ring_parity(T - kS));
-            mbar_expect_tx(FULLV(s), static_cast<uint32_t>(kKV));
+            if (elect_one()) {
+              mbar_expect_tx(FULLV(s), static_cast<uint32_t>(kKV));
 #pragma unroll
-            for (int h = 0; h < 2; ++h) tma_load_3d(vst + h * kHalf, &tm_v128, FULLV(s), h * 64, y0, z);
+              for (int h = 0; h < 2; ++h) tma_load_3d(vst + h * kHalf, &tm_v128, FULLV(s), h * 64, y0, z);
+            }
+            __syncwarp();
           } else {
             if (t >= kS) mbar_wait(PVDONE(T - kS), ring_parity(T - kS));
             mbar_expect_tx(FULLK(s), static_cast<uint32_t>(2 * kKV));
@@ -564,9 +582,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     cluster_wait();
   } else if (warp == 1) {
     // -------------------------------------------------------------- S issue
-    // S(T) and PV(T) come from two threads (this one and the PV warp's), so
-    // that one batch is issued while the other executes.
-    if (lane == 0 && n_tiles > 0) {
+    // S(T) and PV(T) come from two warps (this one and the PV warp), so that
+    // one batch is issued while the other executes; the whole warp waits and
+    // one elected lane issues.
+    if (n_tiles > 0) {
       mbar_wait(QFULL, 0);
       // base descriptors; a K step only moves the start address (low field, no carry)
       const uint64_t dK0 = umma_desc(base, 16, 1024);  // K tile: K-major
@@ -586,11 +605,14 @@ __global__ void __launch_bounds__(kThreads, 1)
           tc_fence_after();
           const uint64_t dk = dK0 + static_cast<uint64_t>((st_ * kKV) >> 4);
           const uint32_t ts = tmem_s + kR * (T & 1);
+          if (elect_one()) {
 #pragma unroll
-          for (int kk = 0; kk < 8; ++kk)
-            umma(ts, dk + (((kk >> 2) * kHalf + (kk & 3) * 32) >> 4),
-                 dQ + (((kk >> 2) * C::kQHalf + (kk & 3) * 32) >> 4), kIdescS, kk > 0 ? 1 : 0);
-          umma_commit(SREADY(T));
+            for (int kk = 0; kk < 8; ++kk)
+              umma(ts, dk + (((kk >> 2) * kHalf + (kk & 3) * 32) >> 4),
+                   dQ + (((kk >> 2) * C::kQHalf + (kk & 3) * 32) >> 4), kIdescS, kk > 0 ? 1 : 0);
+            umma_commit(SREADY(T));
+          }
+          __syncwarp();
         }
       }
     }
@@ -599,7 +621,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     cluster_wait();
   } else if (warp == kPvWarp) {
     // -------------------------------------------------------------- PV issue
-    if (lane == 0 && n_tiles > 0) {
+    if (n_tiles > 0) {
       const uint64_t dV0 = umma_desc(base + C::kRingV, kHalf, 1024);  // V^T: MN-major
       // P^T: MN-major, one swizzle atom wide (kR rows), 8-key groups 8 * kPRow apart
       const uint64_t dP0 = umma_desc(base + C::kOffP, 0, 8 * C::kPRow, C::kPLayout);
@@ -616,11 +638,14 @@ __global__ void __launch_bounds__(kThreads, 1)
           tc_fence_after();
           const uint64_t dv = dV0 + static_cast<uint64_t>(((T % kS) * kKV) >> 4);
           const uint64_t dp = dP0 + static_cast<uint64_t>(((T & 1) * C::kP) >> 4);
+          if (elect_one()) {
 #pragma unroll
-          for (int kk = 0; kk < 8; ++kk)
-            umma(tmem_o, dv + (kk * 2048 >> 4), dp + (kk * 16 * C::kPRow >> 4), kIdescO,
-                 (t > 0 || kk > 0) ? 1 : 0);
-          umma_commit(PVDONE(T));
+            for (int kk = 0; kk < 8; ++kk)
+              umma(tmem_o, dv + (kk * 2048 >> 4), dp + (kk * 16 * C::kPRow >> 4), kIdescO,
+                   (t > 0 || kk > 0) ? 1 : 0);
+            umma_commit(PVDONE(T));
+          }
+          __syncwarp();
         }
       }
     }
