@@ -241,6 +241,11 @@ __device__ __forceinline__ void umma(uint32_t d_tmem, uint64_t a, uint64_t b, ui
       "l"(a), "l"(b), "r"(idesc), "r"(accumulate)
       : "memory");
 }
+__device__ __forceinline__ __nv_bfloat162 as_bf162(uint32_t w) {
+  __nv_bfloat162 v;
+  memcpy(&v, &w, 4);
+  return v;
+}
 // one lane of the (converged) warp
 __device__ __forceinline__ bool elect_one() {
   uint32_t pred = 0;
@@ -795,7 +800,57 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (tail) ok[j] = ok[j] && key <= row_lim[row0 + j0 + j];
       }
     };
-    if (n_tiles > 0) {
+    if (kFused) {
+      // references: the larger score of each row against its own new key and
+      // new key 0 (keys the row sees, so its largest weight is at least about
+      // 1 and its sum cannot vanish), taken while S(0) and S(1) run; bf16 dot
+      // products suffice for a reference. 8 threads a row, 16 d each.
+      const int sub = lane & 7;
+#pragma unroll 1
+      for (int r = st >> 3; r < kR; r += kSoftThreads / 8) {  // warp-uniform trip count
+        const int p = mblock * kR + r;
+        const bool row_ok = valid && p < a.M;
+        const int n = row_ok ? gdiv(p) : 0;  // the row's own new key
+        __nv_bfloat162 acc0 = __float2bfloat162_rn(0.f), acc1 = acc0, acc2 = acc0, acc3 = acc0;
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+          const int c = sub + 8 * u;
+          const uint4 qw = *reinterpret_cast<const uint4*>(smem + C::kOffQ + (c >> 3) * C::kQHalf + r * 128 +
+                                                           (((c & 7) ^ (r & 7)) << 4));
+          const uint4 kw = *reinterpret_cast<const uint4*>(smem + C::kOffNewK + n * kNewRow + c * 16);
+          const uint4 k0 = *reinterpret_cast<const uint4*>(smem + C::kOffNewK + c * 16);
+          acc0 = __hfma2(as_bf162(qw.x), as_bf162(kw.x), acc0);
+          acc1 = __hfma2(as_bf162(qw.y), as_bf162(kw.y), acc1);
+          acc2 = __hfma2(as_bf162(qw.x), as_bf162(k0.x), acc2);
+          acc3 = __hfma2(as_bf162(qw.y), as_bf162(k0.y), acc3);
+          acc0 = __hfma2(as_bf162(qw.z), as_bf162(kw.z), acc0);
+          acc1 = __hfma2(as_bf162(qw.w), as_bf162(kw.w), acc1);
+          acc2 = __hfma2(as_bf162(qw.z), as_bf162(k0.z), acc2);
+          acc3 = __hfma2(as_bf162(qw.w), as_bf162(k0.w), acc3);
+        }
+        float sd = (__low2float(acc0) + __high2float(acc0)) + (__low2float(acc1) + __high2float(acc1));
+        float s0 = (__low2float(acc2) + __high2float(acc2)) + (__low2float(acc3) + __high2float(acc3));
+#pragma unroll
+        for (int sh = 1; sh < 8; sh <<= 1) {
+          sd += __shfl_xor_sync(0xffffffffu, sd, sh);
+          s0 += __shfl_xor_sync(0xffffffffu, s0, sh);
+        }
+        const float best = row_ok ? fmaxf(sd, s0) : -INFINITY;
+        if (sub == 0) row_ref[r] = best == -INFINITY ? -INFINITY : best * sl;
+      }
+      named_bar_sync(2, kSoftThreads);
+      if (kRefRegs) {
+        const float4* rr4 = reinterpret_cast<const float4*>(row_ref + row0);
+#pragma unroll
+        for (int j4 = 0; j4 < (kRefRegs ? kRpt / 4 : 0); ++j4) {
+          const float4 x = rr4[j4];
+          ref[(4 * j4 + 0) % (kRefRegs ? kRpt : 1)] = x.x;
+          ref[(4 * j4 + 1) % (kRefRegs ? kRpt : 1)] = x.y;
+          ref[(4 * j4 + 2) % (kRefRegs ? kRpt : 1)] = x.z;
+          ref[(4 * j4 + 3) % (kRefRegs ? kRpt : 1)] = x.w;
+        }
+      }
+    } else if (n_tiles > 0) {
       // references: exact row maxima of the first tile (through the P buffers,
       // which no P has used yet)
       mbar_wait(SREADY(0), 0);

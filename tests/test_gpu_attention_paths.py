@@ -51,7 +51,7 @@ def test_attention_kernel_paths(kernel):
     assert "OK" in res.stdout
 
 
-def _planted(seed, plants, fused, R=8):
+def _planted(seed, plants, fused, R=8, new_plants=()):
     """B=1, 32 q / 8 KV heads x 128, L=4096 prefix, R=8: key n of KV head h // 4
     is set to alpha * (rotated) q[i][h], so that row i of head h scores it far
     above everything in the first tile of its split."""
@@ -73,6 +73,15 @@ def _planted(seed, plants, fused, R=8):
     q_rot = oracle.mrope_apply(q64, pos[:, :, None, :], sections, 0, 1e6) if fused else q64
     for (h, i, n, alpha) in plants:
         k[0, h // (Hq // Hkv), n] = alpha * q_rot[0, i, h] / np.linalg.norm(q_rot[0, i, h]) * 12.0
+    if new_plants:
+        # new key rows i and 0 of KV head h // 4 set (after their rotation) to
+        # alpha * q[i][h]: raw rows are the inverse rotation of the target
+        kn = k_new.float().numpy().astype(np.float64)
+        for (h, i, alpha) in new_plants:
+            target = alpha * q_rot[0, i, h] / np.linalg.norm(q_rot[0, i, h]) * 12.0
+            for n in (i, 0):
+                kn[0, n, h // (Hq // Hkv)] = oracle.mrope_apply(target, -pos[0, n], sections, 0, 1e6)
+        k_new = workloads.to_bf16(kn)
     if fused:
         k[:, :, L:] = np.nan  # stale rows past the prefix
         v[:, :, L:] = np.nan
@@ -98,9 +107,10 @@ def _planted(seed, plants, fused, R=8):
 def test_fixed_reference_fallback_pass(fused, R):
     # a planted key scores ~17 * alpha in log2 units (|k| = 12 alpha along q,
     # |q| ~ 11.3, scale log2(e) / sqrt(128)): alpha 6 puts it ~100 above the
-    # first tile's maximum (beyond the 64 one pass allows, so its split runs the
-    # fallback pass), alpha 2.5 ~40 above (kept by the single pass), alpha -6
-    # far below; keys in later tiles of splits 0, 3 and 7
+    # row's reference (the first tile's maximum, or in the fused layer the
+    # row's score against its own new key and new key 0; beyond the 64 one pass
+    # allows, so its split runs the fallback pass), alpha 2.5 ~40 above (kept by
+    # the single pass), alpha -6 far below; keys in later tiles of splits 0, 3 and 7
     import numpy as np
     from tests.helpers import ATTN_ATOL
     plants = [(0, 0, 300, 6.0), (5, 3, 2000, 6.0), (31, 7, 4000, 6.0), (12, 2, 1700, 2.5),
@@ -112,6 +122,22 @@ def test_fixed_reference_fallback_pass(fused, R):
     assert e <= ATTN_ATOL, e
     # the planted rows are dominated by their key (the output is its value row)
     assert np.abs(ref[0, 0, 0]).max() > 0.5
+
+
+@pytest.mark.parametrize("alpha", [-9.0, -2.5])
+def test_fused_reference_below_the_prefix(alpha):
+    # the fused layer's reference of a row is its larger score against its own
+    # new key and new key 0; both planted at ~17 * alpha in log2 units leave
+    # every prefix key of that row ~150 (alpha -9: beyond the 64 one pass
+    # allows, so its head's splits run the fallback pass; a single pass would
+    # overflow fp32 there) or ~40 (alpha -2.5) above the reference
+    import numpy as np
+    from tests.helpers import ATTN_ATOL
+    out, ref, err = _planted(11, [], True, 8, new_plants=[(9, 5, alpha), (22, 3, alpha), (30, 0, alpha)])
+    assert err == 0
+    assert np.isfinite(out).all()
+    e = np.abs(out - ref).max()
+    assert e <= ATTN_ATOL, e
 
 
 def _fused_case(R, prefix, layer):
