@@ -1118,23 +1118,19 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
       for (int sh = 16; sh >= 1; sh >>= 1) lsum += __shfl_xor_sync(0xffffffffu, lsum, sh);
       float2 acc = make_float2(0.f, 0.f);
-#pragma unroll 1
+#pragma unroll 4
       for (int c = 0; c < csize; ++c) {
-        {
-          const float w = __shfl_sync(0xffffffffu, wp, c);
-          const float2 o = *reinterpret_cast<const float2*>(recv + (c * rpc + rr) * kRowF + d);
-          acc.x = fmaf(w, o.x, acc.x);
-          acc.y = fmaf(w, o.y, acc.y);
-        }
+        const float w = __shfl_sync(0xffffffffu, wp, c);
+        const float2 o = *reinterpret_cast<const float2*>(recv + (c * rpc + rr) * kRowF + d);
+        acc.x = fmaf(w, o.x, acc.x);
+        acc.y = fmaf(w, o.y, acc.y);
       }
-#pragma unroll 1
+#pragma unroll 4
       for (int n = 0; n < n_new; ++n) {
-        {
-          const float w = __shfl_sync(0xffffffffu, wn, n);
-          const uint32_t v2 = *reinterpret_cast<const uint32_t*>(smem + C::kOffNewV + n * kNewRow + d * 2);
-          acc.x = fmaf(w, sd_bf16_lo(v2), acc.x);
-          acc.y = fmaf(w, sd_bf16_hi(v2), acc.y);
-        }
+        const float w = __shfl_sync(0xffffffffu, wn, n);
+        const uint32_t v2 = *reinterpret_cast<const uint32_t*>(smem + C::kOffNewV + n * kNewRow + d * 2);
+        acc.x = fmaf(w, sd_bf16_lo(v2), acc.x);
+        acc.y = fmaf(w, sd_bf16_hi(v2), acc.y);
       }
       if (valid && p < a.M && lsum > 0.f) {
         const float inv_l = 1.f / lsum;
