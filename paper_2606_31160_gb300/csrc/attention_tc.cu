@@ -455,19 +455,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (kFused && !a.early) griddep_wait();  // len, pos and the prefix may come from the previous kernel
   int* s_len = reinterpret_cast<int*>(smem + C::kOffMisc + 12);
   if (threadIdx.x == 0) {
-    const int len0 = a.len[b];
-    *s_len = len0;
-    if (kFused) {
-      // advance the scene's length once every CTA of the scene has read it:
-      // the last CTA to take a ticket writes it (the fence orders this CTA's
-      // read before its ticket)
-      __threadfence();
-      const uint32_t total = gridDim.x * gridDim.y;
-      if (atomicAdd(&a.ticket[b], 1u) == total - 1) {
-        if (len0 >= 0 && len0 + a.R <= a.cap) a.len[b] = len0 + a.R;
-        a.ticket[b] = 0;
-      }
-    }
+    *s_len = a.len[b];  // the scene's length advances at the producer's end
   }
   if (kFused && threadIdx.x >= 64 && threadIdx.x < 64 + kSoftThreads) {
     // rotation table of the R new positions: (cos, sin) per (row, pair),
@@ -504,8 +492,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   // the tensor-core loop covers the prefix (fused) or every key (standalone)
   const int loop_keys = valid ? (kFused ? L_pre : n_keys) : 0;
   const int nblk = (loop_keys + 31) / 32;
-  const int blk_begin = static_cast<int>((static_cast<long long>(rank) * nblk) / csize);
-  const int blk_end = static_cast<int>((static_cast<long long>(rank + 1) * nblk) / csize);
+  // rank * nblk < 2^31 (16 ranks, nblk <= cap / 32): 32-bit division
+  const int blk_begin = static_cast<int>((static_cast<uint32_t>(rank) * nblk) / static_cast<uint32_t>(csize));
+  const int blk_end = static_cast<int>((static_cast<uint32_t>(rank + 1) * nblk) / static_cast<uint32_t>(csize));
   const int key_begin = blk_begin * 32;
   const int key_end = min(blk_end * 32, loop_keys);
   const int n_tiles = (blk_end - blk_begin + 3) / 4;
@@ -584,6 +573,20 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     __syncwarp();
     cluster_arrive();  // the cluster's rings are free (see the softmax branch)
+    if (kFused && elect_one()) {
+      // advance the scene's length once every CTA of the scene has read it:
+      // the last CTA to take a ticket writes it. This lane (thread 0) read
+      // the length in the prologue; the fence orders that read before the
+      // ticket. Taken after the cluster arrival, so no barrier waits for it.
+      __threadfence();
+      const uint32_t total = gridDim.x * gridDim.y;
+      if (atomicAdd(&a.ticket[b], 1u) == total - 1) {
+        const int len0 = *s_len;
+        if (len0 >= 0 && len0 + a.R <= a.cap) a.len[b] = len0 + a.R;
+        a.ticket[b] = 0;
+      }
+    }
+    __syncwarp();
     cluster_wait();
   } else if (warp == 1) {
     // -------------------------------------------------------------- S issue
@@ -1118,12 +1121,27 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
       for (int sh = 16; sh >= 1; sh >>= 1) lsum += __shfl_xor_sync(0xffffffffu, lsum, sh);
       float2 acc = make_float2(0.f, 0.f);
+      // the fused layer's ranks share each row's reference unless one of them
+      // ran the second pass: then every partial has the same weight
+      const float m0 = __shfl_sync(0xffffffffu, ml.x, 0);
+      if (__all_sync(0xffffffffu, lane >= csize || ml.x == m0)) {
 #pragma unroll 4
-      for (int c = 0; c < csize; ++c) {
-        const float w = __shfl_sync(0xffffffffu, wp, c);
-        const float2 o = *reinterpret_cast<const float2*>(recv + (c * rpc + rr) * kRowF + d);
-        acc.x = fmaf(w, o.x, acc.x);
-        acc.y = fmaf(w, o.y, acc.y);
+        for (int c = 0; c < csize; ++c) {
+          const float2 o = *reinterpret_cast<const float2*>(recv + (c * rpc + rr) * kRowF + d);
+          acc.x += o.x;
+          acc.y += o.y;
+        }
+        const float w = __shfl_sync(0xffffffffu, wp, 0);
+        acc.x *= w;
+        acc.y *= w;
+      } else {
+#pragma unroll 4
+        for (int c = 0; c < csize; ++c) {
+          const float w = __shfl_sync(0xffffffffu, wp, c);
+          const float2 o = *reinterpret_cast<const float2*>(recv + (c * rpc + rr) * kRowF + d);
+          acc.x = fmaf(w, o.x, acc.x);
+          acc.y = fmaf(w, o.y, acc.y);
+        }
       }
 #pragma unroll 4
       for (int n = 0; n < n_new; ++n) {
