@@ -1051,13 +1051,18 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int my_rows = rows_of(rank);
     if (st == 0) mbar_expect_tx(RECV, static_cast<uint32_t>(csize * my_rows * kRowBytes));
     cluster_wait();  // every peer's ring is free to receive
-    if (st < csize && rows_of(st) > 0) {
-      // thread c sends rank c's rows to rank c, into its slots [rank * rpc, ...)
-      bulk_copy_s2s(cluster_map(base + C::kRecv + rank * rpc * kRowBytes, st),
-                    base + C::kSend + st * rpc * kRowBytes, static_cast<uint32_t>(rows_of(st) * kRowBytes),
-                    cluster_map(RECV, st));
+    // softmax warp w sends rank c's rows to rank c (c = w, w + 8), into its
+    // slots [rank * rpc, ...); one elected lane of the converged warp issues
+    if (elect_one()) {
+#pragma unroll 1
+      for (int c = warp - 2; c < csize; c += kSoftWarps)
+        if (rows_of(c) > 0)
+          bulk_copy_s2s(cluster_map(base + C::kRecv + rank * rpc * kRowBytes, c),
+                        base + C::kSend + c * rpc * kRowBytes, static_cast<uint32_t>(rows_of(c) * kRowBytes),
+                        cluster_map(RECV, c));
       asm volatile("cp.async.bulk.commit_group;" ::: "memory");
     }
+    __syncwarp();
     const int mrow0 = rank * rpc;  // the rows this CTA merges
     float* s_new = reinterpret_cast<float*>(smem + C::kNewS);  // [rpc][R] scores of the new keys
     if (kFused && valid) {
@@ -1157,7 +1162,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                                      d) = cvt_bf16x2(acc.x * inv_l, acc.y * inv_l);
       }
     }
-    if (st < csize && rows_of(st) > 0) asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+    if (elect_one()) asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+    __syncwarp();
     if (kFused && valid) {
       // every CTA of the cluster read the raw rows before its main loop (the
       // cluster barrier above is behind all of them): store the rotated query
