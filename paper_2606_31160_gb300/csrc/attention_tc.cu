@@ -13,27 +13,28 @@
 // an N = 64 product costs about what an N = 32 one does. Both accumulators
 // live in tensor memory (S double-buffered): 3 kR columns.
 //
-// Warp roles in a CTA (320 threads):
+// Warp roles in a CTA (352 threads). The issuing warps run converged: every
+// lane waits on the barriers and one elected lane issues (issued from a
+// one-lane branch instead, a batch of 8 MMAs took ~270 ns).
 //   warp 0      TMA producer: 128-key tiles of K and V (128B-swizzled boxes)
-//               into a K ring and a V ring of kS slots each. 32 rows: 3 slots,
-//               a tile's K and V load together once the slot's previous PV
-//               is done. 64 rows (less shared memory left): 2 slots, a K slot
-//               is refilled once its S product is done and a V slot once its
-//               PV product is, so S still runs two tiles ahead.
-//   warp 1      allocates tensor memory; one lane issues every tcgen05.mma.
-//               S runs two tiles ahead: per tile it issues PV(t) and commits
-//               "PV(t) done" (V slot free), then S(t+2) and commits
-//               "S(t+2) ready" (K slot free; implies PV(t) done, so the
-//               softmax needs no other wait). Two commits a tile: each drains
-//               the MMA pipe for ~180 cycles.
+//               into a K ring and a V ring of kS slots each (32 rows: 3, 64
+//               rows: 2), with a barrier each: a K slot refills once its S
+//               product is done, a V slot once its PV product is.
+//   warp 1      allocates tensor memory; issues S(t) once the softmax has read
+//               S(t - 2) and commits "S(t) ready".
 //   warps 2..9  softmax: thread (t, h) owns key lane t of S^T and query rows
 //               h kR/2 .. h kR/2 + kR/2 - 1; P = exp2(S - ref) goes to shared
 //               memory as P^T (MN-major; 64-byte swizzle for 32 rows, 128-byte
-//               for 64), 16-byte stores.
+//               for 64), 16-byte stores, once PV(t - 2) has read that buffer.
+//   warp 10     issues PV(t) once P(t) is stored and commits "PV(t) done";
+//               one batch is issued while the other executes.
 //
-// Softmax with a fixed reference. The reference of a row is the exact maximum
-// of the CTA's first tile; every later tile uses it unchanged, so the loop has
-// no cross-warp step and O is never rescaled. The result is exact as long as
+// Softmax with a fixed reference. The reference of a row is, in the
+// standalone kernel, the exact maximum of the CTA's first tile and, in the
+// fused layer, the row's larger score against its own new key and new key 0
+// (keys the row sees, so its largest weight is about 1 or more), taken while
+// the first S products run; every tile uses it unchanged, so the loop has no
+// cross-warp step and O is never rescaled. The result is exact as long as
 // no score exceeds its reference by more than kSlack (log2 units), which keeps
 // every weight below 2^kSlack and every sum far inside fp32 range; each thread
 // tracks the largest excess it saw, and a CTA where some excess is larger runs
@@ -397,15 +398,13 @@ __global__ void __launch_bounds__(kThreads, 1)
   // (one slot per ring stage) are tcgen05.commit arrivals. A slot's next
   // phase cannot complete before each of its waiters has seen the current
   // one: S(T + kS) needs the K tile loaded after the producer's wait for
-  // SREADY(T), and is issued after PV(T + kS - 2), which needs PFULL from the
-  // softmax's tile T + kS - 2 >= T; PV(T + kS) needs the V tile loaded after
-  // the producer's wait for PVDONE(T), and the softmax waits for PVDONE only
-  // once a pass, on its last tile.
+  // SREADY(T); PV(T + kS) needs the V tile loaded after the producer's wait
+  // for PVDONE(T); the softmax's tile T + 1 follows its wait for SREADY(T),
+  // and its wait for PVDONE(T) comes before P(T + 2), which PV(T + kS) needs.
   // K and V of a tile have their own barriers: a K slot refills once its S
   // product is done, a V slot once its PV product is.
-  constexpr bool kSplit = true;
   auto FULLK = [&](int s) { return bar(s); };
-  auto FULLV = [&](int s) { return kSplit ? bar(kS + s) : bar(s); };
+  auto FULLV = [&](int s) { return bar(kS + s); };
   auto PFULL = [&](int b) { return bar(2 * kS + b); };
   auto SREADY = [&](int T) { return bar(2 * kS + 2 + T % kS); };
   auto PVDONE = [&](int T) { return bar(3 * kS + 2 + T % kS); };
@@ -433,7 +432,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (threadIdx.x == 0) {
     for (int s = 0; s < kS; ++s) {
       mbar_init(FULLK(s), 1);
-      if (kSplit) mbar_init(FULLV(s), 1);
+      mbar_init(FULLV(s), 1);
       mbar_init(SREADY(s), 1);
       mbar_init(PVDONE(s), 1);
     }
@@ -544,30 +543,20 @@ __global__ void __launch_bounds__(kThreads, 1)
           const int y0 = key_begin + t * kStageKeys;
           // slot s last held tile T - kS (all of pass 0 is done before pass 1)
           const uint32_t kst = base + s * kKV, vst = base + C::kRingV + s * kKV;
-          if (kSplit) {
-            if (t >= kS) mbar_wait(SREADY(T - kS), ring_parity(T - kS));
-            if (elect_one()) {
-              mbar_expect_tx(FULLK(s), static_cast<uint32_t>(kKV));
+          if (t >= kS) mbar_wait(SREADY(T - kS), ring_parity(T - kS));
+          if (elect_one()) {
+            mbar_expect_tx(FULLK(s), static_cast<uint32_t>(kKV));
 #pragma unroll
-              for (int h = 0; h < 2; ++h) tma_load_3d(kst + h * kHalf, &tm_k128, FULLK(s), h * 64, y0, z);
-            }
-            __syncwarp();
-            if (t >= kS) mbar_wait(PVDONE(T - kS), ring_parity(T - kS));
-            if (elect_one()) {
-              mbar_expect_tx(FULLV(s), static_cast<uint32_t>(kKV));
-#pragma unroll
-              for (int h = 0; h < 2; ++h) tma_load_3d(vst + h * kHalf, &tm_v128, FULLV(s), h * 64, y0, z);
-            }
-            __syncwarp();
-          } else {
-            if (t >= kS) mbar_wait(PVDONE(T - kS), ring_parity(T - kS));
-            mbar_expect_tx(FULLK(s), static_cast<uint32_t>(2 * kKV));
-#pragma unroll
-            for (int h = 0; h < 2; ++h) {
-              tma_load_3d(kst + h * kHalf, &tm_k128, FULLK(s), h * 64, y0, z);
-              tma_load_3d(vst + h * kHalf, &tm_v128, FULLK(s), h * 64, y0, z);
-            }
+            for (int h = 0; h < 2; ++h) tma_load_3d(kst + h * kHalf, &tm_k128, FULLK(s), h * 64, y0, z);
           }
+          __syncwarp();
+          if (t >= kS) mbar_wait(PVDONE(T - kS), ring_parity(T - kS));
+          if (elect_one()) {
+            mbar_expect_tx(FULLV(s), static_cast<uint32_t>(kKV));
+#pragma unroll
+            for (int h = 0; h < 2; ++h) tma_load_3d(vst + h * kHalf, &tm_v128, FULLV(s), h * 64, y0, z);
+          }
+          __syncwarp();
         }
       }
     }
@@ -642,7 +631,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int t = 0; t < n_tiles; ++t) {
           const int T = T0 + t;
           mbar_wait(PFULL(T & 1), (T >> 1) & 1);
-          mbar_wait(FULLV(T % kS), ring_parity(T));  // (FULLK when K and V share a barrier)
+          mbar_wait(FULLV(T % kS), ring_parity(T));  // the V tile has landed
           tc_fence_after();
           const uint64_t dv = dV0 + static_cast<uint64_t>(((T % kS) * kKV) >> 4);
           const uint64_t dp = dP0 + static_cast<uint64_t>(((T & 1) * C::kP) >> 4);
@@ -778,7 +767,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // The reference of a row (log2 units, -inf: no key yet) lives in row_ref;
     // with 32 rows a thread also keeps its 16 in registers, with 64 rows it
     // reloads them every tile (broadcast loads) to stay within the registers
-    // that 10 warps leave a thread.
+    // that 11 warps leave a thread.
     constexpr bool kRefRegs = kR == 32;
     float ref[kRefRegs ? kRpt : 1];
     float lp[kRpt];   // per-row partial sums of this thread's key lane
