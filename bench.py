@@ -197,20 +197,25 @@ class Step:
         self.cases = [workloads.target_layer(B=1, layer=l, ell=[3], scene=scene) for l in range(LAYERS)]
         self.gen_s = time.time() - gen_t0
         c0 = self.cases[0]
-        # host copies (pinned) of the per-step inputs, for the end-to-end leg
-        self.h_q = torch.stack([c.q for c in self.cases]).pin_memory()          # [36,1,R,HQ,D]
-        self.h_k = torch.stack([c.k_new for c in self.cases]).pin_memory()
-        self.h_v = torch.stack([c.v_new for c in self.cases]).pin_memory()
-        self.h_pos = c0.pos.clone().pin_memory()
-        self.h_logits = c0.extra["logits"].clone().pin_memory()
-        self.h_draft = c0.extra["draft"].clone().pin_memory()
-        # device buffers
-        self.q = self.h_q.to(device)
-        self.k = self.h_k.to(device)
-        self.v = self.h_v.to(device)
-        self.pos = self.h_pos.to(device)
-        self.logits = self.h_logits.to(device)
-        self.draft = self.h_draft.to(device)
+        # the per-step inputs live in one device buffer, and their host copies
+        # (the end-to-end leg's source) in one pinned buffer of the same layout,
+        # so that a step's inputs travel in a single copy
+        parts = [("q", torch.stack([c.q for c in self.cases])),         # [36,1,R,HQ,D]
+                 ("k", torch.stack([c.k_new for c in self.cases])),
+                 ("v", torch.stack([c.v_new for c in self.cases])),
+                 ("pos", c0.pos), ("logits", c0.extra["logits"]), ("draft", c0.extra["draft"])]
+        offs, off = [], 0
+        for _, t in parts:
+            offs.append(off)
+            off += (t.numel() * t.element_size() + 255) // 256 * 256
+        self.h_in = torch.empty(off, dtype=torch.uint8).pin_memory()
+        self.d_in = torch.empty(off, dtype=torch.uint8, device=device)
+        for (name, t), o in zip(parts, offs):
+            n = t.numel() * t.element_size()
+            h = self.h_in[o:o + n].view(t.dtype).view(t.shape)
+            h.copy_(t)
+            setattr(self, name, self.d_in[o:o + n].view(t.dtype).view(t.shape))
+        self.d_in.copy_(self.h_in)
         self.lens = torch.full((LAYERS, 1), L, dtype=torch.int32, device=device)
         self.lens0 = self.lens.clone()
         self.caches = [sd.KVCache(c.k_cache.to(device), c.v_cache.to(device), self.lens[l])
@@ -219,8 +224,10 @@ class Step:
         self.ws = sd.workspace(sd.greedy_workspace_bytes(1, K, V), device)
         need = sd.layer_workspace_bytes(1, R, HQ, HKV, D, self.caches[0].shape[2])
         self.ws_layer = [sd.workspace(need, device) for _ in range(LAYERS)]
-        self.n_emit = torch.zeros(1, dtype=torch.int32, device=device)
-        self.tokens = torch.zeros((1, R), dtype=torch.int32, device=device)
+        # the step's result (n_emit, then the R tokens) in one buffer: one copy back
+        self.res = torch.zeros((1 + R,), dtype=torch.int32, device=device)
+        self.n_emit = self.res[:1]
+        self.tokens = self.res[1:].view(1, R)
         self.argmax = torch.zeros((1, R), dtype=torch.int32, device=device)
         self.h_out = torch.zeros((1 + R,), dtype=torch.int32).pin_memory()
         for c in self.cases:  # free host copies of the caches
@@ -276,25 +283,18 @@ class Step:
                                   argmax=self.argmax)
 
     def h2d(self):
-        self.q.copy_(self.h_q, non_blocking=True)
-        self.k.copy_(self.h_k, non_blocking=True)
-        self.v.copy_(self.h_v, non_blocking=True)
-        self.pos.copy_(self.h_pos, non_blocking=True)
-        self.logits.copy_(self.h_logits, non_blocking=True)
-        self.draft.copy_(self.h_draft, non_blocking=True)
+        self.d_in.copy_(self.h_in, non_blocking=True)
 
     def d2h(self):
-        self.h_out[:1].copy_(self.n_emit, non_blocking=True)
-        self.h_out[1:].copy_(self.tokens[0], non_blocking=True)
+        self.h_out.copy_(self.res, non_blocking=True)
 
     @property
     def h2d_bytes(self):
-        return sum(t.numel() * t.element_size() for t in (self.h_q, self.h_k, self.h_v, self.h_pos,
-                                                          self.h_logits, self.h_draft))
+        return self.h_in.numel()  # the inputs and the 256-byte alignment between them
 
     @property
     def d2h_bytes(self):
-        return (1 + R) * 4
+        return self.h_out.numel() * 4
 
 
 def capture(fn):
