@@ -546,9 +546,10 @@ def main():
     ap.add_argument("--sweep-b", type=int, nargs="*", default=None, help="restrict the sweep's batch sizes")
     ap.add_argument("--sweep-l", type=int, nargs="*", default=None, help="restrict the sweep's prefix lengths")
     ap.add_argument("--sweep-k", type=int, nargs="*", default=None, help="restrict the sweep's draft lengths")
-    ap.add_argument("--only", choices=["attention", "layer", "accept", "step"], default=None,
+    ap.add_argument("--only", choices=["attention", "layer", "accept", "step", "sample"], default=None,
                     help="profiling mode: run one kernel family eagerly `steps` times on the "
-                         "target-layer workload (for ncu captures); prints no bench line")
+                         "target-layer workload (sample: the stochastic-acceptance workload) "
+                         "for ncu captures; prints no bench line")
     args = ap.parse_args()
     world, rank, local = dist_env()
     if args.warmup < 3:
@@ -787,9 +788,22 @@ def sweep(args):
 def profile_only(args):
     """Eager launches of one kernel family on the 36-layer target workload,
     for profiler captures (a handful of launches, no timing output)."""
-    from paper_2606_31160_gb300 import build, sd
+    from paper_2606_31160_gb300 import build, sd, workloads
     build.build()
     torch.cuda.set_device(0)
+    if args.only == "sample":
+        # sd_accept_sample on the stochastic-acceptance workload (B=8, K=7, V=151936)
+        dev = torch.device("cuda", 0)
+        w = workloads.stochastic()
+        zt, zd = w["z_target"].to(dev), w["z_draft"].to(dev)
+        dr, u = w["draft"].to(dev), w["u"].to(dev)
+        ws = sd.workspace(sd.sample_workspace_bytes(w["B"], w["K"], w["V"]), dev)
+        for _ in range(args.steps):
+            sd.accept_sample(zt, zd, dr, u, w["temperature"], ws=ws)
+        torch.cuda.synchronize()
+        print(json.dumps({"profile_only": args.only, "launches": args.steps,
+                          "device_error": sd.get_device_error()}))
+        return
     st = Step(torch.device("cuda", 0))
     st.run()  # one full step: rope, append, attention, accept, rollback
     torch.cuda.synchronize()
