@@ -81,7 +81,6 @@ constexpr int round_up(int x, int m) { return (x + m - 1) / m * m; }
 template <int kR>
 struct Cfg {
   static_assert(kR == 32 || kR == 64, "row tile");
-  static constexpr int kRows = kR;
   static constexpr int kRpt = kR / 2;                       // rows per softmax thread
   static constexpr int kMaxNew = kR == 32 ? 16 : 32;        // new rows the fused kernel takes
   // K and V rings of kStages tiles each: a K slot is free once its S product

@@ -92,6 +92,35 @@ def test_back_to_back_layers_with_early_prefix():
     assert sd.get_device_error() == 0
 
 
+@pytest.mark.parametrize("B,K", [(3, 7), (2, 8), (1, 16)])
+def test_back_to_back_layers_several_scenes_and_tiles(B, K):
+    # chained layers with ragged scenes (the cluster launched last is the last
+    # KV head of the last scene) and with the 64-row tile (K = 8: one m-block,
+    # K = 16: two): the early chain gives the same bits as the plain one
+    R = K + 1
+    prefix = [4096 - 37 * s for s in range(B)]
+    qpos = np.stack([workloads.text_positions(int(p) + 1, R) for p in prefix])
+    cases = [workloads.verify_case(workloads.TARGET_LAYER, B=B, Hq=32, Hkv=8, D=128, prefix=prefix, K=K,
+                                   sections=(16, 24, 24), base=1e6, query_pos=qpos, cap=max(prefix) + R + 8,
+                                   layer=300 + l) for l in range(4)]
+    runs = []
+    for early in (False, True):
+        outs, state = [], [gpu_case(c) for c in cases]
+        for l, (q, k_new, v_new, pos, cache) in enumerate(state):
+            outs.append(sd.verify_layer(q, k_new, v_new, pos, cases[l].sections, cache, 0, 1e6,
+                                        early=early and l > 0))
+        torch.cuda.synchronize()
+        runs.append((outs, state))
+    (oa, sa), (ob, sb) = runs
+    for l in range(len(cases)):
+        assert torch.equal(oa[l], ob[l])
+        assert torch.equal(sa[l][4].k, sb[l][4].k) and torch.equal(sa[l][4].len, sb[l][4].len)
+        assert sb[l][4].len.cpu().tolist() == [p + R for p in prefix]
+    q, _, _, _, cache = sb[2]
+    _check_against_oracle(cases[2], q, cache, ob[2])
+    assert sd.get_device_error() == 0
+
+
 def test_fused_overflow_sets_error_and_leaves_scene():
     case = workloads.target_layer()
     q, k_new, v_new, pos, cache = gpu_case(case)
