@@ -11,7 +11,8 @@
 //     O^T[128 d][kR rows]   += V_tile^T[128 d][128 keys] . P^T     (MN-major A, B)
 // kR = 32 (G*R <= 32) or 64 (G*R <= 64, and m-blocks of 64 rows up to 128);
 // an N = 64 product costs about what an N = 32 one does. Both accumulators
-// live in tensor memory (S double-buffered): 3 kR columns.
+// live in tensor memory: S triple-buffered for 32 rows (4 kR columns), double-
+// buffered for 64 rows (3 kR columns).
 //
 // Warp roles in a CTA (352 threads). The issuing warps run converged: every
 // lane waits on the barriers and one elected lane issues (issued from a
@@ -21,7 +22,8 @@
 //               rows: 2), with a barrier each: a K slot refills once its S
 //               product is done, a V slot once its PV product is.
 //   warp 1      allocates tensor memory; issues S(t) once the softmax has read
-//               S(t - 2) and commits "S(t) ready".
+//               the buffer's previous S (S(t - 3) for 32 rows, S(t - 2) for 64)
+//               and commits "S(t) ready".
 //   warps 2..9  softmax: thread (t, h) owns key lane t of S^T and query rows
 //               h kR/2 .. h kR/2 + kR/2 - 1; P = exp2(S - ref) goes to shared
 //               memory as P^T (MN-major; 64-byte swizzle for 32 rows, 128-byte
@@ -95,15 +97,19 @@ struct Cfg {
   // P^T is MN-major: 64-byte swizzle for 32 rows (a 64-byte key row), 128-byte
   // swizzle for 64 rows; 8-key groups are kPRow * 8 bytes apart
   static constexpr uint64_t kPLayout = kR == 32 ? 4 : 2;
-  static constexpr int kTmemCols = kR == 32 ? 128 : 256;    // S0 | S1 | O, kR columns each
+  static constexpr int kTmemCols = kR == 32 ? 128 : 256;    // S0 | S1 (| S2) | O, kR columns each
   // shared memory layout (offsets from the 1024-aligned base)
   static constexpr int kOffQ = kRing;
   static constexpr int kOffP = kOffQ + kQ;                  // also the rotation table before the loop
   static constexpr int kOffNewK = kOffP + 2 * kP;
   static constexpr int kOffNewV = kOffNewK + kMaxNew * kNewRow;
   static constexpr int kOffBar = kOffNewV + kMaxNew * kNewRow;
-  // barriers: full_k[S] full_v[S] p_full[2] s_ready[S] pv_done[S] q_full recv decide
-  static constexpr int kNumBars = 4 * kStages + 5;
+  // S buffers in tensor memory: 3 for 32 rows (S0 | S1 | S2 | O fill the 128
+  // columns), 2 for 64 rows
+  static constexpr int kSBuf = kR == 32 ? 3 : 2;
+  // barriers: full_k[S] full_v[S] p_full[2] s_ready[S] pv_done[S] q_full recv
+  // decide s_free[3]
+  static constexpr int kNumBars = 4 * kStages + 8;
   // tmem slot, excess, decision, len (and, 64 rows, the last reader of the new key rows)
   static constexpr int kOffMisc = round_up(kOffBar + kNumBars * 8, 16);
   static constexpr int kOffRowA = kOffMisc + (kR == 32 ? 16 : 32);  // [kR] per-row results (reductions)
@@ -411,6 +417,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t QFULL = bar(4 * kS + 2);
   const uint32_t RECV = bar(4 * kS + 3);    // the cluster merge's incoming partial rows
   const uint32_t DECIDE = bar(4 * kS + 4);  // whether the range runs a second time
+  // 32 rows: the softmax has read S(T) (its tensor-memory buffer takes S(T + 3))
+  auto SFREE = [&](int T) { return bar(4 * kS + 5 + T % 3); };
+  constexpr int kSB = C::kSBuf;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::kOffMisc);
   int* s_excess = reinterpret_cast<int*>(smem + C::kOffMisc + 4);
   int* s_redo = reinterpret_cast<int*>(smem + C::kOffMisc + 8);
@@ -439,6 +448,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(QFULL, 1);  // one softmax thread, once the query tile is stored
     mbar_init(RECV, 1);
     mbar_init(DECIDE, 1);
+    for (int i = 0; i < 3; ++i) mbar_init(SFREE(i), kSoftWarps);
     *s_excess = 0;
     *s_redo = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -470,8 +480,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  const uint32_t tmem_s = tmem;          // S buffer b at column kR * b
-  const uint32_t tmem_o = tmem + 2 * kR; // O^T
+  const uint32_t tmem_s = tmem;            // S buffer b at column kR * b
+  const uint32_t tmem_o = tmem + kSB * kR; // O^T
 
   int n_keys, L_pre;
   bool valid;
@@ -593,14 +603,19 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         const int T0 = pass * n_tiles;
         for (int t = 0; t < n_tiles; ++t) {
-          // S(T) reuses the S buffer of tile T - 2: the softmax has read it
-          // once PFULL(T - 2) is out (pass 1 starts after all of pass 0)
+          // S(T) reuses the S buffer of tile T - kSB: the softmax has read it
+          // once SFREE(T - 3) (32 rows) or PFULL(T - 2) (64 rows) is out;
+          // pass 1 starts after all of pass 0
           const int T = T0 + t, st_ = T % kS;
-          if (t >= 2) mbar_wait(PFULL(T & 1), ((T - 2) >> 1) & 1);
+          if (kSB == 3) {
+            if (t >= 3) mbar_wait(SFREE(T), static_cast<uint32_t>(((T - 3) / 3) & 1));
+          } else {
+            if (t >= 2) mbar_wait(PFULL(T & 1), ((T - 2) >> 1) & 1);
+          }
           mbar_wait(FULLK(st_), ring_parity(T));
           tc_fence_after();
           const uint64_t dk = dK0 + static_cast<uint64_t>((st_ * kKV) >> 4);
-          const uint32_t ts = tmem_s + kR * (T & 1);
+          const uint32_t ts = tmem_s + kR * (T % kSB);
           if (elect_one()) {
 #pragma unroll
             for (int kk = 0; kk < 8; ++kk)
@@ -883,12 +898,18 @@ __global__ void __launch_bounds__(kThreads, 1)
         // P^T key row kl (its buffer's previous tile, T - 2, is done: see
         // above): kRpt rows = kRpt / 8 16-byte chunks of 8 query rows, swizzled
         const uint32_t prow = base + C::kOffP + bb * C::kP + kl * C::kPRow;
-        if (T >= 2) mbar_wait(PVDONE(T - 2), ring_parity(T - 2));  // PV(T - 2) has read P buffer bb
+        if (kSB == 2 && T >= 2) mbar_wait(PVDONE(T - 2), ring_parity(T - 2));  // PV(T - 2) has read P buffer bb
         const int sw = kR == 32 ? (kl >> 1) & 3 : kl & 7;
 #pragma unroll
         for (int j0 = 0; j0 < kRpt; j0 += 16) {
           uint32_t r[16];
-          tmem_ld16(tmem_s + kR * bb + row0 + j0 + lane_off, r);
+          tmem_ld16(tmem_s + kR * (T % kSB) + row0 + j0 + lane_off, r);
+          if (kSB == 3) {
+            // S(T) is in registers: its buffer may take S(T + 3)
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(SFREE(T));
+          }
           bool ok[16];
           tile_mask(key0, j0, ok);
           float rc[16];
@@ -920,6 +941,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             lp[j0 + j] += sd_bf16_lo(w);
             lp[j0 + j + 1] += sd_bf16_hi(w);
           }
+          if (kSB == 3 && T >= 2 && j0 == 0) mbar_wait(PVDONE(T - 2), ring_parity(T - 2));  // PV(T - 2) has read P buffer bb
           const int ch = (row0 + j0) >> 3;
           st_shared_v4(prow + ((ch ^ sw) << 4), pw[0], pw[1], pw[2], pw[3]);
           st_shared_v4(prow + (((ch + 1) ^ sw) << 4), pw[4], pw[5], pw[6], pw[7]);
