@@ -895,8 +895,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         mbar_wait(SREADY(T), ring_parity(T));  // S(T) is ready
         tc_fence_after();
         const bool key_ok = key < key_end;
-        // P^T key row kl (its buffer's previous tile, T - 2, is done: see
-        // above): kRpt rows = kRpt / 8 16-byte chunks of 8 query rows, swizzled
+        // P^T key row kl, once PV(T - 2) has read the buffer: kRpt rows =
+        // kRpt / 8 16-byte chunks of 8 query rows, swizzled
         const uint32_t prow = base + C::kOffP + bb * C::kP + kl * C::kPRow;
         if (kSB == 2 && T >= 2) mbar_wait(PVDONE(T - 2), ring_parity(T - 2));  // PV(T - 2) has read P buffer bb
         const int sw = kR == 32 ? (kl >> 1) & 3 : kl & 7;
