@@ -11,8 +11,7 @@
 //     O^T[128 d][kR rows]   += V_tile^T[128 d][128 keys] . P^T     (MN-major A, B)
 // kR = 32 (G*R <= 32) or 64 (G*R <= 64, and m-blocks of 64 rows up to 128);
 // an N = 64 product costs about what an N = 32 one does. Both accumulators
-// live in tensor memory: S triple-buffered for 32 rows (4 kR columns), double-
-// buffered for 64 rows (3 kR columns).
+// live in tensor memory, S triple-buffered: 4 kR columns.
 //
 // Warp roles in a CTA (352 threads). The issuing warps run converged: every
 // lane waits on the barriers and one elected lane issues (issued from a
@@ -22,8 +21,7 @@
 //               rows: 2), with a barrier each: a K slot refills once its S
 //               product is done, a V slot once its PV product is.
 //   warp 1      allocates tensor memory; issues S(t) once the softmax has read
-//               the buffer's previous S (S(t - 3) for 32 rows, S(t - 2) for 64)
-//               and commits "S(t) ready".
+//               the buffer's previous S, S(t - 3), and commits "S(t) ready".
 //   warps 2..9  softmax: thread (t, h) owns key lane t of S^T and query rows
 //               h kR/2 .. h kR/2 + kR/2 - 1; P = exp2(S - ref) goes to shared
 //               memory as P^T (MN-major; 64-byte swizzle for 32 rows, 128-byte
@@ -104,12 +102,12 @@ struct Cfg {
   static constexpr int kOffNewK = kOffP + 2 * kP;
   static constexpr int kOffNewV = kOffNewK + kMaxNew * kNewRow;
   static constexpr int kOffBar = kOffNewV + kMaxNew * kNewRow;
-  // S buffers in tensor memory: 3 for 32 rows (S0 | S1 | S2 | O fill the 128
-  // columns), 2 for 64 rows
-  static constexpr int kSBuf = kR == 32 ? 3 : 2;
-  // barriers: full_k[S] full_v[S] p_full[2] s_ready[S] pv_done[S] q_full recv
+  // three S buffers in tensor memory (S0 | S1 | S2 | O fill the 128 or 256
+  // columns)
+  static constexpr int kSBuf = 3;
+  // barriers: full_k[S] full_v[S] p_full[2] s_ready[3] pv_done[S] q_full recv
   // decide s_free[3]
-  static constexpr int kNumBars = 4 * kStages + 8;
+  static constexpr int kNumBars = 3 * kStages + 11;
   // tmem slot, excess, decision, len (and, 64 rows, the last reader of the new key rows)
   static constexpr int kOffMisc = round_up(kOffBar + kNumBars * 8, 16);
   static constexpr int kOffRowA = kOffMisc + (kR == 32 ? 16 : 32);  // [kR] per-row results (reductions)
@@ -411,14 +409,15 @@ __global__ void __launch_bounds__(kThreads, 1)
   auto FULLK = [&](int s) { return bar(s); };
   auto FULLV = [&](int s) { return bar(kS + s); };
   auto PFULL = [&](int b) { return bar(2 * kS + b); };
-  auto SREADY = [&](int T) { return bar(2 * kS + 2 + T % kS); };
-  auto PVDONE = [&](int T) { return bar(3 * kS + 2 + T % kS); };
+  auto SREADY = [&](int T) { return bar(2 * kS + 2 + T % 3); };  // one per S buffer
+  auto PVDONE = [&](int T) { return bar(2 * kS + 5 + T % kS); };
   auto ring_parity = [](int T) { return static_cast<uint32_t>((T / kS) & 1); };
-  const uint32_t QFULL = bar(4 * kS + 2);
-  const uint32_t RECV = bar(4 * kS + 3);    // the cluster merge's incoming partial rows
-  const uint32_t DECIDE = bar(4 * kS + 4);  // whether the range runs a second time
+  const uint32_t QFULL = bar(3 * kS + 5);
+  const uint32_t RECV = bar(3 * kS + 6);    // the cluster merge's incoming partial rows
+  const uint32_t DECIDE = bar(3 * kS + 7);  // whether the range runs a second time
   // 32 rows: the softmax has read S(T) (its tensor-memory buffer takes S(T + 3))
-  auto SFREE = [&](int T) { return bar(4 * kS + 5 + T % 3); };
+  auto SFREE = [&](int T) { return bar(3 * kS + 8 + T % 3); };
+  auto s_parity = [](int T) { return static_cast<uint32_t>((T / 3) & 1); };  // SREADY, SFREE phases
   constexpr int kSB = C::kSBuf;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::kOffMisc);
   int* s_excess = reinterpret_cast<int*>(smem + C::kOffMisc + 4);
@@ -441,9 +440,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int s = 0; s < kS; ++s) {
       mbar_init(FULLK(s), 1);
       mbar_init(FULLV(s), 1);
-      mbar_init(SREADY(s), 1);
       mbar_init(PVDONE(s), 1);
     }
+    for (int i = 0; i < 3; ++i) mbar_init(SREADY(i), 1);
     for (int i = 0; i < 2; ++i) mbar_init(PFULL(i), kSoftWarps);
     mbar_init(QFULL, 1);  // one softmax thread, once the query tile is stored
     mbar_init(RECV, 1);
@@ -552,7 +551,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           const int y0 = key_begin + t * kStageKeys;
           // slot s last held tile T - kS (all of pass 0 is done before pass 1)
           const uint32_t kst = base + s * kKV, vst = base + C::kRingV + s * kKV;
-          if (t >= kS) mbar_wait(SREADY(T - kS), ring_parity(T - kS));
+          if (t >= kS) mbar_wait(SREADY(T - kS), s_parity(T - kS));
           if (elect_one()) {
             mbar_expect_tx(FULLK(s), static_cast<uint32_t>(kKV));
 #pragma unroll
@@ -603,15 +602,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         const int T0 = pass * n_tiles;
         for (int t = 0; t < n_tiles; ++t) {
-          // S(T) reuses the S buffer of tile T - kSB: the softmax has read it
-          // once SFREE(T - 3) (32 rows) or PFULL(T - 2) (64 rows) is out;
-          // pass 1 starts after all of pass 0
+          // S(T) reuses the S buffer of tile T - 3: the softmax has read it
+          // once SFREE(T - 3) is out; pass 1 starts after all of pass 0
           const int T = T0 + t, st_ = T % kS;
-          if (kSB == 3) {
-            if (t >= 3) mbar_wait(SFREE(T), static_cast<uint32_t>(((T - 3) / 3) & 1));
-          } else {
-            if (t >= 2) mbar_wait(PFULL(T & 1), ((T - 2) >> 1) & 1);
-          }
+          if (t >= 3) mbar_wait(SFREE(T), s_parity(T - 3));
           mbar_wait(FULLK(st_), ring_parity(T));
           tc_fence_after();
           const uint64_t dk = dK0 + static_cast<uint64_t>((st_ * kKV) >> 4);
@@ -892,20 +886,19 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int bb = T & 1, s = T % kS;
         const int key0 = key_begin + t * kStageKeys;
         const int key = key0 + kl;
-        mbar_wait(SREADY(T), ring_parity(T));  // S(T) is ready
+        mbar_wait(SREADY(T), s_parity(T));  // S(T) is ready
         tc_fence_after();
         const bool key_ok = key < key_end;
         // P^T key row kl, once PV(T - 2) has read the buffer: kRpt rows =
         // kRpt / 8 16-byte chunks of 8 query rows, swizzled
         const uint32_t prow = base + C::kOffP + bb * C::kP + kl * C::kPRow;
-        if (kSB == 2 && T >= 2) mbar_wait(PVDONE(T - 2), ring_parity(T - 2));  // PV(T - 2) has read P buffer bb
         const int sw = kR == 32 ? (kl >> 1) & 3 : kl & 7;
 #pragma unroll
         for (int j0 = 0; j0 < kRpt; j0 += 16) {
           uint32_t r[16];
           tmem_ld16(tmem_s + kR * (T % kSB) + row0 + j0 + lane_off, r);
-          if (kSB == 3) {
-            // S(T) is in registers: its buffer may take S(T + 3)
+          if (j0 + 16 >= kRpt) {
+            // S(T) is in registers (its last 16 rows): its buffer may take S(T + 3)
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(SFREE(T));
@@ -941,7 +934,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             lp[j0 + j] += sd_bf16_lo(w);
             lp[j0 + j + 1] += sd_bf16_hi(w);
           }
-          if (kSB == 3 && T >= 2 && j0 == 0) mbar_wait(PVDONE(T - 2), ring_parity(T - 2));  // PV(T - 2) has read P buffer bb
+          if (T >= 2 && j0 == 0) mbar_wait(PVDONE(T - 2), ring_parity(T - 2));  // PV(T - 2) has read P buffer bb
           const int ch = (row0 + j0) >> 3;
           st_shared_v4(prow + ((ch ^ sw) << 4), pw[0], pw[1], pw[2], pw[3]);
           st_shared_v4(prow + (((ch + 1) ^ sw) << 4), pw[4], pw[5], pw[6], pw[7]);
