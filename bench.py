@@ -622,6 +622,23 @@ def main():
     ms_attn_launch = time_graph(g_attn, reps) / LAYERS
     st.lens.copy_(st.lens0)
     torch.cuda.synchronize()
+    # ---- the small kernels of the path, per call: M-RoPE of one layer's rows,
+    #      the rollback of all 36 lengths (committed = R: lengths unchanged), and
+    #      one layer's append (timed with a rollback of the same R rows that puts
+    #      its length back; the rollback alone is subtracted)
+    full = torch.full((1,), R, dtype=torch.int32, device=device)
+    zero = torch.zeros(1, dtype=torch.int32, device=device)
+    g_rope = capture(lambda: [sd.rope_apply(st.q[l], st.k[l], st.pos, SECTIONS, 0, BASE) for l in range(LAYERS)])
+    g_rb = capture(lambda: [sd.kv_rollback(st.lens, full, R) for _ in range(LAYERS)])
+    g_ap = capture(lambda: [(sd.kv_append(st.caches[l], st.k[l], st.v[l]), sd.kv_rollback(st.lens[l], zero, R))
+                            for l in range(LAYERS)])
+    ms_rope = time_graph(g_rope, reps) / LAYERS
+    ms_rollback = time_graph(g_rb, reps) / LAYERS
+    ms_append = time_graph(g_ap, reps) / LAYERS - ms_rollback
+    st.d_in.copy_(st.h_in)  # the rotations above changed the q / k rows in place
+    st.lens.copy_(st.lens0)
+    torch.cuda.synchronize()
+    assert sd.get_device_error() == 0
 
     # ---- end to end: pinned host inputs -> device, step, result -> host
     e2e_steps = max(10, min(500, args.steps))
@@ -685,6 +702,9 @@ def main():
         "layer_us": round(ms_layer_launch * 1e3, 3),
         "attention_us": round(ms_attn_launch * 1e3, 3),
         "unfused_verify_step_us": round(ms_unfused * 1e3, 3),
+        "rope_us": round(ms_rope * 1e3, 3),
+        "kv_append_us": round(ms_append * 1e3, 3),
+        "kv_rollback_us": round(ms_rollback * 1e3, 3),
         "accept_us": round(ms_accept * 1e3, 3),
         "sample_accept_us": round(sample_us, 3),
         "sample_accept_gbs": round(sample_bytes / (sample_us * 1e-6) / 1e9, 1),
