@@ -78,5 +78,15 @@ def test_reference_arm_prints_on_rank_zero_only(rank):
         assert len(lines) == 1
         line = json.loads(lines[0])
         assert line["impl"] == "reference" and line["n_gpus"] == 2
+        # the line a bench arm prints: same metric and unit as ours, the oracle
+        # described as the cpu baseline, an e2e object with no host copies
+        for key in ("metric", "value", "unit", "steps", "warmup", "ms_per_step", "higher_is_better",
+                    "scaling", "dtype", "data", "config", "cpu_baseline", "e2e"):
+            assert key in line, key
+        assert line["unit"] == "GB/s" and line["higher_is_better"] is True and line["warmup"] >= 3
+        assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["cores"] >= 1
+        assert line["cpu_baseline"]["value"] == line["value"] and line["cpu_baseline"]["sample"]
+        assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["e2e"]["d2h_bytes_per_step"] == 0
+        assert line["e2e"]["value"] == line["value"] and line["e2e"]["unit"] == line["unit"]
     else:
         assert lines == []
