@@ -383,6 +383,41 @@ def time_draft_steps(device, reps=20):
     return ms * 1e3 / steps
 
 
+def time_tiny_step(device, reps=200):
+    """The tiny verify step (B = 1, 4 q / 1 KV head, head_dim 64, L = 256 = 192
+    vision patches + 64 text tokens, K = 4, M-RoPE sections [8,12,12]): one
+    sd_verify_layer call (head_dim 64 runs M-RoPE, append and attention as three
+    kernels), the greedy accept over fp32 logits [1][5][4096] and the rollback,
+    then the length put back, in a graph of `reps` steps. A latency figure: the
+    step moves ~0.1 MB. Returns us per step."""
+    from paper_2606_31160_gb300 import sd, workloads
+    case = workloads.tiny()
+    R_ = case.R
+    q, k, v, pos = (x.to(device) for x in (case.q, case.k_new, case.v_new, case.pos))
+    lens = torch.from_numpy(case.prefix.astype(np.int32)).to(device)
+    lens0 = lens.clone()
+    cache = sd.KVCache(case.k_cache.to(device), case.v_cache.to(device), lens)
+    logits, draft = case.extra["logits"].to(device), case.extra["draft"].to(device)
+    ws = sd.workspace(sd.greedy_workspace_bytes(1, R_ - 1, logits.shape[-1]), device)
+    ws_l = sd.workspace(sd.layer_workspace_bytes(1, R_, case.Hq, case.Hkv, case.D, case.cap), device)
+    out = torch.empty_like(q)
+    n_emit = torch.zeros(1, dtype=torch.int32, device=device)
+    tokens = torch.zeros((1, R_), dtype=torch.int32, device=device)
+    argmax = torch.zeros((1, R_), dtype=torch.int32, device=device)
+
+    def steps():
+        for _ in range(reps):
+            sd.verify_layer(q, k, v, pos, case.sections, cache, case.interleaved, case.base, out=out, ws=ws_l)
+            sd.accept_greedy(logits, draft, ws=ws, n_emit=n_emit, tokens=tokens, argmax=argmax)
+            sd.kv_rollback(lens, n_emit, R_)
+            lens.copy_(lens0, non_blocking=True)
+
+    g = capture(steps)
+    ms = time_graph(g, 5)
+    assert sd.get_device_error() == 0
+    return ms * 1e3 / reps
+
+
 def time_stochastic_step(device, layers=LAYERS):
     """The stochastic-acceptance step: 36 fused target layers at B = 8 (L = 4096,
     R = 8, 32 q / 8 KV x 128, one cache per layer: 4.84 GB streamed from HBM),
@@ -507,13 +542,16 @@ def oracle_layer_sample(case, logits, draft):
     return layer_bytes(1) + (step_bytes(1) - LAYERS * layer_bytes(1))
 
 
-def cpu_threads():
+def host_cores():
+    """Cores this process may run on (its affinity mask)."""
     try:
-        from threadpoolctl import threadpool_info
-        n = max((i.get("num_threads", 1) for i in threadpool_info()), default=1)
-        return int(n)
-    except Exception:
         return len(os.sched_getaffinity(0))
+    except Exception:
+        return os.cpu_count() or 1
+
+
+THREAD_VARS = ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS", "BLIS_NUM_THREADS",
+               "NUMEXPR_NUM_THREADS", "VECLIB_MAXIMUM_THREADS")
 
 
 def time_oracle(budget_s, max_layers=None):
@@ -532,6 +570,35 @@ def time_oracle(budget_s, max_layers=None):
     return done_bytes / el / 1e9, n, el
 
 
+def time_oracle_threads(budget_s, threads):
+    """The oracle leg in a fresh interpreter whose BLAS / OpenMP pools are capped
+    at `threads` (the variables must be set before numpy loads, hence a child
+    process). Returns (GB/s, layers, seconds)."""
+    env = dict(os.environ)
+    for v in THREAD_VARS:
+        env[v] = str(threads)
+    out = subprocess.run([sys.executable, os.path.abspath(__file__), "--oracle-leg", "--cpu-budget", str(budget_s)],
+                         env=env, capture_output=True, text=True, timeout=budget_s * 4 + 300)
+    if out.returncode != 0:
+        raise RuntimeError("oracle leg failed:\n" + out.stderr[-2000:])
+    d = json.loads(out.stdout.strip().splitlines()[-1])
+    return d["gbs"], d["layers"], d["seconds"]
+
+
+def oracle_leg(args):
+    """Child-process entry of time_oracle_threads: one JSON line."""
+    gbs, n, el = time_oracle(args.cpu_budget)
+    print(json.dumps({"gbs": gbs, "layers": n, "seconds": el}), flush=True)
+
+
+def cpu_baseline_pair(budget_s):
+    """The oracle timed at 1 thread and at every core of the affinity mask."""
+    cores = host_cores()
+    one = time_oracle_threads(budget_s, 1)
+    every = time_oracle_threads(budget_s, cores)
+    return cores, one, every
+
+
 # ------------------------------------------------------------------ main
 def main():
     ap = argparse.ArgumentParser()
@@ -539,7 +606,9 @@ def main():
     ap.add_argument("--steps", type=int, default=2000)
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--cpu-budget", type=float, default=12.0, help="seconds of oracle time (rank 0)")
+    ap.add_argument("--cpu-budget", type=float, default=10.0,
+                    help="seconds of oracle time per leg (rank 0; two legs: 1 thread, all cores)")
+    ap.add_argument("--oracle-leg", action="store_true", help=argparse.SUPPRESS)
     ap.add_argument("--sweep", action="store_true",
                     help="time sd_verify_attention over the batched sweep grid (B x L x K) and "
                          "print one JSON line per point; prints no bench line")
@@ -555,6 +624,8 @@ def main():
     if args.warmup < 3:
         args.warmup = 3
 
+    if args.oracle_leg:
+        return oracle_leg(args)
     if args.impl == "reference":
         return reference_arm(args, world, rank)
     if args.only:
@@ -659,6 +730,7 @@ def main():
     # its whole step (36 layers at B = 8 + sampling), and the draft's propose loop
     sample_us, sample_bytes = time_sample_accept(device) if rank == 0 else (None, None)
     draft_us = time_draft_steps(device) if rank == 0 else None
+    tiny_us = time_tiny_step(device) if rank == 0 else None
     stoch_us, stoch_bytes = time_stochastic_step(device) if rank == 0 else (None, None)
     long_us, long_bytes = time_long_draft_step(device) if rank == 0 else (None, None)
     assert sd.get_device_error() == 0
@@ -673,7 +745,7 @@ def main():
     value = aggregate_gbs(step_bytes(1), world, ms_step)
     achieved = layer_bytes(1) / (ms_layer_launch * 1e-3) / 1e9
     traffic = ncu_traffic()
-    cpu_gbs, cpu_layers, cpu_s = time_oracle(args.cpu_budget)
+    cores, (one_gbs, one_layers, one_s), (all_gbs, all_layers, all_s) = cpu_baseline_pair(args.cpu_budget)
     line = {
         "metric": METRIC,
         "value": round(value, 2),
@@ -709,6 +781,7 @@ def main():
         "sample_accept_us": round(sample_us, 3),
         "sample_accept_gbs": round(sample_bytes / (sample_us * 1e-6) / 1e9, 1),
         "draft_step_us": round(draft_us, 3),
+        "tiny_step_us": round(tiny_us, 3),
         "stochastic_step_us": round(stoch_us, 2),
         "stochastic_step_gbs": round(stoch_bytes / (stoch_us * 1e-6) / 1e9, 1),
         "block_draft_step_us": round(long_us, 2),
@@ -727,13 +800,15 @@ def main():
             "timing": "36 chained launches of the layer kernel in one graph; average = total / 36",
         },
         "cpu_baseline": {
-            "value": round(cpu_gbs, 4),
+            "value": round(all_gbs, 4),
             "unit": "GB/s",
-            "cores": cpu_threads(),
+            "cores": cores,
             "kind": "oracle",
             "sample": "%d full target layers (M-RoPE, append, attention over 4104 keys, all 32 heads) each "
-                      "with the greedy accept over 8 x 151936 and the rollback, float64 numpy, %.1f s"
-                      % (cpu_layers, cpu_s),
+                      "with the greedy accept over 8 x 151936 and the rollback, float64 numpy, %.1f s, BLAS and "
+                      "OpenMP pools at %d threads (the affinity mask)" % (all_layers, all_s, cores),
+            "one_thread": {"value": round(one_gbs, 4), "unit": "GB/s", "cores": 1,
+                           "sample": "%d layers in %.1f s, every pool at 1 thread" % (one_layers, one_s)},
         },
         "e2e": {
             "value": round(aggregate_gbs(step_bytes(1), world, ms_e2e), 2),
@@ -881,8 +956,9 @@ def reference_arm(args, world, rank):
         "config": {"workload": "8B-class target verify step, one layer per step (sample): M-RoPE + append + "
                                "attention L=4096 K=7 32q/8kv x 128 + greedy accept V=151936 + rollback",
                    "parallelism": "host cores"},
-        "cpu_baseline": {"value": round(value, 4), "unit": "GB/s", "cores": cpu_threads(), "kind": "oracle",
-                         "sample": "one target layer + acceptance per step, %d steps" % steps},
+        "cpu_baseline": {"value": round(value, 4), "unit": "GB/s", "cores": host_cores(), "kind": "oracle",
+                         "sample": "one target layer + acceptance per step, %d steps, numpy's default "
+                                   "BLAS pool over the affinity mask" % steps},
         "e2e": {"value": round(value, 4), "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)

@@ -161,6 +161,11 @@ size_t sd_verify_attention_workspace(int B, int R, int Hq, int Hkv, int D, int c
  * SD_DEVERR_LENGTH and its output is left unwritten. The first call per
  * device and shape should come before any stream capture (it sets kernel
  * attributes and queries the occupancy).
+ * Kernel choice is by shape: head_dim 128 with G*R <= 128 takes the tcgen05
+ * kernel, every other shape the mma.sync kernel. A test-only override exists:
+ * the environment variable SD_ATTENTION_KERNEL=mma, read once per process,
+ * sends every shape to the mma.sync kernel so that tests can compare the two
+ * kernels on the same inputs; production callers leave it unset.
  */
 sd_status sd_verify_attention(const void* q, const sd_kv_cache* cache, void* out,
                               int R, int Hq, float scale, void* workspace, size_t ws_bytes,

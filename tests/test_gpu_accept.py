@@ -1,12 +1,13 @@
 """GPU parity of sd_accept_greedy and sd_accept_sample against the float64 oracle.
 
 Greedy: n_emit, tokens and argmax bit-exact. Sampling: bit-exact on every
-scene whose decisions all sit clear of their boundary in the oracle's float64
-arithmetic -- acceptance tests farther than ACCEPT_MARGIN (relative) and the
-final draw farther than DRAW_MARGIN (probability units) from a step of the
-cumulative sum; these bounds sit well above the fp32 error of the kernel's
-normalisers (~1e-6 relative) and running sums (~1e-6 absolute).
-Near-boundary scenes are counted and must be rare.
+decision that sits clear of its boundary in the oracle's float64 arithmetic
+-- acceptance tests farther than ACCEPT_MARGIN (relative) and the final draw
+farther than DRAW_MARGIN (probability units) from a step of the cumulative
+sum; these bounds sit well above the fp32 error of the kernel's normalisers
+(~1e-6 relative) and running sums (~1e-6 absolute). A near decision leaves
+open only what depends on it: the accepted length and prefix before it are
+still checked. Near decisions are counted per seed.
 """
 import numpy as np
 import pytest
@@ -101,31 +102,59 @@ def test_greedy_draft_out_of_range_sets_error():
 # ------------------------------------------------------------------ sampling
 
 def _sample_both(z_t, z_d, draft, u, T):
+    """Kernel against oracle, every decision that the oracle's float64 margins
+    decide. Acceptance tests are taken in order; when test j sits within
+    ACCEPT_MARGIN of its boundary the tests before it were clear accepts, so
+    the kernel must have accepted drafts 0..j-1 (n_emit > j, tokens[:j] equal)
+    and only what follows test j is left open. When every acceptance test is
+    clear, n_emit and the accepted prefix are exact, and the drawn token is too
+    unless the draw sits within DRAW_MARGIN of a step of its cumulative sum.
+    Returns (oracle n_emit, scenes with a near acceptance test, scenes whose
+    only near decision is the final draw)."""
     n, t = sd.accept_sample(z_t.cuda(), z_d.cuda(), draft.cuda(), u.cuda(), T)
     rn, rt, margins = oracle.accept_sample(z_t.numpy(), z_d.numpy(), draft.numpy(), u.numpy(), T)
     n, t = n.cpu().numpy(), t.cpu().numpy()
-    near = [b for b in range(len(rn))
-            if min(margins[b][:-1], default=1.0) < ACCEPT_MARGIN or margins[b][-1] < DRAW_MARGIN]
+    V = z_t.shape[-1]
+    accept_near, draw_near = [], []
     for b in range(len(rn)):
-        if b in near:
+        acc_m, draw_m = margins[b][:-1], margins[b][-1]
+        assert 1 <= n[b] <= t.shape[1] and (t[b][n[b]:] == -1).all(), (b, n[b], t[b])
+        j_near = next((j for j, m in enumerate(acc_m) if m < ACCEPT_MARGIN), None)
+        if j_near is not None:
+            accept_near.append(b)
+            assert n[b] >= j_near + 1, (b, n[b], j_near)
+            assert t[b][:j_near].tolist() == rt[b][:j_near].tolist(), (b, t[b], rt[b])
             continue
         assert n[b] == rn[b], (b, n[b], rn[b])
-        assert t[b].tolist() == rt[b].tolist(), (b, t[b], rt[b])
-    return rn, near
+        assert t[b][:rn[b] - 1].tolist() == rt[b][:rn[b] - 1].tolist(), (b, t[b], rt[b])
+        if draw_m < DRAW_MARGIN:
+            draw_near.append(b)
+            assert 0 <= t[b][rn[b] - 1] < V
+        else:
+            assert t[b][rn[b] - 1] == rt[b][rn[b] - 1], (b, t[b], rt[b])
+    return rn, accept_near, draw_near
 
 
 def test_sample_stochastic_workload():
     w = workloads.stochastic()
-    rn, near = _sample_both(w["z_target"], w["z_draft"], w["draft"], w["u"], w["temperature"])
-    assert len(near) == 0
+    rn, accept_near, draw_near = _sample_both(w["z_target"], w["z_draft"], w["draft"], w["u"], w["temperature"])
+    assert accept_near == [] and draw_near == []
     assert rn.min() >= 1 and rn.max() <= w["K"] + 1
+
+
+# scenes (of 16) whose final draw the oracle puts within DRAW_MARGIN of a step
+# of its cumulative sum, per seed: only their drawn token goes unchecked
+DRAW_NEAR_PER_SEED = (0, 0, 1, 2)
 
 
 @pytest.mark.parametrize("seed", range(4))
 def test_sample_more_seeds(seed):
+    # flatter T = 0.8 rows over 50k tokens: smaller steps in the cumulative sums
     w = workloads.stochastic(B=16, K=5, V=50000, temperature=0.8, seed_layer=10 + seed)
-    rn, near = _sample_both(w["z_target"], w["z_draft"], w["draft"], w["u"], w["temperature"])
-    assert len(near) <= 4   # flatter T = 0.8 rows over 50k tokens have small CDF steps
+    rn, accept_near, draw_near = _sample_both(w["z_target"], w["z_draft"], w["draft"], w["u"], w["temperature"])
+    print("seed %d: near acceptance tests %s, near final draws %s" % (seed, accept_near, draw_near))
+    assert accept_near == []
+    assert len(draw_near) == DRAW_NEAR_PER_SEED[seed]
 
 
 def test_sample_equal_distributions_always_accept():

@@ -154,3 +154,37 @@ def test_fused_layer_long_drafts(K):
     _check_against_oracle(case, qb, cb, ob)
     assert (ob.float() - oa.float()).abs().max().item() <= 2 * ATTN_ATOL
     assert sd.get_device_error() == 0
+
+
+@pytest.mark.parametrize("K", [7, 8, 16])
+def test_fused_layer_interleaved_mrope(K):
+    # interleaved axis assignment a(d) = (T, H, W)[d mod 3] (Sec. 3.2 Eq.
+    # axis-assign) through the fused kernel's own rotation table, on the
+    # 32-row tile (K = 7), the 64-row tile (K = 8) and two 64-row m-blocks
+    # (K = 16); query rows at distinct (t, h, w) so that the layout matters
+    R = K + 1
+    prefix = [3000, 4096]
+    rng = np.random.default_rng(900 + K)
+    qpos = rng.integers(0, 5000, size=(2, R, 3)).astype(np.int32)
+    case = workloads.verify_case(workloads.TARGET_LAYER, B=2, Hq=32, Hkv=8, D=128, prefix=prefix, K=K,
+                                 sections=(16, 24, 24), base=1e6, query_pos=qpos, cap=max(prefix) + R + 8,
+                                 interleaved=1, layer=500 + K, tail_fill=float("nan"))
+    qa, ka, ca, oa = _unfused(case)
+    qb, kb, cb, ob = _fused(case)
+
+    def same(x, y):  # stale cache rows hold NaN on both sides
+        return bool(((x == y) | (x.isnan() & y.isnan())).all())
+
+    assert torch.equal(qa, qb) and torch.equal(ka, kb)
+    assert same(ca.k, cb.k) and same(ca.v, cb.v) and torch.equal(ca.len, cb.len)
+    pos = case.pos.numpy()[:, :, None, :]
+    ref_k = oracle.mrope_apply(to64(case.k_new), pos, case.sections, 1, case.base)
+    assert np.all(np.abs(to64(kb) - ref_k) <= rope_bound(ref_k, pair_magnitude(to64(case.k_new))))
+    for b, p in enumerate(prefix):   # the appended rows are the rotated keys and the values
+        assert torch.equal(cb.k[b, :, p:p + R].transpose(0, 1).cpu(), kb[b].cpu())
+        assert torch.equal(cb.v[b, :, p:p + R].transpose(0, 1).cpu(), case.v_new[b])
+    _check_against_oracle(case, qb, cb, ob)
+    # the blocked layout rotates these rows differently: the test sees the layout
+    ref_blocked = oracle.mrope_apply(to64(case.q), pos, case.sections, 0, case.base)
+    assert np.abs(to64(qb) - ref_blocked).max() > 0.1
+    assert sd.get_device_error() == 0
