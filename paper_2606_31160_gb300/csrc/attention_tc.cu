@@ -71,8 +71,11 @@ constexpr int kPvWarp = 2 + kSoftWarps;        // the warp after the softmax war
 constexpr int kThreads = 96 + kSoftThreads;
 constexpr uint32_t kSpinLimit = 1u << 20;
 constexpr float kSlack = 64.f;              // log2 units a score may exceed its reference by
-// a merged partial row is [O(128) | m | l | 2 pad] fp32 = 528 bytes
-constexpr int kRowF = kD + 4;
+// a partial row sent to its owner is [O(128) | l by TMEM lane quarter (4) | m |
+// 3 pad] fp32 = 544 bytes (16-byte multiple: one bulk copy per peer)
+constexpr int kRowF = kD + 8;
+constexpr int kRowL = kD;       // the four l terms (float4)
+constexpr int kRowM = kD + 4;   // the row's reference m
 constexpr int kRowBytes = kRowF * 4;
 constexpr int round_up(int x, int m) { return (x + m - 1) / m * m; }
 
@@ -95,10 +98,19 @@ struct Cfg {
   // P^T is MN-major: 64-byte swizzle for 32 rows (a 64-byte key row), 128-byte
   // swizzle for 64 rows; 8-key groups are kPRow * 8 bytes apart
   static constexpr uint64_t kPLayout = kR == 32 ? 4 : 2;
-  static constexpr int kTmemCols = kR == 32 ? 128 : 256;    // S0 | S1 (| S2) | O, kR columns each
+  static constexpr int kTmemCols = kR == 32 ? 128 : 256;    // S0 | S1 | S2 | O, kR columns each
+  // fused layer: one more kR-column buffer after O for S_new = K_new Q^T
+  static constexpr int kTmemColsFused = 2 * kTmemCols;
   // shared memory layout (offsets from the 1024-aligned base)
   static constexpr int kOffQ = kRing;
-  static constexpr int kOffP = kOffQ + kQ;                  // also the rotation table before the loop
+  // P^T buffers. Fused layer: before the tiles the first one holds the rotated
+  // new keys as a K-major, 128-byte-swizzled S_new operand (rows 0..kMaxNew-1
+  // of each 64-column half, halves kNewHalf apart; the MMA reads 128 rows, the
+  // rest is whatever follows and only fills score lanes that are never read),
+  // and the second one the rotation table
+  static constexpr int kOffP = kOffQ + kQ;
+  static constexpr int kNewHalf = kMaxNew * 128;
+  static constexpr int kOffTab = kOffP + kP;
   static constexpr int kOffNewK = kOffP + 2 * kP;
   static constexpr int kOffNewV = kOffNewK + kMaxNew * kNewRow;
   static constexpr int kOffBar = kOffNewV + kMaxNew * kNewRow;
@@ -106,26 +118,28 @@ struct Cfg {
   // columns)
   static constexpr int kSBuf = 3;
   // barriers: full_k[S] full_v[S] p_full[2] s_ready[3] pv_done[S] q_full recv
-  // decide s_free[3]
-  static constexpr int kNumBars = 3 * kStages + 11;
-  // tmem slot, excess, decision, len (and, 64 rows, the last reader of the new key rows)
+  // decide s_free[3] s_new
+  static constexpr int kNumBars = 3 * kStages + 12;
+  // tmem slot, (unused), decision, len (and, 64 rows, the last reader of the new key rows)
   static constexpr int kOffMisc = round_up(kOffBar + kNumBars * 8, 16);
   static constexpr int kOffRowA = kOffMisc + (kR == 32 ? 16 : 32);  // [kR] per-row results (reductions)
   static constexpr int kOffRef = kOffRowA + kR * 4;         // [kR] per-row references
   static constexpr int kOffLim = kOffRef + kR * 4;          // [kR] per-row causal key limits
   static constexpr int kSmemBytes = kOffLim + kR * 4 + 1024;
+  static_assert(kOffP + kNewHalf + 128 * 128 <= kSmemBytes - 1024, "the S_new operand's 128 rows stay inside");
   static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
   static_assert(kOffQ % 1024 == 0 && kOffP % 1024 == 0 && kP % 1024 == 0 && kOffNewK % 16 == 0 &&
                     kOffNewV % 16 == 0 && kOffBar % 8 == 0 && kOffRowA % 16 == 0 && kOffRef % 16 == 0,
                 "alignment of the shared-memory regions (swizzle atoms, vector accesses, mbarriers)");
-  static_assert(kMaxNew * 64 * 8 <= 2 * kP, "rotation table fits the P buffers");
+  static_assert(kMaxNew * 64 * 8 <= kP, "rotation table fits the second P buffer");
+  static_assert(kP >= 2 * kNewHalf && kOffP % 1024 == 0, "new-key operand fits the first P buffer");
   static_assert(kR * 128 * 4 <= 2 * kP, "row reductions fit the P buffers");
   // cluster merge buffers (in the rings, free once this CTA's last MMA is done)
   static constexpr int kSend = 0;                           // this CTA's kR rows
   static constexpr int kRecv = round_up(kR * kRowBytes, 1024);
   // slots for ceil(kR / c) rows from each of c ranks, c in {1, 2, 4, 6, 8, 16}
   static constexpr int kRecvSlots = kR == 32 ? 36 : 66;
-  static constexpr int kNewS = round_up(kRecv + kRecvSlots * kRowBytes, 1024);  // new-key scores
+  static constexpr int kNewS = round_up(kRecv + kRecvSlots * kRowBytes, 1024);  // new-key scores [rows][R]
   static_assert(kNewS + kR * kMaxNew * 4 <= kRing, "merge buffers");
 };
 
@@ -195,8 +209,51 @@ __device__ __forceinline__ uint32_t cvt_bf16x2(float lo, float hi) {
 __device__ __forceinline__ void named_bar_sync(int id, int threads) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(threads) : "memory");
 }
+// bar.sync over `threads` threads that also ORs a predicate across them
+__device__ __forceinline__ bool named_bar_or(int id, int threads, bool p) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred pi, po;\n\tsetp.ne.u32 pi, %1, 0;\n\t"
+      "bar.red.or.pred po, %2, %3, pi;\n\tselp.u32 %0, 1, 0, po;\n\t}"
+      : "=r"(r)
+      : "r"(static_cast<uint32_t>(p)), "r"(id), "r"(threads)
+      : "memory");
+  return r != 0;
+}
+// Sum over the 32 lanes of a warp of each of kN per-lane values (kN = 16 or
+// 32), by a butterfly reduce-scatter: at the step of stride s a lane keeps the
+// half of its values selected by its bit s and adds its partner's copy of that
+// half. Lane L ends with the sum of value `row` (kN = 16: lanes L and L ^ 1
+// hold the same value).
+template <int kN>
+__device__ __forceinline__ float warp_rows_sum(const float (&v0)[kN], int lane, int& row) {
+  static_assert(kN == 16 || kN == 32, "rows per thread");
+  float v[kN];
+#pragma unroll
+  for (int i = 0; i < kN; ++i) v[i] = v0[i];
+  int r = 0;
+#pragma unroll
+  for (int n = kN, s = 16; n > 1; n >>= 1, s >>= 1) {
+    const bool hi = (lane & s) != 0;
+#pragma unroll
+    for (int i = 0; i < n / 2; ++i) {
+      const float keep = hi ? v[i + n / 2] : v[i];
+      const float give = hi ? v[i] : v[i + n / 2];
+      v[i] = keep + __shfl_xor_sync(0xffffffffu, give, s);
+    }
+    if (hi) r += n / 2;
+  }
+  float x = v[0];
+  if (kN == 16) x += __shfl_xor_sync(0xffffffffu, x, 1);
+  row = r;
+  return x;
+}
 __device__ __forceinline__ void cluster_arrive() {
   asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+}
+// an arrival that orders nothing: no data passes through the barrier
+__device__ __forceinline__ void cluster_arrive_relaxed() {
+  asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
 }
 __device__ __forceinline__ void cluster_wait() {
   asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
@@ -391,6 +448,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   constexpr int kRpt = C::kRpt;
   constexpr uint32_t kIdescS = umma_idesc(128, kR, 0, 0);
   constexpr uint32_t kIdescO = umma_idesc(128, kR, 1, 1);
+  constexpr int kTmemAlloc = kFused ? C::kTmemColsFused : C::kTmemCols;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
@@ -418,9 +476,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   // 32 rows: the softmax has read S(T) (its tensor-memory buffer takes S(T + 3))
   auto SFREE = [&](int T) { return bar(3 * kS + 8 + T % 3); };
   auto s_parity = [](int T) { return static_cast<uint32_t>((T / 3) & 1); };  // SREADY, SFREE phases
+  const uint32_t SNEW = bar(3 * kS + 11);  // fused layer: S_new = K_new Q^T is in tensor memory
   constexpr int kSB = C::kSBuf;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::kOffMisc);
-  int* s_excess = reinterpret_cast<int*>(smem + C::kOffMisc + 4);
   int* s_redo = reinterpret_cast<int*>(smem + C::kOffMisc + 8);
   int* s_kvlast = reinterpret_cast<int*>(smem + C::kOffMisc + 16);  // 64 rows only
   float* row_a = reinterpret_cast<float*>(smem + C::kOffRowA);  // [kR] reduction results
@@ -448,14 +506,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(RECV, 1);
     mbar_init(DECIDE, 1);
     for (int i = 0; i < 3; ++i) mbar_init(SFREE(i), kSoftWarps);
-    *s_excess = 0;
+    mbar_init(SNEW, 1);
     *s_redo = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (warp == 1) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
                      smem_addr(tmem_slot)),
-                 "r"(C::kTmemCols)
+                 "r"(kTmemAlloc)
                  : "memory");
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
@@ -467,7 +525,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (kFused && threadIdx.x >= 64 && threadIdx.x < 64 + kSoftThreads) {
     // rotation table of the R new positions: (cos, sin) per (row, pair),
     // built while thread 0 takes the scene's length
-    float2* tabw = reinterpret_cast<float2*>(smem + C::kOffP);
+    float2* tabw = reinterpret_cast<float2*>(smem + C::kOffTab);
 #pragma unroll 1
     for (int idx = threadIdx.x - 64; idx < a.R * 64; idx += kSoftThreads) {
       const int i = idx >> 6, d = idx & 63;
@@ -481,6 +539,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem = *tmem_slot;
   const uint32_t tmem_s = tmem;            // S buffer b at column kR * b
   const uint32_t tmem_o = tmem + kSB * kR; // O^T
+  const uint32_t tmem_snew = tmem + (kSB + 1) * kR;  // fused layer: S_new^T (new keys on lanes 0..R-1)
 
   int n_keys, L_pre;
   bool valid;
@@ -505,12 +564,41 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int key_begin = blk_begin * 32;
   const int key_end = min(blk_end * 32, loop_keys);
   const int n_tiles = (blk_end - blk_begin + 3) / 4;
-
+  // rank c merges packed rows [c * rpc, c * rpc + rows_of(c)), rpc = ceil(kR / csize)
+  const int rpc = (kR + csize - 1) / csize;
+  auto rows_of = [&](int c) { return max(0, min(rpc, kR - c * rpc)); };
+  const int my_rows = rows_of(rank);
+  const int mrow0 = rank * rpc;
   if (warp == 0) {
     // -------------------------------------------------------------- producer
     // the whole warp waits, one elected lane issues the copies
+    const int z = b * a.Hkv + kvh;
+    auto issue_tiles = [&](int pass) {
+      for (int t = 0; t < n_tiles; ++t) {
+        const int T = pass * n_tiles + t;
+        const int s = T % kS;
+        // a whole 128-row box even for a short last tile: keys past the
+        // range are masked, rows past the capacity arrive zero-filled
+        const int y0 = key_begin + t * kStageKeys;
+        // slot s last held tile T - kS (all of pass 0 is done before pass 1)
+        const uint32_t kst = base + s * kKV, vst = base + C::kRingV + s * kKV;
+        if (t >= kS) mbar_wait(SREADY(T - kS), s_parity(T - kS));
+        if (elect_one()) {
+          mbar_expect_tx(FULLK(s), static_cast<uint32_t>(kKV));
+#pragma unroll
+          for (int h = 0; h < 2; ++h) tma_load_3d(kst + h * kHalf, &tm_k128, FULLK(s), h * 64, y0, z);
+        }
+        __syncwarp();
+        if (t >= kS) mbar_wait(PVDONE(T - kS), ring_parity(T - kS));
+        if (elect_one()) {
+          mbar_expect_tx(FULLV(s), static_cast<uint32_t>(kKV));
+#pragma unroll
+          for (int h = 0; h < 2; ++h) tma_load_3d(vst + h * kHalf, &tm_v128, FULLV(s), h * 64, y0, z);
+        }
+        __syncwarp();
+      }
+    };
     if (n_tiles > 0) {
-      const int z = b * a.Hkv + kvh;
       if (elect_one()) {
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_k128)) : "memory");
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_v128)) : "memory");
@@ -537,39 +625,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
       __syncwarp();
-      for (int pass = 0; pass < 2; ++pass) {
-        if (pass == 1) {
-          // every MMA of pass 0 is done when the decision is out
-          mbar_wait(DECIDE, 0);
-          if (!*reinterpret_cast<volatile int*>(s_redo)) break;
-        }
-        for (int t = 0; t < n_tiles; ++t) {
-          const int T = pass * n_tiles + t;
-          const int s = T % kS;
-          // a whole 128-row box even for a short last tile: keys past the
-          // range are masked, rows past the capacity arrive zero-filled
-          const int y0 = key_begin + t * kStageKeys;
-          // slot s last held tile T - kS (all of pass 0 is done before pass 1)
-          const uint32_t kst = base + s * kKV, vst = base + C::kRingV + s * kKV;
-          if (t >= kS) mbar_wait(SREADY(T - kS), s_parity(T - kS));
-          if (elect_one()) {
-            mbar_expect_tx(FULLK(s), static_cast<uint32_t>(kKV));
-#pragma unroll
-            for (int h = 0; h < 2; ++h) tma_load_3d(kst + h * kHalf, &tm_k128, FULLK(s), h * 64, y0, z);
-          }
-          __syncwarp();
-          if (t >= kS) mbar_wait(PVDONE(T - kS), ring_parity(T - kS));
-          if (elect_one()) {
-            mbar_expect_tx(FULLV(s), static_cast<uint32_t>(kKV));
-#pragma unroll
-            for (int h = 0; h < 2; ++h) tma_load_3d(vst + h * kHalf, &tm_v128, FULLV(s), h * 64, y0, z);
-          }
-          __syncwarp();
-        }
-      }
+      issue_tiles(0);
     }
     __syncwarp();
-    cluster_arrive();  // the cluster's rings are free (see the softmax branch)
+    // The cluster barrier lets peers write partials into this CTA's rings: the
+    // softmax threads arrive only after the last MMA of the last pass, so this
+    // warp (as the issuing warps) arrives before the second-pass decision.
+    cluster_arrive_relaxed();
     if (kFused && elect_one()) {
       // advance the scene's length once every CTA of the scene has read it:
       // the last CTA to take a ticket writes it. This lane (thread 0) read
@@ -584,19 +646,46 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
     __syncwarp();
+    if (n_tiles > 0) {
+      // every MMA of pass 0 is done when the decision is out
+      mbar_wait(DECIDE, 0);
+      if (*reinterpret_cast<volatile int*>(s_redo)) issue_tiles(1);
+    }
+    __syncwarp();
     cluster_wait();
   } else if (warp == 1) {
     // -------------------------------------------------------------- S issue
     // S(T) and PV(T) come from two warps (this one and the PV warp), so that
     // one batch is issued while the other executes; the whole warp waits and
     // one elected lane issues.
-    if (n_tiles > 0) {
+    const bool snew = kFused && valid;
+    bool arrived = false;
+    if (n_tiles > 0 || snew) {
       mbar_wait(QFULL, 0);
       // base descriptors; a K step only moves the start address (low field, no carry)
       const uint64_t dK0 = umma_desc(base, 16, 1024);  // K tile: K-major
       const uint64_t dQ = umma_desc(qs, 16, 1024);     // Q: K-major
+      // fused layer: the scores of the R new keys, S_new^T = K_new Q^T (new
+      // key n on lane n), into their own tensor-memory buffer after S(0); the
+      // operand sits in the first P buffer, which P(0) overwrites only once
+      // SNEW is out
+      auto issue_snew = [&]() {
+        tc_fence_after();
+        const uint64_t dN = umma_desc(base + C::kOffP, 16, 1024);
+        if (elect_one()) {
+#pragma unroll
+          for (int kk = 0; kk < 8; ++kk)
+            umma(tmem_snew, dN + (((kk >> 2) * C::kNewHalf + (kk & 3) * 32) >> 4),
+                 dQ + (((kk >> 2) * C::kQHalf + (kk & 3) * 32) >> 4), kIdescS, kk > 0 ? 1 : 0);
+          umma_commit(SNEW);
+        }
+        __syncwarp();
+      };
+      if (snew && n_tiles == 0) issue_snew();
       for (int pass = 0; pass < 2; ++pass) {
         if (pass == 1) {
+          cluster_arrive_relaxed();  // before the decision (see the producer)
+          arrived = true;
           mbar_wait(DECIDE, 0);
           if (!*reinterpret_cast<volatile int*>(s_redo)) break;
         }
@@ -618,20 +707,24 @@ __global__ void __launch_bounds__(kThreads, 1)
             umma_commit(SREADY(T));
           }
           __syncwarp();
+          if (snew && T == 0) issue_snew();
         }
       }
     }
     __syncwarp();
-    cluster_arrive();
+    if (!arrived) cluster_arrive_relaxed();
     cluster_wait();
   } else if (warp == kPvWarp) {
     // -------------------------------------------------------------- PV issue
+    bool arrived = false;
     if (n_tiles > 0) {
       const uint64_t dV0 = umma_desc(base + C::kRingV, kHalf, 1024);  // V^T: MN-major
       // P^T: MN-major, one swizzle atom wide (kR rows), 8-key groups 8 * kPRow apart
       const uint64_t dP0 = umma_desc(base + C::kOffP, 0, 8 * C::kPRow, C::kPLayout);
       for (int pass = 0; pass < 2; ++pass) {
         if (pass == 1) {
+          cluster_arrive_relaxed();  // before the decision (see the producer)
+          arrived = true;
           mbar_wait(DECIDE, 0);
           if (!*reinterpret_cast<volatile int*>(s_redo)) break;
         }
@@ -655,7 +748,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
     __syncwarp();
-    cluster_arrive();
+    if (!arrived) cluster_arrive_relaxed();
     cluster_wait();
   } else {
     // -------------------------------------------------------------- softmax
@@ -665,7 +758,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int kl = quarter * 32 + lane;    // key lane of S^T / d lane of O^T
     const uint32_t lane_off = static_cast<uint32_t>(quarter * 32) << 16;
     const int row0 = kRpt * half;          // first query row of this thread
-    const float2* cs_tab = reinterpret_cast<const float2*>(smem + C::kOffP);  // [R][64] (cos, sin)
+    const float2* cs_tab = reinterpret_cast<const float2*>(smem + C::kOffTab);  // [R][64] (cos, sin)
     {
       // the packed query tile: this thread's 16-byte chunks (row, chunk c),
       // rows past M zero; in the fused layer also one chunk of a new key and
@@ -686,6 +779,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // new key / value rows: chunk st + u * 256 (row >> 4, 16-byte chunk & 15);
       // one chunk a thread with 32 rows (16 new rows), two with 64 (32)
       constexpr int kKvc = C::kMaxNew * 16 / kSoftThreads;
+      const bool append = kFused && valid && rank == csize - 1 && mblock == 0;
       bool has_kv[kKvc];
       long long kv_src[kKvc];
 #pragma unroll
@@ -738,7 +832,16 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
             for (int j = 0; j < 4; ++j) w[j] = sd_rope_pair(w[j], cs[j].x, cs[j].y);
             st_shared_v4(base + C::kOffNewK + i * kNewRow + c * 16, w[0], w[1], w[2], w[3]);
+            st_shared_v4(base + C::kOffP + (c >> 3) * C::kNewHalf + i * 128 + (((c & 7) ^ (i & 7)) << 4), w[0], w[1],
+                         w[2], w[3]);
             st_shared_v4(base + C::kOffNewV + i * kNewRow + c * 16, vv[u].x, vv[u].y, vv[u].z, vv[u].w);
+            if (append && it == 1) {
+              // the append (the head's last rank of m-block 0): cache rows
+              // L_pre .. L_pre + R - 1, which no CTA of this launch reads
+              const long long dst = ((static_cast<long long>(b) * a.Hkv + kvh) * a.cap + L_pre + i) * kD + c * 8;
+              *reinterpret_cast<uint4*>(a.kc + dst) = make_uint4(w[0], w[1], w[2], w[3]);
+              *reinterpret_cast<uint4*>(a.vc + dst) = vv[u];
+            }
           } else {
             st_shared_v4(base + C::kOffNewV + i * kNewRow + c * 16, 0u, 0u, 0u, 0u);
           }
@@ -935,6 +1038,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             lp[j0 + j + 1] += sd_bf16_hi(w);
           }
           if (T >= 2 && j0 == 0) mbar_wait(PVDONE(T - 2), ring_parity(T - 2));  // PV(T - 2) has read P buffer bb
+          if (kFused && T == 0 && j0 == 0 && valid) mbar_wait(SNEW, 0);  // S_new has read its operand
           const int ch = (row0 + j0) >> 3;
           st_shared_v4(prow + ((ch ^ sw) << 4), pw[0], pw[1], pw[2], pw[3]);
           st_shared_v4(prow + (((ch + 1) ^ sw) << 4), pw[4], pw[5], pw[6], pw[7]);
@@ -958,13 +1062,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         mbar_wait(PVDONE(Tl), ring_parity(Tl));
       }
       if (pass == 0) {
-        // did any score exceed its reference by more than kSlack?
+        // did any score exceed its reference by more than kSlack? (one
+        // OR-reducing barrier over the softmax threads)
         bool over = false;
 #pragma unroll
         for (int j = 0; j < kRpt; ++j) over |= ex[j] > kSlack;
-        if (__any_sync(0xffffffffu, over) && lane == 0) atomicOr(s_excess, 1);
-        named_bar_sync(2, kSoftThreads);
-        redo = *reinterpret_cast<volatile int*>(s_excess) != 0;
+        redo = named_bar_or(2, kSoftThreads, over);
         if (st == 0) {
           *s_redo = redo ? 1 : 0;
           mbar_arrive(DECIDE);
@@ -994,16 +1097,36 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
 
-    // ---- CTA partial: O^T (tensor memory) of this thread's d lane and rows,
-    //      and the per-row m (reference) and l (sum over all 128 key lanes)
-    // every MMA of this CTA is done: its rings may now receive peers' partials.
-    // Relaxed: no data passes through this barrier (the tensor core's reads of
-    // the rings are complete, PVDONE was waited), it only orders execution.
-    // The partial is staged row-major: row j = [O(128) | m | l | pad], 528
-    // bytes; the l terms of the 128 key lanes go through the (free) P buffers.
+    // ---- this CTA's partial, staged row-major for the rows' owners: row r =
+    //      [O(128) | l per TMEM lane quarter (4) | m | pad]. Every MMA of the
+    //      CTA is done (PVDONE was waited), so its rings may receive peers'
+    //      partials. Relaxed: no data passes through this barrier, it only
+    //      orders execution.
     float* send = reinterpret_cast<float*>(smem + C::kSend);
-    float* lbuf = reinterpret_cast<float*>(smem + C::kOffP);  // [kR rows][128 key lanes]
     if (n_tiles > 0) tc_fence_after();
+    asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+    // the new-key scores of the rows this CTA merges, from S_new^T (new key n
+    // on lane n of the first TMEM lane quarter), scaled, causally masked
+    float* s_new = reinterpret_cast<float*>(smem + C::kNewS);  // [my_rows][R]
+    if (kFused && valid && quarter == 0 && half == 0) {
+      mbar_wait(SNEW, 0);
+      tc_fence_after();
+#pragma unroll 1
+      for (int rr0 = 0; rr0 < my_rows; rr0 += 4) {
+        // columns past the merged rows stay inside the allocation and go unused
+        uint32_t v[4];
+        asm volatile("tcgen05.ld.sync.aligned.32x32b.x4.b32 {%0,%1,%2,%3}, [%4];"
+                     : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3])
+                     : "r"(tmem_snew + mrow0 + rr0));
+        asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const int rr = rr0 + j, p = mblock * kR + mrow0 + rr;
+          if (rr < my_rows && lane < a.R)
+            s_new[rr * a.R + lane] = (p < a.M && lane <= gdiv(p)) ? __uint_as_float(v[j]) * a.scale_log2 : -INFINITY;
+        }
+      }
+    }
 #pragma unroll
     for (int j0 = 0; j0 < kRpt; j0 += 16) {
       uint32_t o[16];
@@ -1013,45 +1136,20 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
         for (int j = 0; j < 16; ++j) o[j] = 0u;
       }
-      if (j0 == 0) asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
 #pragma unroll
-      for (int j = 0; j < 16; ++j) {
-        send[(row0 + j0 + j) * kRowF + kl] = __uint_as_float(o[j]);
-        lbuf[(row0 + j0 + j) * 128 + kl] = lp[j0 + j];
-      }
+      for (int j = 0; j < 16; ++j) send[(row0 + j0 + j) * kRowF + kl] = __uint_as_float(o[j]);
     }
-    named_bar_sync(2, kSoftThreads);
     {
-      // softmax warp w sums rows kRw * w .. kRw * w + kRw - 1: 512 contiguous
-      // bytes per load
-      constexpr int kRw = kR / kSoftWarps;
-      const int w = warp - 2;
-      const float4* src = reinterpret_cast<const float4*>(lbuf + w * kRw * 128);
-      float lw[kRw];
-#pragma unroll
-      for (int i = 0; i < kRw; ++i) {
-        const float4 x = src[i * 32 + lane];
-        lw[i] = (x.x + x.y) + (x.z + x.w);
-      }
-#pragma unroll
-      for (int sh = 16; sh >= 1; sh >>= 1)
-#pragma unroll
-        for (int i = 0; i < kRw; ++i) lw[i] += __shfl_xor_sync(0xffffffffu, lw[i], sh);
-      float l = lw[0];
-#pragma unroll
-      for (int i = 1; i < kRw; ++i) l = lane == i ? lw[i] : l;
-      if (lane < kRw) {
-        const int r = kRw * w + lane;
-        send[r * kRowF + kD] = n_tiles > 0 ? row_ref[r] : -INFINITY;
-        send[r * kRowF + kD + 1] = l;
-      }
+      // l of each row over this warp's 32 key lanes; the owner adds the four
+      // quarters
+      int lrow;
+      const float lw = warp_rows_sum<kRpt>(lp, lane, lrow);
+      if (kRpt == 32 || (lane & 1) == 0) send[(row0 + lrow) * kRowF + kRowL + quarter] = lw;
+      if (quarter == 0 && lane < kRpt)
+        send[(row0 + lane) * kRowF + kRowM] = n_tiles > 0 ? row_ref[row0 + lane] : -INFINITY;
     }
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     named_bar_sync(2, kSoftThreads);
-    // rank c merges rows [c * rpc, c * rpc + rows_of(c)): rpc = ceil(kR / csize)
-    const int rpc = (kR + csize - 1) / csize;
-    auto rows_of = [&](int c) { return max(0, min(rpc, kR - c * rpc)); };
-    const int my_rows = rows_of(rank);
     if (st == 0) mbar_expect_tx(RECV, static_cast<uint32_t>(csize * my_rows * kRowBytes));
     cluster_wait();  // every peer's ring is free to receive
     // softmax warp w sends rank c's rows to rank c (c = w, w + 8), into its
@@ -1066,152 +1164,138 @@ __global__ void __launch_bounds__(kThreads, 1)
       asm volatile("cp.async.bulk.commit_group;" ::: "memory");
     }
     __syncwarp();
-    const int mrow0 = rank * rpc;  // the rows this CTA merges
-    float* s_new = reinterpret_cast<float*>(smem + C::kNewS);  // [rpc][R] scores of the new keys
-    if (kFused && valid) {
-      // new-key scores (log2 units) of the merged rows, 8 threads per dot product;
-      // query row p = i * G + g sees new keys 0..i (Eq. verify's causal mask)
-      const int sub = lane & 7;
-      const int n_pairs = my_rows * a.R;
-#pragma unroll 1
-      for (int pr0 = (st >> 5) * 4; pr0 < n_pairs; pr0 += kSoftThreads / 8) {  // warp-uniform
-        const int pr = min(pr0 + (lane >> 3), n_pairs - 1);
-        const bool act = pr0 + (lane >> 3) < n_pairs;
-        const int rr = pr / a.R, n = pr % a.R;
-        const int row = mrow0 + rr;
-        const int p = mblock * kR + row;
-        float acc = 0.f;
-#pragma unroll
-        for (int u = 0; u < 2; ++u) {
-          const int c = sub + 8 * u;
-          const uint4 qw4 = *reinterpret_cast<const uint4*>(smem + C::kOffQ + (c >> 3) * C::kQHalf + row * 128 +
-                                                             (((c & 7) ^ (row & 7)) << 4));
-          const uint4 kw4 = *reinterpret_cast<const uint4*>(smem + C::kOffNewK + n * kNewRow + c * 16);
-          const uint32_t qa[4] = {qw4.x, qw4.y, qw4.z, qw4.w};
-          const uint32_t ka[4] = {kw4.x, kw4.y, kw4.z, kw4.w};
-#pragma unroll
-          for (int j = 0; j < 4; ++j) {
-            acc = fmaf(sd_bf16_lo(qa[j]), sd_bf16_lo(ka[j]), acc);
-            acc = fmaf(sd_bf16_hi(qa[j]), sd_bf16_hi(ka[j]), acc);
-          }
-        }
-        acc += __shfl_xor_sync(0xffffffffu, acc, 1);
-        acc += __shfl_xor_sync(0xffffffffu, acc, 2);
-        acc += __shfl_xor_sync(0xffffffffu, acc, 4);
-        if (sub == 0 && act) s_new[pr] = (p < a.M && n <= gdiv(p)) ? acc * sl : -INFINITY;
-      }
-      named_bar_sync(2, kSoftThreads);
-    }
     // ---- merge of the rows this CTA owns; slot c * rpc + rr came from rank c.
-    // A warp takes one row (kD / 2 = 64 items a row, so a row is two whole
-    // warps) and a thread two adjacent d. Lane c forms the weight of partial c
-    // (c < csize) and of new key c (c < R) once for the warp; the weights are
-    // broadcast by shuffles to the FMAs of every lane.
-    mbar_wait(RECV, 0);
-    const float* recv = reinterpret_cast<const float*>(smem + C::kRecv);
+    // 64 threads a row, two adjacent d a thread. While the partials travel,
+    // the new keys' part: with M = max(the row's reference, its new-key
+    // scores), sum_n w_n v_n and sum_n w_n, w_n = 2^(s_n - M). When every rank
+    // used the row's reference (the common case: the second pass is rare), the
+    // partials then add with the one weight 2^(ref - M); otherwise every
+    // partial takes its own weight.
     const int n_new = (kFused && valid) ? a.R : 0;
-    static_assert(C::kMaxNew <= 32, "one new key a lane");
+    const int rr = st >> 6, d = 2 * (st & 63);  // my_rows <= 4 here; more rows loop below
+    float nx = 0.f, ny = 0.f, nl = 0.f, mloc = -INFINITY, rref = -INFINITY;
+    if (rr < my_rows) {
+      rref = n_tiles > 0 ? row_ref[mrow0 + rr] : -INFINITY;
+      mloc = rref;
+      const float* sn = s_new + rr * a.R;
 #pragma unroll 1
-    for (int idx = st; idx < my_rows * (kD / 2); idx += kSoftThreads) {  // warp-uniform
-      const int rr = idx / (kD / 2), d = 2 * (idx % (kD / 2));
-      const int row = mrow0 + rr;
-      const int p = mblock * kR + row;
-      float2 ml = make_float2(-INFINITY, 0.f);  // (m, l) of partial `lane`
-      if (lane < csize) ml = *reinterpret_cast<const float2*>(recv + (lane * rpc + rr) * kRowF + kD);
-      const float sn = lane < n_new ? s_new[rr * a.R + lane] : -INFINITY;
-      float mx = fmaxf(ml.x, sn);
-#pragma unroll
-      for (int sh = 16; sh >= 1; sh >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, sh));
-      const float msub = mx == -INFINITY ? 0.f : mx;  // no key at all: every weight 0
-      const float wp = ex2(ml.x - msub);              // ex2(-inf) = 0
-      const float wn = ex2(sn - msub);
-      float lsum = fmaf(wp, ml.y, wn);
-#pragma unroll
-      for (int sh = 16; sh >= 1; sh >>= 1) lsum += __shfl_xor_sync(0xffffffffu, lsum, sh);
-      float2 acc = make_float2(0.f, 0.f);
-      // the fused layer's ranks share each row's reference unless one of them
-      // ran the second pass: then every partial has the same weight
-      const float m0 = __shfl_sync(0xffffffffu, ml.x, 0);
-      if (__all_sync(0xffffffffu, lane >= csize || ml.x == m0)) {
-#pragma unroll 4
-        for (int c = 0; c < csize; ++c) {
-          const float2 o = *reinterpret_cast<const float2*>(recv + (c * rpc + rr) * kRowF + d);
-          acc.x += o.x;
-          acc.y += o.y;
-        }
-        const float w = __shfl_sync(0xffffffffu, wp, 0);
-        acc.x *= w;
-        acc.y *= w;
-      } else {
-#pragma unroll 4
-        for (int c = 0; c < csize; ++c) {
-          const float w = __shfl_sync(0xffffffffu, wp, c);
-          const float2 o = *reinterpret_cast<const float2*>(recv + (c * rpc + rr) * kRowF + d);
-          acc.x = fmaf(w, o.x, acc.x);
-          acc.y = fmaf(w, o.y, acc.y);
-        }
-      }
+      for (int n = 0; n < n_new; ++n) mloc = fmaxf(mloc, sn[n]);
+      const float msub = mloc == -INFINITY ? 0.f : mloc;
 #pragma unroll 4
       for (int n = 0; n < n_new; ++n) {
-        const float w = __shfl_sync(0xffffffffu, wn, n);
+        const float w = ex2(sn[n] - msub);
         const uint32_t v2 = *reinterpret_cast<const uint32_t*>(smem + C::kOffNewV + n * kNewRow + d * 2);
-        acc.x = fmaf(w, sd_bf16_lo(v2), acc.x);
-        acc.y = fmaf(w, sd_bf16_hi(v2), acc.y);
-      }
-      if (valid && p < a.M && lsum > 0.f) {
-        const float inv_l = 1.f / lsum;
-        const int i = gdiv(p), gq = (p - gdiv(p) * a.G);
-        *reinterpret_cast<uint32_t*>(a.out + ((static_cast<long long>(b) * a.R + i) * a.Hq + kvh * a.G + gq) * kD +
-                                     d) = cvt_bf16x2(acc.x * inv_l, acc.y * inv_l);
+        nl += w;
+        nx = fmaf(w, sd_bf16_lo(v2), nx);
+        ny = fmaf(w, sd_bf16_hi(v2), ny);
       }
     }
-    if (elect_one()) asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
-    __syncwarp();
-    if (kFused && valid) {
-      // every CTA of the cluster read the raw rows before its main loop (the
-      // cluster barrier above is behind all of them): store the rotated query
-      // rows of this m-block (rank 0), and append the new key / value rows
-      // and store the rotated keys back (last rank of m-block 0)
-      if (rank == 0) {
+    mbar_wait(RECV, 0);
+    const float* recv = reinterpret_cast<const float*>(smem + C::kRecv);
 #pragma unroll 1
-        for (int idx = st; idx < kR * 16; idx += kSoftThreads) {
-          const int row = idx / 16, c = idx % 16;
-          const int p = mblock * kR + row;
-          if (p >= a.M) continue;
-          const uint4 v = *reinterpret_cast<const uint4*>(smem + C::kOffQ + (c >> 3) * C::kQHalf + row * 128 +
-                                                          (((c & 7) ^ (row & 7)) << 4));
-          *reinterpret_cast<uint4*>(a.qw + ((static_cast<long long>(b) * a.R + gdiv(p)) * a.Hq + kvh * a.G +
-                                            (p - gdiv(p) * a.G)) * kD + c * 8) = v;
+    for (int r = rr; r < my_rows; r += kSoftThreads / 64) {  // warp-uniform
+      if (r != rr) {
+        // rows beyond the first four (clusters of fewer than 8): their new keys here
+        rref = n_tiles > 0 ? row_ref[mrow0 + r] : -INFINITY;
+        mloc = rref;
+        nx = ny = nl = 0.f;
+        const float* sn = s_new + r * a.R;
+#pragma unroll 1
+        for (int n = 0; n < n_new; ++n) mloc = fmaxf(mloc, sn[n]);
+        const float msub = mloc == -INFINITY ? 0.f : mloc;
+#pragma unroll 1
+        for (int n = 0; n < n_new; ++n) {
+          const float w = ex2(sn[n] - msub);
+          const uint32_t v2 = *reinterpret_cast<const uint32_t*>(smem + C::kOffNewV + n * kNewRow + d * 2);
+          nl += w;
+          nx = fmaf(w, sd_bf16_lo(v2), nx);
+          ny = fmaf(w, sd_bf16_hi(v2), ny);
         }
       }
-      const bool append = rank == csize - 1 && mblock == 0;
-      // the head's last reader of the raw key rows (32 rows: one m-block, one cluster)
-      bool write_k = append;
+      const float* part = recv + r * kRowF;  // rank c's partial at part + c * rpc * kRowF
+      float ox = 0.f, oy = 0.f, ls = 0.f;
+      bool same = true;
+#pragma unroll 4
+      for (int c = 0; c < csize; ++c) {
+        const float* pc = part + c * rpc * kRowF;
+        const float2 o = *reinterpret_cast<const float2*>(pc + d);
+        const float4 lq = *reinterpret_cast<const float4*>(pc + kRowL);
+        same = same && pc[kRowM] == rref;
+        ox += o.x;
+        oy += o.y;
+        ls += (lq.x + lq.y) + (lq.z + lq.w);
+      }
+      float wp = ex2(rref - (mloc == -INFINITY ? 0.f : mloc));  // ex2(-inf) = 0
+      if (!same) {
+        // some rank ran the second pass: weigh every partial by its own reference
+        float mx = mloc;
+#pragma unroll 1
+        for (int c = 0; c < csize; ++c) mx = fmaxf(mx, part[c * rpc * kRowF + kRowM]);
+        const float msub = mx == -INFINITY ? 0.f : mx;
+        const float rescale = ex2((mloc == -INFINITY ? 0.f : mloc) - msub);  // the new keys' part was scaled by mloc
+        nx *= rescale;
+        ny *= rescale;
+        nl *= rescale;
+        ox = oy = ls = 0.f;
+#pragma unroll 1
+        for (int c = 0; c < csize; ++c) {
+          const float* pc = part + c * rpc * kRowF;
+          const float w = ex2(pc[kRowM] - msub);
+          const float2 o = *reinterpret_cast<const float2*>(pc + d);
+          const float4 lq = *reinterpret_cast<const float4*>(pc + kRowL);
+          ox = fmaf(w, o.x, ox);
+          oy = fmaf(w, o.y, oy);
+          ls = fmaf(w, (lq.x + lq.y) + (lq.z + lq.w), ls);
+        }
+        wp = 1.f;
+      }
+      const float l = fmaf(wp, ls, nl);
+      const int p = mblock * kR + mrow0 + r;
+      if (valid && p < a.M && l > 0.f) {
+        const float inv_l = 1.f / l;
+        const int i = gdiv(p), gq = p - i * a.G;
+        *reinterpret_cast<uint32_t*>(a.out + ((static_cast<long long>(b) * a.R + i) * a.Hq + kvh * a.G + gq) * kD +
+                                     d) = cvt_bf16x2(fmaf(wp, ox, nx) * inv_l, fmaf(wp, oy, ny) * inv_l);
+      }
+    }
+    if (kFused && valid) {
+      // every CTA of the cluster read the raw rows before its tiles (the
+      // cluster barrier above is behind all of them): the rotated query rows
+      // this CTA merged go back to q, and the head's last reader of the raw
+      // key rows writes the rotated ones back to k_new
+#pragma unroll 1
+      for (int idx = st; idx < my_rows * 16; idx += kSoftThreads) {
+        const int row = mrow0 + idx / 16, c = idx % 16;
+        const int p = mblock * kR + row;
+        if (p >= a.M) continue;
+        const uint4 v = *reinterpret_cast<const uint4*>(smem + C::kOffQ + (c >> 3) * C::kQHalf + row * 128 +
+                                                        (((c & 7) ^ (row & 7)) << 4));
+        *reinterpret_cast<uint4*>(a.qw + ((static_cast<long long>(b) * a.R + gdiv(p)) * a.Hq + kvh * a.G +
+                                          (p - gdiv(p) * a.G)) * kD + c * 8) = v;
+      }
+      // 32 rows: one m-block, one cluster, so its last rank
+      bool write_k = rank == csize - 1 && mblock == 0;
       if constexpr (kR == 64) write_k = *s_kvlast != 0;
-      if (append || write_k) {
+      if (write_k) {
 #pragma unroll 1
         for (int idx = st; idx < a.R * 16; idx += kSoftThreads) {
           const int i = idx / 16, c = idx % 16;
           const long long src = ((static_cast<long long>(b) * a.R + i) * a.Hkv + kvh) * kD + c * 8;
-          const long long dst = ((static_cast<long long>(b) * a.Hkv + kvh) * a.cap + L_pre + i) * kD + c * 8;
-          const uint4 kr = *reinterpret_cast<const uint4*>(smem + C::kOffNewK + i * kNewRow + c * 16);
-          if (append) {
-            *reinterpret_cast<uint4*>(a.kc + dst) = kr;
-            *reinterpret_cast<uint4*>(a.vc + dst) =
-                *reinterpret_cast<const uint4*>(smem + C::kOffNewV + i * kNewRow + c * 16);
-          }
-          if (write_k) *reinterpret_cast<uint4*>(a.k_new + src) = kr;
+          *reinterpret_cast<uint4*>(a.k_new + src) =
+              *reinterpret_cast<const uint4*>(smem + C::kOffNewK + i * kNewRow + c * 16);
         }
-        if (kR == 64 && write_k && a.n_mblocks > 1 && st == 0) a.kv_ticket[b * a.Hkv + kvh] = 0;  // re-armed
+        if (kR == 64 && a.n_mblocks > 1 && st == 0) a.kv_ticket[b * a.Hkv + kvh] = 0;  // re-armed
       }
     }
+    if (elect_one()) asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+    __syncwarp();
   }
   tc_fence_before();
   __syncthreads();  // every tensor-memory read is done
   if (warp == 1) {
     tc_fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
-                 "r"(C::kTmemCols)
+                 "r"(kTmemAlloc)
                  : "memory");
   }
 }
