@@ -118,8 +118,8 @@ struct Cfg {
   // columns)
   static constexpr int kSBuf = 3;
   // barriers: full_k[S] full_v[S] p_full[2] s_ready[3] pv_done[S] q_full recv
-  // decide s_free[3] s_new
-  static constexpr int kNumBars = 3 * kStages + 12;
+  // decide s_free[3] s_new tmem_done
+  static constexpr int kNumBars = 3 * kStages + 13;
   // tmem slot, (unused), decision, len (and, 64 rows, the last reader of the new key rows)
   static constexpr int kOffMisc = round_up(kOffBar + kNumBars * 8, 16);
   static constexpr int kOffRowA = kOffMisc + (kR == 32 ? 16 : 32);  // [kR] per-row results (reductions)
@@ -185,6 +185,22 @@ __device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap* map
       "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(x), "r"(y), "r"(z)
       : "memory");
 }
+// The same load with an L2 eviction policy (createpolicy): the cached prefix is
+// read once per step, so its lines go first and the code and the per-step rows
+// stay in L2 (an instruction fetch that misses L2 waits behind the stream).
+__device__ __forceinline__ void tma_load_3d_hint(uint32_t dst, const CUtensorMap* map, uint32_t bar, int x, int y,
+                                                 int z, uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.L2::cache_hint"
+      " [%0], [%1, {%3, %4, %5}], [%2], %6;" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(x), "r"(y), "r"(z), "l"(policy)
+      : "memory");
+}
+__device__ __forceinline__ uint64_t l2_evict_first_policy() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
 __device__ __forceinline__ void tma_prefetch_3d(const CUtensorMap* map, int x, int y, int z) {
   asm volatile("cp.async.bulk.prefetch.tensor.3d.L2.global.tile [%0, {%1, %2, %3}];" ::"l"(
                    reinterpret_cast<uint64_t>(map)),
@@ -247,9 +263,6 @@ __device__ __forceinline__ float warp_rows_sum(const float (&v0)[kN], int lane, 
   if (kN == 16) x += __shfl_xor_sync(0xffffffffu, x, 1);
   row = r;
   return x;
-}
-__device__ __forceinline__ void cluster_arrive() {
-  asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
 }
 // an arrival that orders nothing: no data passes through the barrier
 __device__ __forceinline__ void cluster_arrive_relaxed() {
@@ -477,6 +490,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   auto SFREE = [&](int T) { return bar(3 * kS + 8 + T % 3); };
   auto s_parity = [](int T) { return static_cast<uint32_t>((T / 3) & 1); };  // SREADY, SFREE phases
   const uint32_t SNEW = bar(3 * kS + 11);  // fused layer: S_new = K_new Q^T is in tensor memory
+  const uint32_t TMEMDONE = bar(3 * kS + 12);  // every softmax warp has read its last column
   constexpr int kSB = C::kSBuf;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::kOffMisc);
   int* s_redo = reinterpret_cast<int*>(smem + C::kOffMisc + 8);
@@ -507,6 +521,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(DECIDE, 1);
     for (int i = 0; i < 3; ++i) mbar_init(SFREE(i), kSoftWarps);
     mbar_init(SNEW, 1);
+    mbar_init(TMEMDONE, kSoftWarps);
     *s_redo = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
@@ -573,6 +588,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // -------------------------------------------------------------- producer
     // the whole warp waits, one elected lane issues the copies
     const int z = b * a.Hkv + kvh;
+    const uint64_t evict_first = l2_evict_first_policy();
     auto issue_tiles = [&](int pass) {
       for (int t = 0; t < n_tiles; ++t) {
         const int T = pass * n_tiles + t;
@@ -586,14 +602,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (elect_one()) {
           mbar_expect_tx(FULLK(s), static_cast<uint32_t>(kKV));
 #pragma unroll
-          for (int h = 0; h < 2; ++h) tma_load_3d(kst + h * kHalf, &tm_k128, FULLK(s), h * 64, y0, z);
+          for (int h = 0; h < 2; ++h) tma_load_3d_hint(kst + h * kHalf, &tm_k128, FULLK(s), h * 64, y0, z, evict_first);
         }
         __syncwarp();
         if (t >= kS) mbar_wait(PVDONE(T - kS), ring_parity(T - kS));
         if (elect_one()) {
           mbar_expect_tx(FULLV(s), static_cast<uint32_t>(kKV));
 #pragma unroll
-          for (int h = 0; h < 2; ++h) tma_load_3d(vst + h * kHalf, &tm_v128, FULLV(s), h * 64, y0, z);
+          for (int h = 0; h < 2; ++h) tma_load_3d_hint(vst + h * kHalf, &tm_v128, FULLV(s), h * 64, y0, z, evict_first);
         }
         __syncwarp();
       }
@@ -713,6 +729,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     __syncwarp();
     if (!arrived) cluster_arrive_relaxed();
+    // the allocating warp frees the tensor memory once every softmax warp has
+    // read its last column (every MMA is done by then)
+    mbar_wait(TMEMDONE, 0);
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemAlloc) : "memory");
     cluster_wait();
   } else if (warp == kPvWarp) {
     // -------------------------------------------------------------- PV issue
@@ -1148,6 +1169,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (quarter == 0 && lane < kRpt)
         send[(row0 + lane) * kRowF + kRowM] = n_tiles > 0 ? row_ref[row0 + lane] : -INFINITY;
     }
+    // this warp's last tensor-memory read is done: the allocating warp frees the
+    // columns while the partials merge (the kernel's end is not held by it)
+    tc_fence_before();
+    __syncwarp();
+    if (lane == 0) mbar_arrive(TMEMDONE);
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     named_bar_sync(2, kSoftThreads);
     if (st == 0) mbar_expect_tx(RECV, static_cast<uint32_t>(csize * my_rows * kRowBytes));
@@ -1164,6 +1190,35 @@ __global__ void __launch_bounds__(kThreads, 1)
       asm volatile("cp.async.bulk.commit_group;" ::: "memory");
     }
     __syncwarp();
+    if (kFused && valid) {
+      // while the partials travel: every CTA of the cluster read the raw rows
+      // before its tiles (the cluster barrier above is behind all of them), so
+      // the rotated query rows this CTA merges go back to q, and the head's
+      // last reader of the raw key rows writes the rotated ones back to k_new
+#pragma unroll 1
+      for (int idx = st; idx < my_rows * 16; idx += kSoftThreads) {
+        const int row = mrow0 + idx / 16, c = idx % 16;
+        const int p = mblock * kR + row;
+        if (p >= a.M) continue;
+        const uint4 v = *reinterpret_cast<const uint4*>(smem + C::kOffQ + (c >> 3) * C::kQHalf + row * 128 +
+                                                        (((c & 7) ^ (row & 7)) << 4));
+        *reinterpret_cast<uint4*>(a.qw + ((static_cast<long long>(b) * a.R + gdiv(p)) * a.Hq + kvh * a.G +
+                                          (p - gdiv(p) * a.G)) * kD + c * 8) = v;
+      }
+      // 32 rows: one m-block, one cluster, so its last rank
+      bool write_k = rank == csize - 1 && mblock == 0;
+      if constexpr (kR == 64) write_k = *s_kvlast != 0;
+      if (write_k) {
+#pragma unroll 1
+        for (int idx = st; idx < a.R * 16; idx += kSoftThreads) {
+          const int i = idx / 16, c = idx % 16;
+          const long long src = ((static_cast<long long>(b) * a.R + i) * a.Hkv + kvh) * kD + c * 8;
+          *reinterpret_cast<uint4*>(a.k_new + src) =
+              *reinterpret_cast<const uint4*>(smem + C::kOffNewK + i * kNewRow + c * 16);
+        }
+        if (kR == 64 && a.n_mblocks > 1 && st == 0) a.kv_ticket[b * a.Hkv + kvh] = 0;  // re-armed
+      }
+    }
     // ---- merge of the rows this CTA owns; slot c * rpc + rr came from rank c.
     // 64 threads a row, two adjacent d a thread. While the partials travel,
     // the new keys' part: with M = max(the row's reference, its new-key
@@ -1258,46 +1313,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                                      d) = cvt_bf16x2(fmaf(wp, ox, nx) * inv_l, fmaf(wp, oy, ny) * inv_l);
       }
     }
-    if (kFused && valid) {
-      // every CTA of the cluster read the raw rows before its tiles (the
-      // cluster barrier above is behind all of them): the rotated query rows
-      // this CTA merged go back to q, and the head's last reader of the raw
-      // key rows writes the rotated ones back to k_new
-#pragma unroll 1
-      for (int idx = st; idx < my_rows * 16; idx += kSoftThreads) {
-        const int row = mrow0 + idx / 16, c = idx % 16;
-        const int p = mblock * kR + row;
-        if (p >= a.M) continue;
-        const uint4 v = *reinterpret_cast<const uint4*>(smem + C::kOffQ + (c >> 3) * C::kQHalf + row * 128 +
-                                                        (((c & 7) ^ (row & 7)) << 4));
-        *reinterpret_cast<uint4*>(a.qw + ((static_cast<long long>(b) * a.R + gdiv(p)) * a.Hq + kvh * a.G +
-                                          (p - gdiv(p) * a.G)) * kD + c * 8) = v;
-      }
-      // 32 rows: one m-block, one cluster, so its last rank
-      bool write_k = rank == csize - 1 && mblock == 0;
-      if constexpr (kR == 64) write_k = *s_kvlast != 0;
-      if (write_k) {
-#pragma unroll 1
-        for (int idx = st; idx < a.R * 16; idx += kSoftThreads) {
-          const int i = idx / 16, c = idx % 16;
-          const long long src = ((static_cast<long long>(b) * a.R + i) * a.Hkv + kvh) * kD + c * 8;
-          *reinterpret_cast<uint4*>(a.k_new + src) =
-              *reinterpret_cast<const uint4*>(smem + C::kOffNewK + i * kNewRow + c * 16);
-        }
-        if (kR == 64 && a.n_mblocks > 1 && st == 0) a.kv_ticket[b * a.Hkv + kvh] = 0;  // re-armed
-      }
-    }
     if (elect_one()) asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
     __syncwarp();
   }
-  tc_fence_before();
-  __syncthreads();  // every tensor-memory read is done
-  if (warp == 1) {
-    tc_fence_after();
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
-                 "r"(kTmemAlloc)
-                 : "memory");
-  }
+  // no CTA-wide barrier at the end: every warp leaves when its own work is
+  // done (the softmax warps last: they wait for the partials coming in and for
+  // their outgoing copies to have been read)
 }
 
 // ------------------------------------------------------------------ host
