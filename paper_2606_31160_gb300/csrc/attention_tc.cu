@@ -1077,18 +1077,17 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncwarp();
         if (lane == 0) mbar_arrive(PFULL(bb));
       }
-      if (n_tiles > 0) {
-        // every MMA of the pass is done (PVDONE's phases complete in order)
-        const int Tl = pass * n_tiles + n_tiles - 1;
-        mbar_wait(PVDONE(Tl), ring_parity(Tl));
-      }
       if (pass == 0) {
         // did any score exceed its reference by more than kSlack? (one
-        // OR-reducing barrier over the softmax threads)
+        // OR-reducing barrier over the softmax threads, while the last PV
+        // product runs)
         bool over = false;
 #pragma unroll
         for (int j = 0; j < kRpt; ++j) over |= ex[j] > kSlack;
         redo = named_bar_or(2, kSoftThreads, over);
+        // before a second pass every MMA of the first is done (the producer
+        // refills the rings once the decision is out)
+        if (redo && n_tiles > 0) mbar_wait(PVDONE(n_tiles - 1), ring_parity(n_tiles - 1));
         if (st == 0) {
           *s_redo = redo ? 1 : 0;
           mbar_arrive(DECIDE);
@@ -1119,13 +1118,24 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
 
     // ---- this CTA's partial, staged row-major for the rows' owners: row r =
-    //      [O(128) | l per TMEM lane quarter (4) | m | pad]. Every MMA of the
-    //      CTA is done (PVDONE was waited), so its rings may receive peers'
-    //      partials. Relaxed: no data passes through this barrier, it only
-    //      orders execution.
+    //      [O(128) | l per TMEM lane quarter (4) | m | pad]. The send, receive
+    //      and score buffers sit in the K ring (32-row tile), free once the
+    //      last S product was read: the l terms, the new keys' scores and the
+    //      cluster arrival (relaxed: no data passes, it only orders execution)
+    //      go ahead of the last PV product; the 64-row tile's buffers reach
+    //      into the V ring, so it arrives after it.
+    constexpr bool kEarlyArrive = C::kNewS + kR * C::kMaxNew * 4 <= C::kRingV;
     float* send = reinterpret_cast<float*>(smem + C::kSend);
-    if (n_tiles > 0) tc_fence_after();
-    asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+    if (kEarlyArrive) asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+    {
+      // l of each row over this warp's 32 key lanes; the owner adds the four
+      // quarters
+      int lrow;
+      const float lw = warp_rows_sum<kRpt>(lp, lane, lrow);
+      if (kRpt == 32 || (lane & 1) == 0) send[(row0 + lrow) * kRowF + kRowL + quarter] = lw;
+      if (quarter == 0 && lane < kRpt)
+        send[(row0 + lane) * kRowF + kRowM] = n_tiles > 0 ? row_ref[row0 + lane] : -INFINITY;
+    }
     // the new-key scores of the rows this CTA merges, from S_new^T (new key n
     // on lane n of the first TMEM lane quarter), scaled, causally masked
     float* s_new = reinterpret_cast<float*>(smem + C::kNewS);  // [my_rows][R]
@@ -1148,6 +1158,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
     }
+    if (n_tiles > 0) {
+      // every MMA is done once the last PV is (PVDONE's phases complete in order)
+      const int Tl = (redo ? 2 : 1) * n_tiles - 1;
+      mbar_wait(PVDONE(Tl), ring_parity(Tl));
+      tc_fence_after();
+    }
+    if (!kEarlyArrive) asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
 #pragma unroll
     for (int j0 = 0; j0 < kRpt; j0 += 16) {
       uint32_t o[16];
@@ -1159,15 +1176,6 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
 #pragma unroll
       for (int j = 0; j < 16; ++j) send[(row0 + j0 + j) * kRowF + kl] = __uint_as_float(o[j]);
-    }
-    {
-      // l of each row over this warp's 32 key lanes; the owner adds the four
-      // quarters
-      int lrow;
-      const float lw = warp_rows_sum<kRpt>(lp, lane, lrow);
-      if (kRpt == 32 || (lane & 1) == 0) send[(row0 + lrow) * kRowF + kRowL + quarter] = lw;
-      if (quarter == 0 && lane < kRpt)
-        send[(row0 + lane) * kRowF + kRowM] = n_tiles > 0 ? row_ref[row0 + lane] : -INFINITY;
     }
     // this warp's last tensor-memory read is done: the allocating warp frees the
     // columns while the partials merge (the kernel's end is not held by it)
