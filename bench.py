@@ -263,9 +263,12 @@ class Step:
         self.layers()
         self.lens.copy_(self.lens0, non_blocking=True)
 
-    def attention_only(self):
+    def attention_only(self, early=True):
+        """The standalone sd_verify_attention over the 36 appended caches; layers
+        after the first are programmatic dependent launches (SD_ATTN_PREFIX_EARLY)
+        unless early=False."""
         for l in range(LAYERS):
-            self.sd.verify_attention(self.q[l], self.caches[l], out=self.out[l])
+            self.sd.verify_attention(self.q[l], self.caches[l], out=self.out[l], early=early and l > 0)
 
     def accept_only(self):
         self.sd.accept_greedy(self.logits, self.draft, ws=self.ws, n_emit=self.n_emit, tokens=self.tokens,
@@ -652,6 +655,7 @@ def main():
     for l in range(LAYERS):  # the standalone attention needs the appended rows
         sd.kv_append(st.caches[l], st.k[l], st.v[l])
     g_attn = capture(st.attention_only)
+    g_attn_plain = capture(lambda: st.attention_only(early=False))
     st.lens.copy_(st.lens0)
     torch.cuda.synchronize()
     g_step = capture(st.run)
@@ -691,6 +695,7 @@ def main():
     for l in range(LAYERS):
         sd.kv_append(st.caches[l], st.k[l], st.v[l])
     ms_attn_launch = time_graph(g_attn, reps) / LAYERS
+    ms_attn_plain = time_graph(g_attn_plain, reps) / LAYERS
     st.lens.copy_(st.lens0)
     torch.cuda.synchronize()
     # ---- the small kernels of the path, per call: M-RoPE of one layer's rows,
@@ -773,6 +778,7 @@ def main():
         "per_layer_us": round(ms_step * 1e3 / LAYERS, 3),
         "layer_us": round(ms_layer_launch * 1e3, 3),
         "attention_us": round(ms_attn_launch * 1e3, 3),
+        "attention_us_no_early_prefix": round(ms_attn_plain * 1e3, 3),
         "unfused_verify_step_us": round(ms_unfused * 1e3, 3),
         "rope_us": round(ms_rope * 1e3, 3),
         "kv_append_us": round(ms_append * 1e3, 3),

@@ -171,16 +171,24 @@ sd_status sd_verify_attention(const void* q, const sd_kv_cache* cache, void* out
                               int R, int Hq, float scale, void* workspace, size_t ws_bytes,
                               sd_stream_t stream);
 
-/* sd_verify_attention_ex flag: the block mask. */
+/* sd_verify_attention_ex flags: the block mask; the prefix read early. */
 #define SD_ATTN_BLOCK_MASK 1
+#define SD_ATTN_PREFIX_EARLY 2
 
 /*
  * sd_verify_attention with flags. SD_ATTN_BLOCK_MASK selects the block mask of
  * the block-diffusion drafts (Sec. 4 "Targets and drafts": a block of K = 16
  * tokens proposed at once): every new row sees the prefix and all R new rows,
- * n = 0 .. len[b] - 1, instead of n <= len[b] - R + i. Other bits:
- * SD_ERR_INVALID_ARG. Everything else as sd_verify_attention (which is this
- * call with flags 0).
+ * n = 0 .. len[b] - 1, instead of n <= len[b] - R + i.
+ * SD_ATTN_PREFIX_EARLY declares that the kernel issued just before this call
+ * on the stream writes neither this cache (its K / V rows, the new rows
+ * included) nor its len (true when a step's layers are issued back to back
+ * after their appends). For head_dim 128 and up to 16 new rows (32 when
+ * G * R > 32) the call is then a programmatic dependent launch that reads len
+ * and streams the whole cache while its predecessor still runs, and reads q
+ * only after the predecessor has completed; other shapes ignore the flag.
+ * Other bits: SD_ERR_INVALID_ARG. Everything else as sd_verify_attention
+ * (which is this call with flags 0).
  */
 sd_status sd_verify_attention_ex(const void* q, const sd_kv_cache* cache, void* out,
                                  int R, int Hq, float scale, int flags, void* workspace,

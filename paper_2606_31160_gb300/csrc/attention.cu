@@ -798,7 +798,7 @@ extern "C" sd_status sd_verify_attention_ex(const void* q, const sd_kv_cache* ca
                                             int R, int Hq, float scale, int flags, void* workspace,
                                             size_t ws_bytes, sd_stream_t stream) {
   if (!cache) return SD_ERR_INVALID_ARG;
-  if (flags & ~SD_ATTN_BLOCK_MASK) return SD_ERR_INVALID_ARG;
+  if (flags & ~(SD_ATTN_BLOCK_MASK | SD_ATTN_PREFIX_EARLY)) return SD_ERR_INVALID_ARG;
   const int block = (flags & SD_ATTN_BLOCK_MASK) ? 1 : 0;
   const int B = cache->batch, Hkv = cache->n_kv_heads, cap = cache->capacity, D = cache->head_dim;
   const sd_status shape = check_shape(B, R, Hq, Hkv, D, cap);
@@ -813,7 +813,7 @@ extern "C" sd_status sd_verify_attention_ex(const void* q, const sd_kv_cache* ca
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   {
     bool handled = false;
-    const sd_status s = sd_internal_verify_attention_tc(q, cache, out, R, Hq, scale_log2, block, st, &handled);
+    const sd_status s = sd_internal_verify_attention_tc(q, cache, out, R, Hq, scale_log2, flags, st, &handled);
     if (handled) return s;
   }
   Plan p;

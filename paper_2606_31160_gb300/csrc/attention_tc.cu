@@ -451,17 +451,25 @@ __device__ __forceinline__ void griddep_launch() {
 // a.early is set they are read before the programmatic-dependency wait.
 // Grid: (cluster size, Hkv * n_mblocks, B); m-block mb takes packed query rows
 // mb * kR .. mb * kR + kR - 1.
-template <int kR, bool kFused>
+template <int kR, int kMode>
 __global__ void __launch_bounds__(kThreads, 1)
     verify_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k128,
                           const __grid_constant__ CUtensorMap tm_v128, const TcArgs a,
                           const RopeTable tab) {
   using C = Cfg<kR>;
+  // kMode 1: the fused layer; 2: attention over a cache holding the new rows,
+  // merged like the fused layer's new keys; 0: attention with every key in the
+  // tensor-core loop (any R)
+  constexpr bool kFused = kMode == 1;
+  constexpr bool kNew = kMode != 0;  // the R new keys enter as S_new, not as tiles
+  // prefix (and len) before the dependency wait; the block mask
+  const bool early = kMode == 1 ? a.early != 0 : (kMode == 2 ? (a.early & 1) != 0 : false);
+  const bool block = kMode == 0 ? a.early != 0 : (kMode == 2 ? (a.early & 2) != 0 : false);
   constexpr int kS = C::kStages;
   constexpr int kRpt = C::kRpt;
   constexpr uint32_t kIdescS = umma_idesc(128, kR, 0, 0);
   constexpr uint32_t kIdescO = umma_idesc(128, kR, 1, 1);
-  constexpr int kTmemAlloc = kFused ? C::kTmemColsFused : C::kTmemCols;
+  constexpr int kTmemAlloc = kNew ? C::kTmemColsFused : C::kTmemCols;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
@@ -532,7 +540,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                  : "memory");
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
-  if (kFused && !a.early) griddep_wait();  // len, pos and the prefix may come from the previous kernel
+  if (kNew && !early) griddep_wait();  // len, pos and the prefix may come from the previous kernel
   int* s_len = reinterpret_cast<int*>(smem + C::kOffMisc + 12);
   if (threadIdx.x == 0) {
     *s_len = a.len[b];  // the scene's length advances at the producer's end
@@ -571,7 +579,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (!valid && rank == 0 && threadIdx.x == 0 && blockIdx.y == 0) sd_set_error(SD_DEVERR_LENGTH);
   }
   // the tensor-core loop covers the prefix (fused) or every key (standalone)
-  const int loop_keys = valid ? (kFused ? L_pre : n_keys) : 0;
+  const int loop_keys = valid ? (kNew ? L_pre : n_keys) : 0;
   const int nblk = (loop_keys + 31) / 32;
   // rank * nblk < 2^31 (16 ranks, nblk <= cap / 32): 32-bit division
   const int blk_begin = static_cast<int>((static_cast<uint32_t>(rank) * nblk) / static_cast<uint32_t>(csize));
@@ -622,7 +630,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // last scene) starts only when the previous layer frees its SMs; the
         // first head's CTAs bring that head's tiles of their own key range
         // into L2 meanwhile
-        if (kFused && a.early && kvh == 0 && b == static_cast<int>(gridDim.z) - 1 && a.Hkv > 1) {
+        if (kNew && early && kvh == 0 && b == static_cast<int>(gridDim.z) - 1 && a.Hkv > 1) {
           const int zl = b * a.Hkv + a.Hkv - 1;
           for (int t = 0; t < n_tiles; ++t)
 #pragma unroll
@@ -634,9 +642,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (rank == 0)
             for (int i = 0; i < a.R; ++i) {
               const long long row = static_cast<long long>(b) * a.R + i;
-              bulk_prefetch_l2(a.qw + (row * a.Hq + (a.Hkv - 1) * a.G) * kD, a.G * kD * 2);
-              bulk_prefetch_l2(a.k_new + (row * a.Hkv + a.Hkv - 1) * kD, kD * 2);
-              bulk_prefetch_l2(a.v_new + (row * a.Hkv + a.Hkv - 1) * kD, kD * 2);
+              bulk_prefetch_l2((kFused ? a.qw : a.q) + (row * a.Hq + (a.Hkv - 1) * a.G) * kD, a.G * kD * 2);
+              if (kFused) {
+                bulk_prefetch_l2(a.k_new + (row * a.Hkv + a.Hkv - 1) * kD, kD * 2);
+                bulk_prefetch_l2(a.v_new + (row * a.Hkv + a.Hkv - 1) * kD, kD * 2);
+              }
             }
         }
       }
@@ -674,7 +684,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // S(T) and PV(T) come from two warps (this one and the PV warp), so that
     // one batch is issued while the other executes; the whole warp waits and
     // one elected lane issues.
-    const bool snew = kFused && valid;
+    const bool snew = kNew && valid;
     bool arrived = false;
     if (n_tiles > 0 || snew) {
       mbar_wait(QFULL, 0);
@@ -806,8 +816,10 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
       for (int u = 0; u < kKvc; ++u) {
         const int idx = st + u * kSoftThreads;
-        has_kv[u] = kFused && valid && idx < a.R * 16;
-        kv_src[u] = ((static_cast<long long>(b) * a.R + (idx >> 4)) * a.Hkv + kvh) * kD + (idx & 15) * 8;
+        has_kv[u] = kNew && valid && idx < a.R * 16;
+        // fused: the raw rows [B][R][Hkv][D]; attention-only: cache rows L_pre + i
+        kv_src[u] = kFused ? ((static_cast<long long>(b) * a.R + (idx >> 4)) * a.Hkv + kvh) * kD + (idx & 15) * 8
+                           : ((static_cast<long long>(b) * a.Hkv + kvh) * a.cap + L_pre + (idx >> 4)) * kD + (idx & 15) * 8;
       }
       // Fused: iteration 0 runs BEFORE the dependency wait on whatever the
       // rows hold: it brings this code into the instruction cache and the rows
@@ -817,16 +829,18 @@ __global__ void __launch_bounds__(kThreads, 1)
       // nearly so: no warm-up pass, its rows are read once, after the wait
       const bool last_cluster = blockIdx.y == gridDim.y - 1 && blockIdx.z == gridDim.z - 1;
 #pragma unroll 1
-      for (int it = (kFused && !(a.early && last_cluster)) ? 0 : 1; it < 2; ++it) {
-        if (kFused && it == 1 && a.early) griddep_wait();  // the raw rows come from earlier kernels
+      for (int it = (kNew && !(early && last_cluster)) ? 0 : 1; it < 2; ++it) {
+        if (kNew && it == 1 && early) griddep_wait();  // the rows come from earlier kernels
         uint4 qv[kQc], kv[kKvc], vv[kKvc];
 #pragma unroll
         for (int u = 0; u < kQc; ++u)
           qv[u] = q_ok[u] ? __ldcg(reinterpret_cast<const uint4*>(q_src[u])) : make_uint4(0, 0, 0, 0);
 #pragma unroll
         for (int u = 0; u < kKvc; ++u) {
-          kv[u] = has_kv[u] ? __ldcg(reinterpret_cast<const uint4*>(a.k_new + kv_src[u])) : make_uint4(0, 0, 0, 0);
-          vv[u] = has_kv[u] ? __ldcg(reinterpret_cast<const uint4*>(a.v_new + kv_src[u])) : make_uint4(0, 0, 0, 0);
+          kv[u] = has_kv[u] ? __ldcg(reinterpret_cast<const uint4*>((kFused ? a.k_new : a.kc) + kv_src[u]))
+                            : make_uint4(0, 0, 0, 0);
+          vv[u] = has_kv[u] ? __ldcg(reinterpret_cast<const uint4*>((kFused ? a.v_new : a.vc) + kv_src[u]))
+                            : make_uint4(0, 0, 0, 0);
         }
         // (fused: M-RoPE of) the packed query rows, straight into the swizzled tile
 #pragma unroll
@@ -845,13 +859,15 @@ __global__ void __launch_bounds__(kThreads, 1)
         // past R stay zero (the merge reads all kMaxNew rows)
 #pragma unroll
         for (int u = 0; u < kKvc; ++u) {
-          if (!kFused) break;
+          if (!kNew) break;
           const int idx = st + u * kSoftThreads, i = idx >> 4, c = idx & 15;
           if (has_kv[u]) {
-            const float2* cs = cs_tab + i * 64 + c * 4;
             uint32_t w[4] = {kv[u].x, kv[u].y, kv[u].z, kv[u].w};
+            if (kFused) {
+              const float2* cs = cs_tab + i * 64 + c * 4;
 #pragma unroll
-            for (int j = 0; j < 4; ++j) w[j] = sd_rope_pair(w[j], cs[j].x, cs[j].y);
+              for (int j = 0; j < 4; ++j) w[j] = sd_rope_pair(w[j], cs[j].x, cs[j].y);
+            }
             st_shared_v4(base + C::kOffNewK + i * kNewRow + c * 16, w[0], w[1], w[2], w[3]);
             st_shared_v4(base + C::kOffP + (c >> 3) * C::kNewHalf + i * 128 + (((c & 7) ^ (i & 7)) << 4), w[0], w[1],
                          w[2], w[3]);
@@ -870,14 +886,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       // causal limit of each packed row: row p = i * G + g is new row i and
       // sees keys 0 .. L_prefix + i (Eq. verify's mask)
-      if (!kFused && st < kR)
-        row_lim[st] = a.early ? n_keys - 1 : min(n_keys - a.R + gdiv(mblock * kR + st), n_keys - 1);
+      if (!kNew && st < kR)
+        row_lim[st] = block ? n_keys - 1 : min(n_keys - a.R + gdiv(mblock * kR + st), n_keys - 1);
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
       named_bar_sync(2, kSoftThreads);  // Q is complete; the rotation table is no longer read
       if (st == 0) {
         mbar_arrive(QFULL);
         // every older kernel has finished: the next layer may launch
-        if (kFused) griddep_launch();
+        if (kNew) griddep_launch();
         // with several m-blocks the head's raw key rows are read by several
         // clusters: the last of the head's CTAs to have read them writes the
         // rotated rows back (the fence orders this CTA's reads before its ticket)
@@ -917,14 +933,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     auto tile_mask = [&](int key0, int j0, bool (&ok)[16]) {
       const int key = key0 + kl;
       const bool key_ok = key < key_end;
-      const bool tail = !kFused && key0 + kStageKeys - 1 > L_prefix;
+      const bool tail = !kNew && key0 + kStageKeys - 1 > L_prefix;
 #pragma unroll
       for (int j = 0; j < 16; ++j) {
         ok[j] = key_ok;
         if (tail) ok[j] = ok[j] && key <= row_lim[row0 + j0 + j];
       }
     };
-    if (kFused) {
+    if (kNew) {
       // references: the larger score of each row against its own new key and
       // new key 0 (keys the row sees, so its largest weight is at least about
       // 1 and its sum cannot vanish), taken while S(0) and S(1) run; bf16 dot
@@ -1059,7 +1075,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             lp[j0 + j + 1] += sd_bf16_hi(w);
           }
           if (T >= 2 && j0 == 0) mbar_wait(PVDONE(T - 2), ring_parity(T - 2));  // PV(T - 2) has read P buffer bb
-          if (kFused && T == 0 && j0 == 0 && valid) mbar_wait(SNEW, 0);  // S_new has read its operand
+          if (kNew && T == 0 && j0 == 0 && valid) mbar_wait(SNEW, 0);  // S_new has read its operand
           const int ch = (row0 + j0) >> 3;
           st_shared_v4(prow + ((ch ^ sw) << 4), pw[0], pw[1], pw[2], pw[3]);
           st_shared_v4(prow + (((ch + 1) ^ sw) << 4), pw[4], pw[5], pw[6], pw[7]);
@@ -1139,7 +1155,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // the new-key scores of the rows this CTA merges, from S_new^T (new key n
     // on lane n of the first TMEM lane quarter), scaled, causally masked
     float* s_new = reinterpret_cast<float*>(smem + C::kNewS);  // [my_rows][R]
-    if (kFused && valid && quarter == 0 && half == 0) {
+    if (kNew && valid && quarter == 0 && half == 0) {
       mbar_wait(SNEW, 0);
       tc_fence_after();
 #pragma unroll 1
@@ -1153,8 +1169,10 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
           const int rr = rr0 + j, p = mblock * kR + mrow0 + rr;
+          // causal: row p = i * G + g sees new keys 0..i; block mask: all R
           if (rr < my_rows && lane < a.R)
-            s_new[rr * a.R + lane] = (p < a.M && lane <= gdiv(p)) ? __uint_as_float(v[j]) * a.scale_log2 : -INFINITY;
+            s_new[rr * a.R + lane] =
+                (p < a.M && (block || lane <= gdiv(p))) ? __uint_as_float(v[j]) * a.scale_log2 : -INFINITY;
         }
       }
     }
@@ -1234,7 +1252,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // used the row's reference (the common case: the second pass is rare), the
     // partials then add with the one weight 2^(ref - M); otherwise every
     // partial takes its own weight.
-    const int n_new = (kFused && valid) ? a.R : 0;
+    const int n_new = (kNew && valid) ? a.R : 0;
     const int rr = st >> 6, d = 2 * (st & 63);  // my_rows <= 4 here; more rows loop below
     float nx = 0.f, ny = 0.f, nl = 0.f, mloc = -INFINITY, rref = -INFINITY;
     if (rr < my_rows) {
@@ -1376,13 +1394,16 @@ struct DevState {
 
 template <int kR>
 bool set_attributes(int* active) {
-  auto kern = verify_attn_tc_kernel<kR, false>;
-  auto kern_f = verify_attn_tc_kernel<kR, true>;
+  auto kern = verify_attn_tc_kernel<kR, 0>;
+  auto kern_f = verify_attn_tc_kernel<kR, 1>;
+  auto kern_n = verify_attn_tc_kernel<kR, 2>;
   constexpr int smem = Cfg<kR>::kSmemBytes;
   if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess ||
       cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess ||
       cudaFuncSetAttribute(kern_f, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess ||
-      cudaFuncSetAttribute(kern_f, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess) {
+      cudaFuncSetAttribute(kern_f, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess ||
+      cudaFuncSetAttribute(kern_n, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess ||
+      cudaFuncSetAttribute(kern_n, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess) {
     (void)cudaGetLastError();
     return false;
   }
@@ -1501,7 +1522,7 @@ bool sd_internal_tc_serves(int B, int R, int Hq, int Hkv, int D, int cap) {
   return tc_plan(B, R, Hq, Hkv, D, cap).cs > 0;
 }
 
-template <int kR, bool kFused>
+template <int kR, int kMode>
 static sd_status launch_tc(const sd_kv_cache* cache, const TcArgs& a, const RopeTable& tab,
                            const TcPlan& plan, bool pdl, cudaStream_t stream) {
   const int B = cache->batch, Hkv = cache->n_kv_heads, cap = cache->capacity;
@@ -1522,32 +1543,46 @@ static sd_status launch_tc(const sd_kv_cache* cache, const TcArgs& a, const Rope
   cfg.stream = stream;
   cfg.attrs = attr;
   cfg.numAttrs = pdl ? 2 : 1;
-  if (cudaLaunchKernelEx(&cfg, verify_attn_tc_kernel<kR, kFused>, k128, v128, a, tab) != cudaSuccess) {
+  if (cudaLaunchKernelEx(&cfg, verify_attn_tc_kernel<kR, kMode>, k128, v128, a, tab) != cudaSuccess) {
     (void)cudaGetLastError();
     return SD_ERR_CUDA;
   }
   return SD_OK;
 }
 
-template <bool kFused>
+template <int kMode>
 static sd_status launch_plan(const sd_kv_cache* cache, const TcArgs& a, const RopeTable& tab,
                              const TcPlan& plan, bool pdl, cudaStream_t stream) {
-  return plan.rows == 32 ? launch_tc<32, kFused>(cache, a, tab, plan, pdl, stream)
-                         : launch_tc<64, kFused>(cache, a, tab, plan, pdl, stream);
+  return plan.rows == 32 ? launch_tc<32, kMode>(cache, a, tab, plan, pdl, stream)
+                         : launch_tc<64, kMode>(cache, a, tab, plan, pdl, stream);
 }
 
-// Routed here by sd_verify_attention for head_dim 128 and G * R <= 128.
+// Routed here by sd_verify_attention for head_dim 128 and G * R <= 128. Up to
+// kMaxNew new rows (and cluster sizes with csize + R <= 32) take the kernel
+// whose tensor-core loop covers the prefix only and whose new rows enter as
+// S_new (as in the fused layer), with the prefix optionally streamed before
+// the dependency wait (SD_ATTN_PREFIX_EARLY); other shapes take the kernel
+// whose loop covers every key (the flag is then a promise it does not need).
 sd_status sd_internal_verify_attention_tc(const void* q, const sd_kv_cache* cache, void* out,
-                                          int R, int Hq, float scale_log2, int block, cudaStream_t stream,
+                                          int R, int Hq, float scale_log2, int flags, cudaStream_t stream,
                                           bool* handled) {
   *handled = false;
   const int B = cache->batch, Hkv = cache->n_kv_heads;
-  const TcPlan plan = tc_plan(B, R, Hq, Hkv, cache->head_dim, cache->capacity);
+  const bool block = (flags & SD_ATTN_BLOCK_MASK) != 0, early = (flags & SD_ATTN_PREFIX_EARLY) != 0;
+  TcPlan plan;
+  int mode = 0;
+  if (R <= 32) {
+    plan = tc_plan(B, R, Hq, Hkv, cache->head_dim, cache->capacity, 32 - R);
+    if (plan.cs > 0 && R <= (plan.rows == 32 ? Cfg<32>::kMaxNew : Cfg<64>::kMaxNew)) mode = 2;
+  }
+  if (mode == 0) plan = tc_plan(B, R, Hq, Hkv, cache->head_dim, cache->capacity);
   if (plan.cs <= 0) return SD_OK;
   TcArgs a = {};
   a.q = static_cast<const __nv_bfloat16*>(q);
   a.out = static_cast<__nv_bfloat16*>(out);
   a.len = cache->len;
+  a.kc = static_cast<__nv_bfloat16*>(cache->k);
+  a.vc = static_cast<__nv_bfloat16*>(cache->v);
   a.R = R;
   a.Hq = Hq;
   a.Hkv = Hkv;
@@ -1556,11 +1591,15 @@ sd_status sd_internal_verify_attention_tc(const void* q, const sd_kv_cache* cach
   a.inv_g = 1.0f / static_cast<float>(a.G);
   a.cap = cache->capacity;
   a.n_mblocks = plan.mblocks;
-  a.early = block;  // the standalone kernel's block mask
   a.scale_log2 = scale_log2;
   RopeTable tab = {};
   *handled = true;
-  return launch_plan<false>(cache, a, tab, plan, false, stream);
+  if (mode == 2) {
+    a.early = (early ? 1 : 0) | (block ? 2 : 0);
+    return launch_plan<2>(cache, a, tab, plan, early, stream);
+  }
+  a.early = block ? 1 : 0;  // the all-keys kernel's block mask
+  return launch_plan<0>(cache, a, tab, plan, false, stream);
 }
 
 // The fused verify layer (rope + append + attention) on the tcgen05 path.
@@ -1602,5 +1641,5 @@ sd_status sd_internal_verify_layer_tc(void* q, void* k_new, const void* v_new, c
   a.n_mblocks = plan.mblocks;
   a.scale_log2 = scale_log2;
   *handled = true;
-  return launch_plan<true>(cache, a, tab, plan, early != 0, stream);
+  return launch_plan<1>(cache, a, tab, plan, early != 0, stream);
 }

@@ -40,7 +40,7 @@ cudaError_t sd_take_error_budget(uint32_t* bits);
 // Verify attention on the tcgen05 path (attention_tc.cu). Sets *handled when
 // the shape is one it serves (head_dim 128, G * R <= 32) and it launched.
 sd_status sd_internal_verify_attention_tc(const void* q, const sd_kv_cache* cache, void* out,
-                                          int R, int Hq, float scale_log2, int block, cudaStream_t stream,
+                                          int R, int Hq, float scale_log2, int flags, cudaStream_t stream,
                                           bool* handled);
 // Whether the tcgen05 path serves this shape on the current device.
 bool sd_internal_tc_serves(int B, int R, int Hq, int Hkv, int D, int cap);

@@ -208,13 +208,16 @@ _attn_ws = {}
 
 
 SD_ATTN_BLOCK_MASK = 1
+SD_ATTN_PREFIX_EARLY = 2
 SD_LAYER_BLOCK_MASK = 2
 
 
-def verify_attention(q, cache, out=None, scale=0.0, ws=None, block=False):
+def verify_attention(q, cache, out=None, scale=0.0, ws=None, block=False, early=False):
     """Causal GQA verify attention of q [B,R,Hq,D] (rotated) over the cache (appended).
     ws: the split-merge workspace (see sd_verify_attention_workspace); when None a
-    zero-filled one is kept per (device, shape) and reused by later calls."""
+    zero-filled one is kept per (device, shape) and reused by later calls.
+    block=True sets SD_ATTN_BLOCK_MASK; early=True sets SD_ATTN_PREFIX_EARLY (the
+    previous kernel on the stream writes neither this cache nor its len)."""
     B, R, Hq, D = q.shape
     if cache.shape[0] != B or cache.shape[3] != D:
         raise ValueError("q and cache disagree")
@@ -230,7 +233,8 @@ def verify_attention(q, cache, out=None, scale=0.0, ws=None, block=False):
     nbytes = ws.numel() * ws.element_size() if ws is not None else 0
     _check(lib().sd_verify_attention_ex(_dev(q, "q", torch.bfloat16), cache.struct,
                                         _dev(out, "out", torch.bfloat16), R, Hq, float(scale),
-                                        SD_ATTN_BLOCK_MASK if block else 0, wp, nbytes, _stream()),
+                                        (SD_ATTN_BLOCK_MASK if block else 0) | (SD_ATTN_PREFIX_EARLY if early else 0),
+                                        wp, nbytes, _stream()),
            "sd_verify_attention")
     return out
 

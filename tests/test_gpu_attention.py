@@ -137,3 +137,31 @@ def test_workspace_is_required_and_left_zeroed():
     n_sp_part = need - units * 8 - 256
     cnt = ws[n_sp_part:n_sp_part + units * 8].view(torch.int32)
     assert int(cnt.abs().sum()) == 0
+
+
+@pytest.mark.parametrize("B,K", [(1, 7), (3, 7), (2, 8), (1, 16)])
+def test_back_to_back_attention_with_early_prefix(B, K):
+    # sd_verify_attention over a step's appended caches issued back to back:
+    # with SD_ATTN_PREFIX_EARLY every call after the first streams its cache
+    # before the previous one finishes; the bits must equal the plain chain's
+    R = K + 1
+    prefix = [4096 - 41 * s for s in range(B)]
+    qpos = np.stack([workloads.text_positions(int(p) + 1, R) for p in prefix])
+    cases = [workloads.verify_case(workloads.TARGET_LAYER, B=B, Hq=32, Hkv=8, D=128, prefix=prefix, K=K,
+                                   sections=(16, 24, 24), base=1e6, query_pos=qpos, cap=max(prefix) + R + 8,
+                                   layer=700 + l, tail_fill=float("nan")) for l in range(4)]
+    state = []
+    for c in cases:
+        q, _, cache, _ = run_verify_layer(c)  # rotated q, appended cache
+        state.append((q, cache))
+    runs = []
+    for early in (False, True):
+        outs = [sd.verify_attention(q, cache, early=early and l > 0) for l, (q, cache) in enumerate(state)]
+        torch.cuda.synchronize()
+        runs.append(outs)
+    for l in range(len(cases)):
+        assert torch.equal(runs[0][l], runs[1][l])
+    q, cache = state[2]
+    ref, _ = _oracle_out(q, cache)
+    _assert_close(to64(runs[1][2]), ref)
+    assert sd.get_device_error() == 0
