@@ -266,9 +266,9 @@ size_t sd_verify_layer_workspace(int B, int R, int Hq, int Hkv, int D, int capac
  *   k_new and v_new are read only after the predecessor has completed.
  *   SD_LAYER_BLOCK_MASK: the attention uses the block mask (as
  *   SD_ATTN_BLOCK_MASK of sd_verify_attention_ex).
- * For head_dim 128, G * R <= 128 and R <= 31 (R <= 16 when G * R <= 32) and
- * without SD_LAYER_BLOCK_MASK this is one tcgen05 kernel; other shapes run
- * the three kernels in sequence. A scene whose append would pass the
+ * For head_dim 128, G * R <= 128 and R <= 31 (R <= 16 when G * R <= 32) this
+ * is one tcgen05 kernel (the block mask only when G * R > 32); other shapes
+ * run the three kernels in sequence. A scene whose append would pass the
  * capacity sets SD_DEVERR_KV_OVERFLOW and is left untouched.
  */
 sd_status sd_verify_layer(void* q, void* k_new, const void* v_new, const int32_t* pos,

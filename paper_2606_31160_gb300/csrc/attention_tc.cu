@@ -428,8 +428,9 @@ struct TcArgs {
   const int32_t* pos;       // [B][R][3]
   uint32_t* ticket;         // [B] per-scene CTA tickets (zeroed, re-armed)
   uint32_t* kv_ticket;      // [B][Hkv] read-before-write-back tickets (several m-blocks)
-  // fused kernel: prefix, len and pos may be read before the dependency wait;
-  // standalone kernel: the block mask (every new row sees all R new rows)
+  // kernels whose new keys enter as S_new: bit 0 = prefix, len (and pos) may
+  // be read before the dependency wait, bit 1 = the block mask (every new row
+  // sees all R new rows); the all-keys kernel: nonzero = the block mask
   int early;
   int R, Hq, Hkv, G, M, cap, n_mblocks;
   float inv_g;              // 1 / G: p / G == int((p + 0.5) / G) exactly for the p < 128 used here
@@ -463,8 +464,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   constexpr bool kFused = kMode == 1;
   constexpr bool kNew = kMode != 0;  // the R new keys enter as S_new, not as tiles
   // prefix (and len) before the dependency wait; the block mask
-  const bool early = kMode == 1 ? a.early != 0 : (kMode == 2 ? (a.early & 1) != 0 : false);
-  const bool block = kMode == 0 ? a.early != 0 : (kMode == 2 ? (a.early & 2) != 0 : false);
+  const bool early = kNew && (a.early & 1) != 0;
+  // (the fused layer's 32-row tile takes no block mask: its callers are the
+  // target's causal verify steps; the host sends block-masked 32-row layers
+  // through the separate kernels)
+  const bool block = kMode == 0 ? a.early != 0 : ((kMode == 2 || kR == 64) && (a.early & 2) != 0);
   constexpr int kS = C::kStages;
   constexpr int kRpt = C::kRpt;
   constexpr uint32_t kIdescS = umma_idesc(128, kR, 0, 0);
@@ -1609,15 +1613,13 @@ sd_status sd_internal_verify_layer_tc(void* q, void* k_new, const void* v_new, c
                                       int block, cudaStream_t stream, bool* handled) {
   *handled = false;
   const int B = cache->batch, Hkv = cache->n_kv_heads;
-  // the block mask (a draft's pattern, not the target's verify) takes the
-  // three separate kernels: the fused kernel's new-key merge stays causal
-  if (block) return SD_OK;
   // the new rows are held in shared memory (16 with the 32-row tile, 32 with
   // the 64-row tile) and merged in the lanes of one warp with the partials
   if (R > 32) return SD_OK;
   const TcPlan plan = tc_plan(B, R, Hq, Hkv, cache->head_dim, cache->capacity, 32 - R);
   if (plan.cs <= 0) return SD_OK;
   if (R > (plan.rows == 32 ? Cfg<32>::kMaxNew : Cfg<64>::kMaxNew)) return SD_OK;
+  if (block && plan.rows == 32) return SD_OK;  // the 32-row fused kernel is causal only
   TcArgs a = {};
   a.q = static_cast<const __nv_bfloat16*>(q);
   a.out = static_cast<__nv_bfloat16*>(out);
@@ -1630,7 +1632,7 @@ sd_status sd_internal_verify_layer_tc(void* q, void* k_new, const void* v_new, c
   a.pos = pos;
   a.ticket = ticket;
   a.kv_ticket = ticket + B;
-  a.early = early ? 1 : 0;
+  a.early = (early ? 1 : 0) | (block ? 2 : 0);  // prefix before the wait; the block mask
   a.R = R;
   a.Hq = Hq;
   a.Hkv = Hkv;
