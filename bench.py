@@ -1,7 +1,7 @@
 """Benchmark of the verify step on GB300: prints ONE JSON line.
 
 Workload: the 8B-class target verify step of the paper's speculative-decoding
-loop (Sec. 2.2 Eq. verify; target shape from Sec. 4 "Targets and drafts":
+loop (Sec. 3.2 Eq. verify; target shape from Sec. 5 "Targets and drafts":
 Qwen3-VL-8B backbone, 36 layers). Per scene and step, every one of the 36
 layers runs, on its own KV cache (L = 4096 prefix = 4 cameras x 896 patches +
 512 text tokens, 32 query / 8 KV heads x 128, bf16):
@@ -23,6 +23,7 @@ independent: weak scaling, no data-path collective).
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
     python bench.py --sweep     # sd_verify_attention over the batched sweep grid
+    python bench.py --floor     # launch and streaming floors of the chained layers
 """
 
 import argparse
@@ -476,7 +477,7 @@ def time_stochastic_step(device, layers=LAYERS):
 
 
 def time_long_draft_step(device, K_=16, layers=LAYERS):
-    """The verify step of a block-diffusion draft (Sec. 4: blocks of K = 16
+    """The verify step of a block-diffusion draft (Sec. 5: blocks of K = 16
     tokens): 36 fused target layers at B = 1, L = 4096, R = 17 (68 packed rows
     per KV head: two 64-row m-blocks), one cache per layer, then the greedy
     accept over bf16 logits [1][17][151936] and the rollback, in a graph.
@@ -618,6 +619,9 @@ def main():
     ap.add_argument("--sweep-b", type=int, nargs="*", default=None, help="restrict the sweep's batch sizes")
     ap.add_argument("--sweep-l", type=int, nargs="*", default=None, help="restrict the sweep's prefix lengths")
     ap.add_argument("--sweep-k", type=int, nargs="*", default=None, help="restrict the sweep's draft lengths")
+    ap.add_argument("--floor", action="store_true",
+                    help="measure the platform floors of the chained layers (empty dependent launches, "
+                         "TMA streams of one layer's bytes) and print one JSON line per point; no bench line")
     ap.add_argument("--only", choices=["attention", "layer", "accept", "step", "sample"], default=None,
                     help="profiling mode: run one kernel family eagerly `steps` times on the "
                          "target-layer workload (sample: the stochastic-acceptance workload) "
@@ -635,6 +639,8 @@ def main():
         return profile_only(args)
     if args.sweep:
         return sweep(args)
+    if args.floor:
+        return floor(args)
 
     import torch.distributed as dist
     torch.cuda.set_device(local)
@@ -884,6 +890,64 @@ def sweep(args):
                                             "bytes": nbytes, "copies": copies}}), flush=True)
                 del caches, outs, ws, g
                 torch.cuda.empty_cache()
+
+
+# The 32-row fused layer kernel's launch shape: 8 heads x a cluster of 8 CTAs
+# of 352 threads, 230,976 bytes of dynamic shared memory, 256 tensor-memory
+# columns.
+FLOOR_SHAPE = {"ctas": 64, "cluster": 8, "threads": 352, "smem": 230976, "tmem_cols": 256}
+
+
+def floor(args):
+    """Platform floors of the chained verify layers (one JSON line each, no
+    bench line). (1) A chain of 36 launches that do no work, in the fused
+    layer kernel's launch shape, each a programmatic dependent launch of the
+    one before (or plain launches): the release latency that every chained
+    layer pays. (2) A chain of 36 launches that only stream one target layer's
+    bytes (17,170,432 B as rows of 256 B, a distinct slice per launch, 618 MB
+    in all: larger than L2) through shared memory by TMA, over 64 to 304 CTAs,
+    with the dependency wait at the start, after the first ring fill (as the
+    layer kernel's early prefix), at the end, or no dependent launch at all.
+    CUDA events around graph replays on the floor library's own stream."""
+    import ctypes
+    from paper_2606_31160_gb300 import build
+    build.build()
+    torch.cuda.set_device(0)
+    device = torch.device("cuda", 0)
+    torch.cuda.init()
+    lib = ctypes.CDLL(build.FLOOR_LIB)
+    lib.sdfloor_empty_chain.restype = ctypes.c_int
+    lib.sdfloor_empty_chain.argtypes = [ctypes.c_int] * 8 + [ctypes.POINTER(ctypes.c_float)]
+    lib.sdfloor_stream_chain.restype = ctypes.c_int
+    lib.sdfloor_stream_chain.argtypes = [ctypes.c_void_p, ctypes.c_longlong, ctypes.c_int, ctypes.c_int,
+                                         ctypes.c_int, ctypes.c_int, ctypes.POINTER(ctypes.c_float)]
+    peak, peak_kind = measured_peaks()
+    us = ctypes.c_float(0.0)
+    sh = FLOOR_SHAPE
+    for pdl in (1, 0):
+        for tmem in (sh["tmem_cols"], 0):
+            rc = lib.sdfloor_empty_chain(LAYERS, sh["ctas"], sh["cluster"], sh["threads"], sh["smem"], tmem, pdl,
+                                         200, ctypes.byref(us))
+            print(json.dumps({"floor": "empty", "layers": LAYERS, "ctas": sh["ctas"], "cluster": sh["cluster"],
+                              "threads": sh["threads"], "smem": sh["smem"], "tmem_cols": tmem, "pdl": pdl,
+                              "us_per_launch": round(us.value, 3), "rc": rc}), flush=True)
+    nbytes = layer_bytes()
+    rows = nbytes // 256
+    buf = torch.zeros(LAYERS * rows * 128, dtype=torch.bfloat16, device=device)
+    torch.cuda.synchronize()
+    names = {-1: "no dependent launch", 0: "wait at start", 1: "wait after first ring fill", 2: "wait at end"}
+    for ctas in (64, 128, 152, 304):
+        for waitpos in (-1, 0, 1, 2):
+            rc = lib.sdfloor_stream_chain(ctypes.c_void_p(buf.data_ptr()), rows, LAYERS, ctas, waitpos, 50,
+                                          ctypes.byref(us))
+            gbs = nbytes / (us.value * 1e-6) / 1e9 if us.value > 0 else 0.0
+            print(json.dumps({"floor": "stream", "layers": LAYERS, "bytes_per_launch": nbytes, "ctas": ctas,
+                              "wait": names[waitpos], "us_per_launch": round(us.value, 3), "gbs": round(gbs, 1),
+                              "frac": round(gbs / peak, 4), "peak": peak, "peak_kind": peak_kind, "rc": rc}),
+                  flush=True)
+    err = lib.sdfloor_take_error()
+    print(json.dumps({"floor": "done", "device_error": err}), flush=True)
+    return 0 if err == 0 else 1
 
 
 def profile_only(args):

@@ -3,10 +3,10 @@
  * speculative decoding ("Reasoning-aware Speculative Decoding for Efficient
  * VLA Models in Autonomous Driving", arxiv 2606.31160).
  *
- * In the paper's propose / verify / commit loop (Sec. 2.2) a small draft
+ * In the paper's propose / verify / commit loop (Sec. 3.2) a small draft
  * proposes K tokens and the unmodified multimodal target scores them in one
  * pass. This library is the data-parallel hot path of that pass: the rotary
- * position encoding of the new rows (Sec. 2.3, Sec. 3.2), the KV-cache append
+ * position encoding of the new rows (Sec. 3.3, Sec. 4.2), the KV-cache append
  * and rollback (Eq. commit), the causally masked GQA attention of the K + 1
  * verify rows (Eq. verify), and the two acceptance rules (Eqs. accept,
  * commit; Leviathan/Chen rejection sampling, cited in Sec. 1-2).
@@ -83,8 +83,8 @@ const char* sd_status_str(sd_status s);
 const char* sd_version(void);
 
 /*
- * M-RoPE rotation of the new Q and K rows, in place (Sec. 2.3 Eq. rope-3d;
- * Sec. 3.2 Eqs. axis-assign, mrope-phase).
+ * M-RoPE rotation of the new Q and K rows, in place (Sec. 3.3 Eq. rope-3d;
+ * Sec. 4.2 Eqs. axis-assign, mrope-phase).
  *   q:   [B][R][Hq][D] bf16, k: [B][R][Hkv][D] bf16 (either may be NULL when
  *        its head count is 0).
  *   pos: [B][R][3] int32 (t, h, w) coordinates of each row, device memory.
@@ -101,7 +101,7 @@ sd_status sd_rope_apply(void* q, void* k, int B, int R, int Hq, int Hkv, int D,
                         int interleaved, float base, sd_stream_t stream);
 
 /*
- * FlatRoPE / plain 1D RoPE (Sec. 2.3 Eq. rope-1d; Sec. 3.2 Eq. flatrope-proj):
+ * FlatRoPE / plain 1D RoPE (Sec. 3.3 Eq. rope-1d; Sec. 4.2 Eq. flatrope-proj):
  * the same rotation with every axis at the sequence index pos1d[b][r]
  * (device int32[B][R]). Equal, bit for bit, to sd_rope_apply with
  * pos = (m, m, m) under any section layout.
@@ -141,7 +141,7 @@ sd_status sd_kv_rollback(int32_t* len, int count, int B, const int32_t* committe
 size_t sd_verify_attention_workspace(int B, int R, int Hq, int Hkv, int D, int capacity);
 
 /*
- * Verify attention (Eq. verify, Sec. 2.2): for scene b, query head h (KV head
+ * Verify attention (Eq. verify, Sec. 3.2): for scene b, query head h (KV head
  * g = h / G) and row i < R,
  *   o[b][i][h] = softmax_n( q[b][i][h] . k[b][g][n] * scale ) v[b][g][n],
  *   n = 0 .. len[b] - R + i
@@ -177,7 +177,7 @@ sd_status sd_verify_attention(const void* q, const sd_kv_cache* cache, void* out
 
 /*
  * sd_verify_attention with flags. SD_ATTN_BLOCK_MASK selects the block mask of
- * the block-diffusion drafts (Sec. 4 "Targets and drafts": a block of K = 16
+ * the block-diffusion drafts (Sec. 5 "Targets and drafts": a block of K = 16
  * tokens proposed at once): every new row sees the prefix and all R new rows,
  * n = 0 .. len[b] - 1, instead of n <= len[b] - R + i.
  * SD_ATTN_PREFIX_EARLY declares that the kernel issued just before this call
@@ -209,7 +209,7 @@ sd_status sd_verify_attention_ex(const void* q, const sd_kv_cache* cache, void* 
 sd_status sd_set_cluster_size(int cluster_size);
 
 /*
- * Attention budget of the verify rows (Sec. 3.2 "Empirical confirmation",
+ * Attention budget of the verify rows (Sec. 4.2 "Empirical confirmation",
  * Table tab:attn-budget), a diagnostic beside the verify path. For scene b,
  * query head h and row i, with p the softmax of q . k * scale over the keys
  * row i sees (0 .. len[b] - R + i, as in sd_verify_attention) and
@@ -242,9 +242,9 @@ sd_status sd_attention_budget(const void* q, const sd_kv_cache* cache, int R, in
 size_t sd_verify_layer_workspace(int B, int R, int Hq, int Hkv, int D, int capacity);
 
 /*
- * One attention layer of the verify pass in one call (Eq. verify, Sec. 2.2):
- * the M-RoPE rotation of the R new query and key rows (Sec. 2.3 Eq. rope-3d,
- * Sec. 3.2 Eqs. axis-assign, mrope-phase), their append to the cache (Eq.
+ * One attention layer of the verify pass in one call (Eq. verify, Sec. 3.2):
+ * the M-RoPE rotation of the R new query and key rows (Sec. 3.3 Eq. rope-3d,
+ * Sec. 4.2 Eqs. axis-assign, mrope-phase), their append to the cache (Eq.
  * commit) and the verify attention over the prefix plus the new rows.
  * Equal to sd_rope_apply(q, k_new, ...) + sd_kv_append(cache, k_new, v_new)
  * + sd_verify_attention(q, cache, out): q and k_new are rotated in place,
@@ -282,7 +282,7 @@ sd_status sd_verify_layer(void* q, void* k_new, const void* v_new, const int32_t
 size_t sd_accept_greedy_workspace(int B, int K, int V);
 
 /*
- * Greedy acceptance (Eqs. verify, accept, commit; Sec. 3.3 Eq. accept-length).
+ * Greedy acceptance (Eqs. verify, accept, commit; Sec. 4.3 Eq. accept-length).
  *   logits: [B][K+1][V] of `dtype` (SD_BF16 or SD_F32).
  *   draft:  [B][K] int32 draft tokens.
  * Outputs (device): argmax [B][K+1] int32, the lowest index among equal

@@ -6,13 +6,13 @@ restatement of what the GPU path computes, written from the paper
 Driving", arxiv 2606.31160):
 
   rope.py       1D RoPE (Eq. rope-1d), 3D M-RoPE (Eqs. rope-3d, axis-assign,
-                mrope-phase) and FlatRoPE (Eq. flatrope-proj), Sec. 2.3 / 3.2
-  attention.py  causal GQA attention of the K+1 verify rows (Eq. verify, Sec. 2.2)
+                mrope-phase) and FlatRoPE (Eq. flatrope-proj), Sec. 3.3 / 4.2
+  attention.py  causal GQA attention of the K+1 verify rows (Eq. verify, Sec. 3.2)
   accept.py     greedy longest-prefix acceptance + bonus (Eqs. accept, commit)
                 and Leviathan/Chen rejection sampling (cited in Sec. 1 and 2)
   kv.py         KV-cache append and rollback to the committed length (Eq. commit)
   budget.py     per-segment attention mass and normalised entropy of the verify
-                rows (Sec. 3.2, Table tab:attn-budget)
+                rows (Sec. 4.2, Table tab:attn-budget)
 
 Only tests/, __graft_entry__.smoke() and bench.py (its cpu_baseline leg and
 its --impl reference arm) may import it. The CUDA library and its Python

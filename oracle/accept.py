@@ -1,6 +1,6 @@
 """Acceptance rules of the verify step, float64 (test infrastructure, oracle only).
 
-Greedy (Sec. 2.2, Eqs. verify, accept, commit; Sec. 3.3, Eq. accept-length):
+Greedy (Sec. 3.2, Eqs. verify, accept, commit; Sec. 4.3, Eq. accept-length):
   r*_j = argmax_v logits[j, v]                       (Eq. verify)
   l    = max{l <= K : r^_j = r*_j for all j <= l}    (Eq. accept)
   emit (r^_1 .. r^_l, r*_{l+1}), t <- t + l + 1      (Eq. commit)

@@ -1,6 +1,6 @@
 """Causal GQA attention of the K+1 verify rows, float64 (test infrastructure, oracle only).
 
-Sec. 2.2, Eq. verify: the target scores the K draft tokens in one batched
+Sec. 3.2, Eq. verify: the target scores the K draft tokens in one batched
 forward; the distribution at draft position j conditions on the committed
 prefix r_{1:t} and the earlier drafts r^_{<j}. Inside each attention layer
 that is one causally masked attention of R = K + 1 new query rows against
@@ -16,7 +16,7 @@ Readings taken where the paper is silent:
   * Grouped-query attention with contiguous groups: q head h reads KV head
     floor(h / G), G = Hq / Hkv.
   * Block mask (block=True): the variant of the block-diffusion drafts
-    (Sec. 4, "Targets and drafts": a block of K = 16 tokens proposed at
+    (Sec. 5, "Targets and drafts": a block of K = 16 tokens proposed at
     once), where every new row also sees the new rows after it: row i sees
     keys 0 .. L_b + R - 1.
 

@@ -1,6 +1,6 @@
 """Attention budget of the verify rows, float64 (test infrastructure, oracle only).
 
-Sec. 3.2 ("Empirical confirmation") and Table tab:attn-budget: how a query
+Sec. 4.2 ("Empirical confirmation") and Table tab:attn-budget: how a query
 row's attention mass divides among the visual tokens, the trajectory / text
 tokens of the prompt and the tokens generated in this step, and how spread
 the attention is among the non-visual tokens.

@@ -1,6 +1,6 @@
 """KV-cache append and rollback (test infrastructure, oracle only).
 
-Sec. 2.2, Eq. commit: an iteration commits l + 1 tokens and advances
+Sec. 3.2, Eq. commit: an iteration commits l + 1 tokens and advances
 t_{i+1} = t_i + l_i + 1. The verify pass appended the keys/values of all
 R = K + 1 rows; of those, the rows that stay valid are the last committed
 token and the l accepted drafts, i.e. n_emit = l + 1 rows. The rejected rows'

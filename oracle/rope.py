@@ -1,22 +1,22 @@
 """Rotary position embeddings in float64 (test infrastructure, oracle only).
 
-Sec. 2.3, Eq. rope-1d: 1D RoPE rotates each adjacent pair (2d, 2d+1) of a
+Sec. 3.3, Eq. rope-1d: 1D RoPE rotates each adjacent pair (2d, 2d+1) of a
 head vector by the angle m * w_d, w_d = b^(-2d/h); the rotation is the
 block-diagonal direct sum of 2x2 rotations.
 
-Sec. 2.3, Eq. rope-3d, and Sec. 3.2, Eqs. axis-assign and mrope-phase: 3D
+Sec. 3.3, Eq. rope-3d, and Sec. 4.2, Eqs. axis-assign and mrope-phase: 3D
 M-RoPE gives each token a (T, H, W) coordinate. Rotary pair d takes its angle
 from the coordinate of axis a(d): phi_d = theta_d * p_{a(d)}, with a(d)
 blocked over mrope_section = (s_T, s_H, s_W) or interleaved as d mod 3.
 
-Sec. 3.2, Eq. flatrope-proj: FlatRoPE sets p_T = p_H = p_W = m, the sequence
+Sec. 4.2, Eq. flatrope-proj: FlatRoPE sets p_T = p_H = p_W = m, the sequence
 index, so the phase is theta_d * m at every pair.
 
 Readings taken where the paper is loose:
   * theta_d is one global schedule indexed by the global pair d (Eq.
     mrope-phase), not three per-axis vectors (Eq. rope-3d's w^T, w^H, w^W).
     Only this reading makes M-RoPE reduce to 1D RoPE when t = h = w, which the
-    paper states in Sec. 2.3 and Sec. 3.2.
+    paper states in Sec. 3.3 and Sec. 4.2.
   * Pairs are adjacent dimensions (2d, 2d+1), the literal block-diagonal form
     of Eq. rope-1d.
   * The base is a parameter (the paper's example is 10000; the workloads use

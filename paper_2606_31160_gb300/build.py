@@ -3,8 +3,10 @@
 Each translation unit under csrc/ compiles to an object in parallel, then the
 objects link into paper_2606_31160_gb300/libsd.so with the CUDA runtime linked
 statically, so the library loads on a machine without a GPU and needs nothing
-but the driver at run time. Rebuilds only when a source, header or flag
-changed (content hash stamp).
+but the driver at run time. floor/floor.cu (the launch and streaming floors
+that `bench.py --floor` measures; not part of the verify path) builds beside
+it into libsdfloor.so. Rebuilds only when a source, header or flag changed
+(content hash stamp).
 
     python -m paper_2606_31160_gb300.build [--force] [--ptxas-info]
 """
@@ -22,6 +24,8 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libsd.so")
+FLOOR_SRC = os.path.join(PKG, "floor", "floor.cu")
+FLOOR_LIB = os.path.join(PKG, "libsdfloor.so")
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC,-O2",
@@ -45,6 +49,8 @@ def _stamp(extra):
             h.update(name.encode())
             with open(path, "rb") as f:
                 h.update(f.read())
+    with open(FLOOR_SRC, "rb") as f:
+        h.update(f.read())
     h.update(" ".join(NVCC_FLAGS + extra).encode())
     return h.hexdigest()
 
@@ -54,7 +60,7 @@ def build(force=False, ptxas_info=False, verbose=False):
     extra = ["-Xptxas", "-v"] if ptxas_info else []
     stamp = _stamp(extra)
     stamp_file = os.path.join(BUILD, "stamp")
-    if not force and os.path.exists(LIB) and os.path.exists(stamp_file):
+    if not force and os.path.exists(LIB) and os.path.exists(FLOOR_LIB) and os.path.exists(stamp_file):
         with open(stamp_file) as f:
             if f.read().strip() == stamp:
                 return LIB
@@ -69,8 +75,19 @@ def build(force=False, ptxas_info=False, verbose=False):
             raise RuntimeError("nvcc failed for %s:\n%s\n%s" % (src, " ".join(cmd), res.stderr))
         return obj, res.stderr
 
-    with ThreadPoolExecutor(max_workers=min(len(SOURCES), os.cpu_count() or 4)) as ex:
+    def floor_lib():
+        tmp = FLOOR_LIB + ".tmp"
+        cmd = [nvcc, "-shared", FLOOR_SRC, "-o", tmp] + NVCC_FLAGS + extra + [
+            "-cudart", "static", "-Xlinker", "--no-undefined", "-lrt", "-lpthread", "-ldl"]
+        res = subprocess.run(cmd, capture_output=True, text=True)
+        if res.returncode != 0:
+            raise RuntimeError("nvcc failed for floor.cu:\n%s\n%s" % (" ".join(cmd), res.stderr))
+        os.replace(tmp, FLOOR_LIB)
+
+    with ThreadPoolExecutor(max_workers=min(len(SOURCES) + 1, os.cpu_count() or 4)) as ex:
+        floor_job = ex.submit(floor_lib)
         results = list(ex.map(compile_one, SOURCES))
+        floor_job.result()
     if verbose or ptxas_info:
         for (obj, err), src in zip(results, SOURCES):
             if err.strip():

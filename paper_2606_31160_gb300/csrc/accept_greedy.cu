@@ -1,5 +1,5 @@
-// K4: greedy acceptance (Eqs. verify, accept, commit, Sec. 2.2; Eq.
-// accept-length, Sec. 3.3).
+// K4: greedy acceptance (Eqs. verify, accept, commit, Sec. 3.2; Eq.
+// accept-length, Sec. 4.3).
 //
 //   r*_j = argmax_v logits[b][j][v]   (lowest index among equal maxima)
 //   l    = number of leading drafts equal to r*   (draft[j] vs r*_j, j < K)

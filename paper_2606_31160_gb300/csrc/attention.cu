@@ -1,5 +1,5 @@
 // K3: verify attention of the K + 1 new rows against the cached prefix
-// (Eq. verify, Sec. 2.2), GQA, causal, bf16 in / bf16 out, fp32 softmax.
+// (Eq. verify, Sec. 3.2), GQA, causal, bf16 in / bf16 out, fp32 softmax.
 //
 // Work decomposition (one launch):
 //   * A "unit" is (scene b, KV head g, block of packed query rows). The G

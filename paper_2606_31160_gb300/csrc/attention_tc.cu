@@ -1,7 +1,7 @@
 // K3 on the 5th-generation tensor cores (tcgen05 + TMEM): verify attention
-// of the K + 1 new rows against the cached prefix (Eq. verify, Sec. 2.2),
+// of the K + 1 new rows against the cached prefix (Eq. verify, Sec. 3.2),
 // for head_dim 128 and up to 128 packed query rows per KV head, and the fused
-// verify layer (M-RoPE of Sec. 2.3 / Sec. 3.2 + the KV append of Eq. commit +
+// verify layer (M-RoPE of Sec. 3.3 / Sec. 4.2 + the KV append of Eq. commit +
 // the attention) on the same machinery.
 //
 // The packed query tile is small (G*R = 32 rows for 32 q / 8 KV heads and
@@ -443,13 +443,17 @@ __device__ __forceinline__ void griddep_launch() {
 }
 
 // ------------------------------------------------------------------ kernel
-// kFused = false: attention over a cache that already holds the R new rows,
-// with the rotated query rows read from a.q.
-// kFused = true: the whole verify layer -- M-RoPE of the raw query and key
-// rows, the KV append and the attention -- with len[b] the prefix length.
+// kMode 0: attention over a cache that already holds the R new rows, every
+// key in the tensor-core loop, the rotated query rows read from a.q.
+// kMode 2: the same attention with the loop over the prefix keys only; the R
+// new rows (read from the cache) enter as one more product S_new.
+// kMode 1: the whole verify layer -- M-RoPE of the raw query and key rows, the
+// KV append and the attention -- with len[b] the prefix length; the rotated
+// new keys enter as S_new.
 // Prefix tiles, len and pos are independent of the kernel that precedes this
-// one in the stream (for every layer but the first of a step), so when
-// a.early is set they are read before the programmatic-dependency wait.
+// one in the stream (for every layer but the first of a step), so when bit 0
+// of a.early is set (modes 1 and 2) they are read before the
+// programmatic-dependency wait.
 // Grid: (cluster size, Hkv * n_mblocks, B); m-block mb takes packed query rows
 // mb * kR .. mb * kR + kR - 1.
 template <int kR, int kMode>
@@ -458,9 +462,6 @@ __global__ void __launch_bounds__(kThreads, 1)
                           const __grid_constant__ CUtensorMap tm_v128, const TcArgs a,
                           const RopeTable tab) {
   using C = Cfg<kR>;
-  // kMode 1: the fused layer; 2: attention over a cache holding the new rows,
-  // merged like the fused layer's new keys; 0: attention with every key in the
-  // tensor-core loop (any R)
   constexpr bool kFused = kMode == 1;
   constexpr bool kNew = kMode != 0;  // the R new keys enter as S_new, not as tiles
   // prefix (and len) before the dependency wait; the block mask

@@ -1,4 +1,4 @@
-// Attention budget of the verify rows (Sec. 3.2 "Empirical confirmation",
+// Attention budget of the verify rows (Sec. 4.2 "Empirical confirmation",
 // Table tab:attn-budget): for every (scene, row, query head), the share of
 // the row's softmax mass on the visual keys, on the trajectory / prompt-text
 // keys and on the rows generated in this step, and the entropy of the

@@ -86,7 +86,7 @@ __device__ __forceinline__ float sd_bf16_lo(uint32_t w) { return __uint_as_float
 __device__ __forceinline__ float sd_bf16_hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
 
 // ---------------------------------------------------------------------------
-// RoPE (Sec. 2.3 Eq. rope-1d, Sec. 3.2 Eqs. axis-assign, mrope-phase) shared by
+// RoPE (Sec. 3.3 Eq. rope-1d, Sec. 4.2 Eqs. axis-assign, mrope-phase) shared by
 // the standalone rotation kernel and the fused verify-layer kernel, so both
 // produce identical bits. The angle theta_d * p is carried in TURNS:
 // tau_d = theta_d / (2 pi) as an fp32 hi/lo pair; p * tau_d is formed with an

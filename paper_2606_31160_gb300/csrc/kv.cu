@@ -1,6 +1,6 @@
 // K2: KV-cache append and rollback (sm_103a).
 //
-// Eq. commit (Sec. 2.2): an iteration commits l + 1 tokens, t <- t + l + 1.
+// Eq. commit (Sec. 3.2): an iteration commits l + 1 tokens, t <- t + l + 1.
 // The verify pass appends the keys/values of all R = K + 1 rows before the
 // acceptance is known; afterwards the length moves back to keep only the
 // n_emit = l + 1 committed rows. Nothing is erased: later appends overwrite.

@@ -1,6 +1,6 @@
-// The fused verify layer: M-RoPE of the new query and key rows (Sec. 2.3,
-// Sec. 3.2), the KV append (Eq. commit) and the verify attention (Eq. verify,
-// Sec. 2.2) of one attention layer as one call.
+// The fused verify layer: M-RoPE of the new query and key rows (Sec. 3.3,
+// Sec. 4.2), the KV append (Eq. commit) and the verify attention (Eq. verify,
+// Sec. 3.2) of one attention layer as one call.
 //
 // On the tcgen05 path (head_dim 128, G * R <= 128, R <= 16) it is one kernel launch that
 // may overlap the previous layer: the cached prefix of a layer does not

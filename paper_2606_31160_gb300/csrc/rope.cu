@@ -1,9 +1,9 @@
 // K1: rotary position encoding of the new verify rows (sm_103a).
 //
-// Sec. 2.3 Eq. rope-1d: each adjacent pair (2d, 2d+1) of a head vector
-// rotates by phi_d; Sec. 2.3 Eq. rope-3d with Sec. 3.2 Eqs. axis-assign and
+// Sec. 3.3 Eq. rope-1d: each adjacent pair (2d, 2d+1) of a head vector
+// rotates by phi_d; Sec. 3.3 Eq. rope-3d with Sec. 4.2 Eqs. axis-assign and
 // mrope-phase: phi_d = theta_d * p_{a(d)}, theta_d = base^(-2d/D), a(d)
-// blocked over (s_T, s_H, s_W) or (T,H,W)[d mod 3]; Sec. 3.2 Eq.
+// blocked over (s_T, s_H, s_W) or (T,H,W)[d mod 3]; Sec. 4.2 Eq.
 // flatrope-proj: FlatRoPE puts every axis at the sequence index.
 //
 // Layout: one thread rotates 4 pairs (8 bf16 = one 16-byte load/store) of

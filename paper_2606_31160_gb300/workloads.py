@@ -6,11 +6,11 @@ arithmetic: no rotation, attention, softmax, argmax over model outputs, or
 acceptance test. It only draws numbers and lays them out.
 
 The paper's workloads are Alpamayo-R1 driving clips on an 8B Qwen3-VL
-backbone (Sec. 4, "Targets and drafts", "Data"); neither the clips nor any
+backbone (Sec. 5, "Targets and drafts", "Data"); neither the clips nor any
 weights are available, so every tensor is synthetic with the shapes and
 structure the paper states: a prompt that is ~96% multi-camera vision
-patches (Sec. 3.2, "Empirical confirmation"), 15-20-token reasoning outputs
-(Sec. 1) and verify blocks of K <= 16 (Sec. 4, "Metric").
+patches (Sec. 4.2, "Empirical confirmation"), 15-20-token reasoning outputs
+(Sec. 1) and verify blocks of K <= 16 (Sec. 5, "Metric").
 
 Random streams: numpy Generator(Philox(key=(1000 + workload id, layer))).
 Normals are drawn in float32 and rounded to bf16 (or kept fp32) before use,

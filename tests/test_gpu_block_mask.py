@@ -1,5 +1,5 @@
 """The block mask (every new row sees all R new rows: the block-diffusion
-draft's pattern, Sec. 4) on both attention kernels and the fused layer,
+draft's pattern, Sec. 5) on both attention kernels and the fused layer,
 against the float64 oracle."""
 import os
 import subprocess

@@ -1,5 +1,5 @@
 """GPU parity of sd_attention_budget against the float64 oracle
-(Sec. 3.2, Table tab:attn-budget): masses and normalised entropies within
+(Sec. 4.2, Table tab:attn-budget): masses and normalised entropies within
 1e-4 (fp32 scores and sums against float64)."""
 import numpy as np
 import pytest

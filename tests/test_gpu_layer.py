@@ -158,7 +158,7 @@ def test_fused_layer_long_drafts(K):
 
 @pytest.mark.parametrize("K", [7, 8, 16])
 def test_fused_layer_interleaved_mrope(K):
-    # interleaved axis assignment a(d) = (T, H, W)[d mod 3] (Sec. 3.2 Eq.
+    # interleaved axis assignment a(d) = (T, H, W)[d mod 3] (Sec. 4.2 Eq.
     # axis-assign) through the fused kernel's own rotation table, on the
     # 32-row tile (K = 7), the 64-row tile (K = 8) and two 64-row m-blocks
     # (K = 16); query rows at distinct (t, h, w) so that the layout matters

@@ -1,4 +1,4 @@
-"""Pins of the float64 verify-attention oracle (Eq. verify, Sec. 2.2).
+"""Pins of the float64 verify-attention oracle (Eq. verify, Sec. 3.2).
 
 The oracle is checked against torch's float64 scaled_dot_product_attention
 (a library routine) with a causal mask built here from the reading "row i

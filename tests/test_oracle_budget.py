@@ -1,4 +1,4 @@
-"""Pins of the float64 attention-budget oracle (Sec. 3.2, Table tab:attn-budget).
+"""Pins of the float64 attention-budget oracle (Sec. 4.2, Table tab:attn-budget).
 
 Checked against closed forms (uniform scores, a dominating key, two keys)
 and against verify_attention -- itself pinned to torch's float64

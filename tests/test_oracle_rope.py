@@ -1,4 +1,4 @@
-"""Pins of the float64 RoPE / M-RoPE / FlatRoPE oracle (Sec. 2.3, Sec. 3.2).
+"""Pins of the float64 RoPE / M-RoPE / FlatRoPE oracle (Sec. 3.3, Sec. 4.2).
 
 Each check is a fact the paper or plain mathematics fixes, chosen so that a
 wrong sign, a wrong pairing, a wrong frequency exponent or a wrong axis
@@ -73,7 +73,7 @@ def test_position_zero_is_identity():
 @pytest.mark.parametrize("inter", [0, 1])
 @pytest.mark.parametrize("base", [1e4, 1e6])
 def test_mrope_reduces_to_1d_when_coordinates_equal(D, sec, inter, base):
-    # Sec. 2.3 / Sec. 3.2: with m^T = m^H = m^W = m, M-RoPE equals 1D RoPE;
+    # Sec. 3.3 / Sec. 4.2: with m^T = m^H = m^W = m, M-RoPE equals 1D RoPE;
     # the 1D side is the explicit block-diagonal matrix of Eq. rope-1d.
     rng = np.random.default_rng(2)
     for m in [0, 1, 7, 544, 4103, 16400]:
@@ -103,7 +103,7 @@ def test_pair_norms_preserved():
 
 @pytest.mark.parametrize("inter", [0, 1])
 def test_scores_depend_only_on_relative_position_per_axis(inter):
-    # Sec. 3.2 ("Why mirroring is harmful", FlatRoPE (ii)): after rotation the
+    # Sec. 4.2 ("Why mirroring is harmful", FlatRoPE (ii)): after rotation the
     # score q.k depends on the coordinate difference of each axis only, so a
     # common shift of one axis leaves it unchanged.
     rng = np.random.default_rng(4)
@@ -124,7 +124,7 @@ def test_scores_depend_only_on_relative_position_per_axis(inter):
 
 
 def test_flatrope_ignores_section_layout():
-    # Sec. 3.2, FlatRoPE (i): with p_T = p_H = p_W = m the section sizes and the
+    # Sec. 4.2, FlatRoPE (i): with p_T = p_H = p_W = m the section sizes and the
     # interleaved flag are irrelevant, so all layouts agree exactly.
     rng = np.random.default_rng(5)
     x = rng.standard_normal((7, 16, 128))
