@@ -449,11 +449,11 @@ __device__ __forceinline__ void griddep_launch() {
 // new rows (read from the cache) enter as one more product S_new.
 // kMode 1: the whole verify layer -- M-RoPE of the raw query and key rows, the
 // KV append and the attention -- with len[b] the prefix length; the rotated
-// new keys enter as S_new.
-// Prefix tiles, len and pos are independent of the kernel that precedes this
-// one in the stream (for every layer but the first of a step), so when bit 0
-// of a.early is set (modes 1 and 2) they are read before the
-// programmatic-dependency wait.
+// new keys enter as S_new. Prefix tiles, len and pos are independent of the
+// kernel that precedes this one in the stream (for every layer but the first
+// of a step), so they are read before the programmatic-dependency wait.
+// kMode 3: the same layer as a plain launch (everything after the wait).
+// kMode 2 reads its prefix before the wait when bit 0 of a.early is set.
 // Grid: (cluster size, Hkv * n_mblocks, B); m-block mb takes packed query rows
 // mb * kR .. mb * kR + kR - 1.
 template <int kR, int kMode>
@@ -462,10 +462,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                           const __grid_constant__ CUtensorMap tm_v128, const TcArgs a,
                           const RopeTable tab) {
   using C = Cfg<kR>;
-  constexpr bool kFused = kMode == 1;
+  constexpr bool kFused = kMode == 1 || kMode == 3;
   constexpr bool kNew = kMode != 0;  // the R new keys enter as S_new, not as tiles
   // prefix (and len) before the dependency wait; the block mask
-  const bool early = kNew && (a.early & 1) != 0;
+  const bool early = kMode == 1 || (kMode == 2 && (a.early & 1) != 0);
   // (the fused layer's 32-row tile takes no block mask: its callers are the
   // target's causal verify steps; the host sends block-masked 32-row layers
   // through the separate kernels)
@@ -550,7 +550,35 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (threadIdx.x == 0) {
     *s_len = a.len[b];  // the scene's length advances at the producer's end
   }
+  // The fused layer's raw q / k / v rows do not depend on len or pos. In a
+  // plain launch (the dependency wait above comes before everything) the
+  // softmax threads issue their row loads together with the pos loads of the
+  // rotation table: one global round trip before the tiles instead of two.
+  constexpr int kQc = kR * 16 / kSoftThreads;        // 16-byte query chunks a thread
+  constexpr int kKvc = C::kMaxNew * 16 / kSoftThreads;  // 16-byte new key / value chunks a thread
+  constexpr bool rows_first = kMode == 3;
+  uint4 pre_q[kQc], pre_k[kKvc], pre_v[kKvc];
+  auto preload_rows = [&](int st) {
+#pragma unroll
+    for (int u = 0; u < kQc; ++u) {
+      const int idx = st + u * kSoftThreads, p = mblock * kR + (idx >> 4), c = idx & 15;
+      const int i = gdiv(p);
+      pre_q[u] = p < a.M ? __ldcg(reinterpret_cast<const uint4*>(
+                               a.qw + ((static_cast<long long>(b) * a.R + i) * a.Hq + kvh * a.G + (p - i * a.G)) * kD +
+                               c * 8))
+                         : make_uint4(0, 0, 0, 0);
+    }
+#pragma unroll
+    for (int u = 0; u < kKvc; ++u) {
+      const int idx = st + u * kSoftThreads;
+      const long long src = ((static_cast<long long>(b) * a.R + (idx >> 4)) * a.Hkv + kvh) * kD + (idx & 15) * 8;
+      const bool ok = idx < a.R * 16;
+      pre_k[u] = ok ? __ldcg(reinterpret_cast<const uint4*>(a.k_new + src)) : make_uint4(0, 0, 0, 0);
+      pre_v[u] = ok ? __ldcg(reinterpret_cast<const uint4*>(a.v_new + src)) : make_uint4(0, 0, 0, 0);
+    }
+  };
   if (kFused && threadIdx.x >= 64 && threadIdx.x < 64 + kSoftThreads) {
+    if (rows_first) preload_rows(threadIdx.x - 64);
     // rotation table of the R new positions: (cos, sin) per (row, pair),
     // built while thread 0 takes the scene's length
     float2* tabw = reinterpret_cast<float2*>(smem + C::kOffTab);
@@ -799,7 +827,6 @@ __global__ void __launch_bounds__(kThreads, 1)
       // the packed query tile: this thread's 16-byte chunks (row, chunk c),
       // rows past M zero; in the fused layer also one chunk of a new key and
       // value row
-      constexpr int kQc = kR * 16 / kSoftThreads;
       const __nv_bfloat16* q_src[kQc];
       int q_cs[kQc];
       bool q_ok[kQc];
@@ -814,7 +841,6 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       // new key / value rows: chunk st + u * 256 (row >> 4, 16-byte chunk & 15);
       // one chunk a thread with 32 rows (16 new rows), two with 64 (32)
-      constexpr int kKvc = C::kMaxNew * 16 / kSoftThreads;
       const bool append = kFused && valid && rank == csize - 1 && mblock == 0;
       bool has_kv[kKvc];
       long long kv_src[kKvc];
@@ -834,18 +860,28 @@ __global__ void __launch_bounds__(kThreads, 1)
       // nearly so: no warm-up pass, its rows are read once, after the wait
       const bool last_cluster = blockIdx.y == gridDim.y - 1 && blockIdx.z == gridDim.z - 1;
 #pragma unroll 1
-      for (int it = (kNew && !(early && last_cluster)) ? 0 : 1; it < 2; ++it) {
-        if (kNew && it == 1 && early) griddep_wait();  // the rows come from earlier kernels
+      for (int it = (kNew && !rows_first && !(early && last_cluster)) ? 0 : 1; it < 2; ++it) {
+        if (kNew && it == 1 && early && !rows_first) griddep_wait();  // the rows come from earlier kernels
         uint4 qv[kQc], kv[kKvc], vv[kKvc];
+        if (rows_first) {
 #pragma unroll
-        for (int u = 0; u < kQc; ++u)
-          qv[u] = q_ok[u] ? __ldcg(reinterpret_cast<const uint4*>(q_src[u])) : make_uint4(0, 0, 0, 0);
+          for (int u = 0; u < kQc; ++u) qv[u] = q_ok[u] ? pre_q[u] : make_uint4(0, 0, 0, 0);
 #pragma unroll
-        for (int u = 0; u < kKvc; ++u) {
-          kv[u] = has_kv[u] ? __ldcg(reinterpret_cast<const uint4*>((kFused ? a.k_new : a.kc) + kv_src[u]))
-                            : make_uint4(0, 0, 0, 0);
-          vv[u] = has_kv[u] ? __ldcg(reinterpret_cast<const uint4*>((kFused ? a.v_new : a.vc) + kv_src[u]))
-                            : make_uint4(0, 0, 0, 0);
+          for (int u = 0; u < kKvc; ++u) {
+            kv[u] = has_kv[u] ? pre_k[u] : make_uint4(0, 0, 0, 0);
+            vv[u] = has_kv[u] ? pre_v[u] : make_uint4(0, 0, 0, 0);
+          }
+        } else {
+#pragma unroll
+          for (int u = 0; u < kQc; ++u)
+            qv[u] = q_ok[u] ? __ldcg(reinterpret_cast<const uint4*>(q_src[u])) : make_uint4(0, 0, 0, 0);
+#pragma unroll
+          for (int u = 0; u < kKvc; ++u) {
+            kv[u] = has_kv[u] ? __ldcg(reinterpret_cast<const uint4*>((kFused ? a.k_new : a.kc) + kv_src[u]))
+                              : make_uint4(0, 0, 0, 0);
+            vv[u] = has_kv[u] ? __ldcg(reinterpret_cast<const uint4*>((kFused ? a.v_new : a.vc) + kv_src[u]))
+                              : make_uint4(0, 0, 0, 0);
+          }
         }
         // (fused: M-RoPE of) the packed query rows, straight into the swizzled tile
 #pragma unroll
@@ -1402,13 +1438,16 @@ bool set_attributes(int* active) {
   auto kern = verify_attn_tc_kernel<kR, 0>;
   auto kern_f = verify_attn_tc_kernel<kR, 1>;
   auto kern_n = verify_attn_tc_kernel<kR, 2>;
+  auto kern_p = verify_attn_tc_kernel<kR, 3>;
   constexpr int smem = Cfg<kR>::kSmemBytes;
   if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess ||
       cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess ||
       cudaFuncSetAttribute(kern_f, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess ||
       cudaFuncSetAttribute(kern_f, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess ||
       cudaFuncSetAttribute(kern_n, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess ||
-      cudaFuncSetAttribute(kern_n, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess) {
+      cudaFuncSetAttribute(kern_n, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess ||
+      cudaFuncSetAttribute(kern_p, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess ||
+      cudaFuncSetAttribute(kern_p, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess) {
     (void)cudaGetLastError();
     return false;
   }
@@ -1644,5 +1683,6 @@ sd_status sd_internal_verify_layer_tc(void* q, void* k_new, const void* v_new, c
   a.n_mblocks = plan.mblocks;
   a.scale_log2 = scale_log2;
   *handled = true;
-  return launch_plan<1>(cache, a, tab, plan, early != 0, stream);
+  if (early) return launch_plan<1>(cache, a, tab, plan, true, stream);
+  return launch_plan<3>(cache, a, tab, plan, false, stream);
 }
