@@ -99,17 +99,11 @@ struct Cfg {
   // swizzle for 64 rows; 8-key groups are kPRow * 8 bytes apart
   static constexpr uint64_t kPLayout = kR == 32 ? 4 : 2;
   static constexpr int kTmemCols = kR == 32 ? 128 : 256;    // S0 | S1 | S2 | O, kR columns each
-  // fused layer: one more kR-column buffer after O for S_new = K_new Q^T
-  static constexpr int kTmemColsFused = 2 * kTmemCols;
   // shared memory layout (offsets from the 1024-aligned base)
   static constexpr int kOffQ = kRing;
-  // P^T buffers. Fused layer: before the tiles the first one holds the rotated
-  // new keys as a K-major, 128-byte-swizzled S_new operand (rows 0..kMaxNew-1
-  // of each 64-column half, halves kNewHalf apart; the MMA reads 128 rows, the
-  // rest is whatever follows and only fills score lanes that are never read),
-  // and the second one the rotation table
+  // P^T buffers; before the tiles the second one holds the fused layer's
+  // rotation table
   static constexpr int kOffP = kOffQ + kQ;
-  static constexpr int kNewHalf = kMaxNew * 128;
   static constexpr int kOffTab = kOffP + kP;
   static constexpr int kOffNewK = kOffP + 2 * kP;
   static constexpr int kOffNewV = kOffNewK + kMaxNew * kNewRow;
@@ -118,21 +112,19 @@ struct Cfg {
   // columns)
   static constexpr int kSBuf = 3;
   // barriers: full_k[S] full_v[S] p_full[2] s_ready[3] pv_done[S] q_full recv
-  // decide s_free[3] s_new tmem_done
-  static constexpr int kNumBars = 3 * kStages + 13;
+  // decide s_free[3] tmem_done
+  static constexpr int kNumBars = 3 * kStages + 12;
   // tmem slot, (unused), decision, len (and, 64 rows, the last reader of the new key rows)
   static constexpr int kOffMisc = round_up(kOffBar + kNumBars * 8, 16);
   static constexpr int kOffRowA = kOffMisc + (kR == 32 ? 16 : 32);  // [kR] per-row results (reductions)
   static constexpr int kOffRef = kOffRowA + kR * 4;         // [kR] per-row references
   static constexpr int kOffLim = kOffRef + kR * 4;          // [kR] per-row causal key limits
   static constexpr int kSmemBytes = kOffLim + kR * 4 + 1024;
-  static_assert(kOffP + kNewHalf + 128 * 128 <= kSmemBytes - 1024, "the S_new operand's 128 rows stay inside");
   static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
   static_assert(kOffQ % 1024 == 0 && kOffP % 1024 == 0 && kP % 1024 == 0 && kOffNewK % 16 == 0 &&
                     kOffNewV % 16 == 0 && kOffBar % 8 == 0 && kOffRowA % 16 == 0 && kOffRef % 16 == 0,
                 "alignment of the shared-memory regions (swizzle atoms, vector accesses, mbarriers)");
   static_assert(kMaxNew * 64 * 8 <= kP, "rotation table fits the second P buffer");
-  static_assert(kP >= 2 * kNewHalf && kOffP % 1024 == 0, "new-key operand fits the first P buffer");
   static_assert(kR * 128 * 4 <= 2 * kP, "row reductions fit the P buffers");
   // cluster merge buffers (in the rings, free once this CTA's last MMA is done)
   static constexpr int kSend = 0;                           // this CTA's kR rows
@@ -474,7 +466,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   constexpr int kRpt = C::kRpt;
   constexpr uint32_t kIdescS = umma_idesc(128, kR, 0, 0);
   constexpr uint32_t kIdescO = umma_idesc(128, kR, 1, 1);
-  constexpr int kTmemAlloc = kNew ? C::kTmemColsFused : C::kTmemCols;
+  constexpr int kTmemAlloc = C::kTmemCols;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
@@ -502,8 +494,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   // 32 rows: the softmax has read S(T) (its tensor-memory buffer takes S(T + 3))
   auto SFREE = [&](int T) { return bar(3 * kS + 8 + T % 3); };
   auto s_parity = [](int T) { return static_cast<uint32_t>((T / 3) & 1); };  // SREADY, SFREE phases
-  const uint32_t SNEW = bar(3 * kS + 11);  // fused layer: S_new = K_new Q^T is in tensor memory
-  const uint32_t TMEMDONE = bar(3 * kS + 12);  // every softmax warp has read its last column
+  const uint32_t TMEMDONE = bar(3 * kS + 11);  // every softmax warp has read its last column
   constexpr int kSB = C::kSBuf;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::kOffMisc);
   int* s_redo = reinterpret_cast<int*>(smem + C::kOffMisc + 8);
@@ -533,7 +524,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(RECV, 1);
     mbar_init(DECIDE, 1);
     for (int i = 0; i < 3; ++i) mbar_init(SFREE(i), kSoftWarps);
-    mbar_init(SNEW, 1);
     mbar_init(TMEMDONE, kSoftWarps);
     *s_redo = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -595,7 +585,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem = *tmem_slot;
   const uint32_t tmem_s = tmem;            // S buffer b at column kR * b
   const uint32_t tmem_o = tmem + kSB * kR; // O^T
-  const uint32_t tmem_snew = tmem + (kSB + 1) * kR;  // fused layer: S_new^T (new keys on lanes 0..R-1)
 
   int n_keys, L_pre;
   bool valid;
@@ -717,30 +706,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     // S(T) and PV(T) come from two warps (this one and the PV warp), so that
     // one batch is issued while the other executes; the whole warp waits and
     // one elected lane issues.
-    const bool snew = kNew && valid;
     bool arrived = false;
-    if (n_tiles > 0 || snew) {
+    if (n_tiles > 0) {
       mbar_wait(QFULL, 0);
       // base descriptors; a K step only moves the start address (low field, no carry)
       const uint64_t dK0 = umma_desc(base, 16, 1024);  // K tile: K-major
       const uint64_t dQ = umma_desc(qs, 16, 1024);     // Q: K-major
-      // fused layer: the scores of the R new keys, S_new^T = K_new Q^T (new
-      // key n on lane n), into their own tensor-memory buffer after S(0); the
-      // operand sits in the first P buffer, which P(0) overwrites only once
-      // SNEW is out
-      auto issue_snew = [&]() {
-        tc_fence_after();
-        const uint64_t dN = umma_desc(base + C::kOffP, 16, 1024);
-        if (elect_one()) {
-#pragma unroll
-          for (int kk = 0; kk < 8; ++kk)
-            umma(tmem_snew, dN + (((kk >> 2) * C::kNewHalf + (kk & 3) * 32) >> 4),
-                 dQ + (((kk >> 2) * C::kQHalf + (kk & 3) * 32) >> 4), kIdescS, kk > 0 ? 1 : 0);
-          umma_commit(SNEW);
-        }
-        __syncwarp();
-      };
-      if (snew && n_tiles == 0) issue_snew();
       for (int pass = 0; pass < 2; ++pass) {
         if (pass == 1) {
           cluster_arrive_relaxed();  // before the decision (see the producer)
@@ -766,7 +737,6 @@ __global__ void __launch_bounds__(kThreads, 1)
             umma_commit(SREADY(T));
           }
           __syncwarp();
-          if (snew && T == 0) issue_snew();
         }
       }
     }
@@ -910,8 +880,6 @@ __global__ void __launch_bounds__(kThreads, 1)
               for (int j = 0; j < 4; ++j) w[j] = sd_rope_pair(w[j], cs[j].x, cs[j].y);
             }
             st_shared_v4(base + C::kOffNewK + i * kNewRow + c * 16, w[0], w[1], w[2], w[3]);
-            st_shared_v4(base + C::kOffP + (c >> 3) * C::kNewHalf + i * 128 + (((c & 7) ^ (i & 7)) << 4), w[0], w[1],
-                         w[2], w[3]);
             st_shared_v4(base + C::kOffNewV + i * kNewRow + c * 16, vv[u].x, vv[u].y, vv[u].z, vv[u].w);
             if (append && it == 1) {
               // the append (the head's last rank of m-block 0): cache rows
@@ -1116,7 +1084,6 @@ __global__ void __launch_bounds__(kThreads, 1)
             lp[j0 + j + 1] += sd_bf16_hi(w);
           }
           if (T >= 2 && j0 == 0) mbar_wait(PVDONE(T - 2), ring_parity(T - 2));  // PV(T - 2) has read P buffer bb
-          if (kNew && T == 0 && j0 == 0 && valid) mbar_wait(SNEW, 0);  // S_new has read its operand
           const int ch = (row0 + j0) >> 3;
           st_shared_v4(prow + ((ch ^ sw) << 4), pw[0], pw[1], pw[2], pw[3]);
           st_shared_v4(prow + (((ch + 1) ^ sw) << 4), pw[4], pw[5], pw[6], pw[7]);
@@ -1193,30 +1160,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (quarter == 0 && lane < kRpt)
         send[(row0 + lane) * kRowF + kRowM] = n_tiles > 0 ? row_ref[row0 + lane] : -INFINITY;
     }
-    // the new-key scores of the rows this CTA merges, from S_new^T (new key n
-    // on lane n of the first TMEM lane quarter), scaled, causally masked
-    float* s_new = reinterpret_cast<float*>(smem + C::kNewS);  // [my_rows][R]
-    if (kNew && valid && quarter == 0 && half == 0) {
-      mbar_wait(SNEW, 0);
-      tc_fence_after();
-#pragma unroll 1
-      for (int rr0 = 0; rr0 < my_rows; rr0 += 4) {
-        // columns past the merged rows stay inside the allocation and go unused
-        uint32_t v[4];
-        asm volatile("tcgen05.ld.sync.aligned.32x32b.x4.b32 {%0,%1,%2,%3}, [%4];"
-                     : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3])
-                     : "r"(tmem_snew + mrow0 + rr0));
-        asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          const int rr = rr0 + j, p = mblock * kR + mrow0 + rr;
-          // causal: row p = i * G + g sees new keys 0..i; block mask: all R
-          if (rr < my_rows && lane < a.R)
-            s_new[rr * a.R + lane] =
-                (p < a.M && (block || lane <= gdiv(p))) ? __uint_as_float(v[j]) * a.scale_log2 : -INFINITY;
-        }
-      }
-    }
+    float* s_new = reinterpret_cast<float*>(smem + C::kNewS);  // [my_rows][R] new-key scores
     if (n_tiles > 0) {
       // every MMA is done once the last PV is (PVDONE's phases complete in order)
       const int Tl = (redo ? 2 : 1) * n_tiles - 1;
@@ -1257,6 +1201,42 @@ __global__ void __launch_bounds__(kThreads, 1)
       asm volatile("cp.async.bulk.commit_group;" ::: "memory");
     }
     __syncwarp();
+    // While the partials travel: the scores of the R new keys against the
+    // rows this CTA merges, on the CUDA cores from the rotated rows in shared
+    // memory (query tile, new key rows): 8 lanes a dot product, 16 d each,
+    // fp32 sums of the bf16 products. Scaled to log2 units; causal: row p =
+    // i * G + g sees new keys 0..i; the block mask: all R. Every lane of a warp
+    // runs the loop and the shuffles (the warp's 4 dot products of an
+    // iteration may run past the last one).
+    const int n_new = (kNew && valid) ? a.R : 0;
+    const int n_dots = my_rows * n_new;
+#pragma unroll 1
+    for (int base0 = (st >> 5) * 4; kNew && base0 < n_dots; base0 += kSoftThreads / 8) {  // warp-uniform
+      const int dot = base0 + (lane >> 3), sub = lane & 7;
+      const bool act = dot < n_dots;
+      const int rr = act ? dot / n_new : 0, n = act ? dot - rr * n_new : 0, row = mrow0 + rr;
+      float acc = 0.f;
+#pragma unroll
+      for (int u = 0; u < 2; ++u) {
+        const int c = sub + 8 * u;
+        const uint4 qw = *reinterpret_cast<const uint4*>(smem + C::kOffQ + (c >> 3) * C::kQHalf + row * 128 +
+                                                         (((c & 7) ^ (row & 7)) << 4));
+        const uint4 kw = *reinterpret_cast<const uint4*>(smem + C::kOffNewK + n * kNewRow + c * 16);
+        acc = fmaf(sd_bf16_lo(qw.x), sd_bf16_lo(kw.x), acc);
+        acc = fmaf(sd_bf16_hi(qw.x), sd_bf16_hi(kw.x), acc);
+        acc = fmaf(sd_bf16_lo(qw.y), sd_bf16_lo(kw.y), acc);
+        acc = fmaf(sd_bf16_hi(qw.y), sd_bf16_hi(kw.y), acc);
+        acc = fmaf(sd_bf16_lo(qw.z), sd_bf16_lo(kw.z), acc);
+        acc = fmaf(sd_bf16_hi(qw.z), sd_bf16_hi(kw.z), acc);
+        acc = fmaf(sd_bf16_lo(qw.w), sd_bf16_lo(kw.w), acc);
+        acc = fmaf(sd_bf16_hi(qw.w), sd_bf16_hi(kw.w), acc);
+      }
+#pragma unroll
+      for (int sh = 1; sh < 8; sh <<= 1) acc += __shfl_xor_sync(0xffffffffu, acc, sh);
+      const int p = mblock * kR + row;
+      if (act && sub == 0)
+        s_new[rr * n_new + n] = (p < a.M && (block || n <= gdiv(p))) ? acc * a.scale_log2 : -INFINITY;
+    }
     if (kFused && valid) {
       // while the partials travel: every CTA of the cluster read the raw rows
       // before its tiles (the cluster barrier above is behind all of them), so
@@ -1293,7 +1273,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // used the row's reference (the common case: the second pass is rare), the
     // partials then add with the one weight 2^(ref - M); otherwise every
     // partial takes its own weight.
-    const int n_new = (kNew && valid) ? a.R : 0;
+    named_bar_sync(2, kSoftThreads);  // every new-key score is in s_new
     const int rr = st >> 6, d = 2 * (st & 63);  // my_rows <= 4 here; more rows loop below
     float nx = 0.f, ny = 0.f, nl = 0.f, mloc = -INFINITY, rref = -INFINITY;
     if (rr < my_rows) {
