@@ -609,9 +609,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int key_begin = blk_begin * 32;
   const int key_end = min(blk_end * 32, loop_keys);
   const int n_tiles = (blk_end - blk_begin + 3) / 4;
-  // rank c merges packed rows [c * rpc, c * rpc + rows_of(c)), rpc = ceil(kR / csize)
-  const int rpc = (kR + csize - 1) / csize;
-  auto rows_of = [&](int c) { return max(0, min(rpc, kR - c * rpc)); };
+  // rank c merges packed rows [c * rpc, c * rpc + rows_of(c)) of the m-block's
+  // rows_in rows that exist (the tile's rows past M are never exchanged: a
+  // single-row draft step with G = 4 moves 4 rows, not 32), rpc = ceil(rows_in / csize)
+  const int rows_in = max(1, min(kR, a.M - mblock * kR));
+  const int rpc = (rows_in + csize - 1) / csize;
+  auto rows_of = [&](int c) { return max(0, min(rpc, rows_in - c * rpc)); };
   const int my_rows = rows_of(rank);
   const int mrow0 = rank * rpc;
   if (warp == 0) {
