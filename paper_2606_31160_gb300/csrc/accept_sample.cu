@@ -16,10 +16,12 @@
 //           last CTA of a scene (atomic ticket, no spin) merges the chunks of
 //           every row in a fixed order, runs the K acceptance tests and
 //           records l and the normalisers of the row to draw from.
-//   draw:   grid (chunk, scene) over that one row; each CTA writes the
-//           chunk sums of the residual weights and of the target weights; the
-//           last CTA of a scene finds the chunk where the running sum passes
-//           u_K * S and scans inside it.
+//   draw:   grid (chunk of 4096 values, scene) over that one row, a thread
+//           owning 16 consecutive values of both logit rows (16-byte loads
+//           when the rows are aligned); each CTA writes the chunk sums of the
+//           residual weights and of the target weights; the last CTA of a
+//           scene finds the chunk where the running sum passes u_K * S and
+//           re-scans the same per-thread runs inside it.
 // All reductions run in a fixed order (deterministic), the weight formula
 // uses non-contractible intrinsics so both passes of the draw evaluate
 // identical values, and every spin-free ticket is re-armed after use.
@@ -380,18 +382,42 @@ __global__ void __launch_bounds__(kStreamThreads)
 }
 
 // ------------------------------------------------------------------ draw
-// Weights of element v of the draw row: residual (p - q)+ (l < K) and the
-// unnormalised target weight exp2((z_T - m_T) * c2).
-__device__ __forceinline__ void weights(const float* rt, const float* rd, const DrawInfo& di, int K,
-                                        float c2, int v, float& w_res, float& w_tgt) {
-  const float et = wexp(rt[v], di.mt, c2);
+// Weights of one element of the draw row from its two logits: residual
+// (p - q)+ (l < K) and the unnormalised target weight exp2((z_T - m_T) * c2).
+__device__ __forceinline__ void weights(float zt_v, float zd_v, const DrawInfo& di, int K, float c2, float& w_res,
+                                        float& w_tgt) {
+  const float et = wexp(zt_v, di.mt, c2);
   w_tgt = et;
   if (di.ell < K) {
     const float p = __fmul_rn(et, di.inv_zt);
-    const float q = __fmul_rn(wexp(rd[v], di.md, c2), di.inv_zd);
+    const float q = __fmul_rn(wexp(zd_v, di.md, c2), di.inv_zd);
     w_res = fmaxf(__fsub_rn(p, q), 0.f);
   } else {
     w_res = 0.f;
+  }
+}
+
+constexpr int kDrawPer = 16;                     // consecutive values a thread owns
+constexpr int kDrawChunk = kThreads * kDrawPer;  // values a CTA owns
+
+// this thread's kDrawPer logits of both rows (missing values: -inf, weight 0)
+__device__ __forceinline__ void draw_load(const float* rt, const float* rd, int v0, int V, bool vec, float (&xt)[kDrawPer],
+                                          float (&xd)[kDrawPer]) {
+  if (vec && v0 + kDrawPer <= V) {
+#pragma unroll
+    for (int q = 0; q < kDrawPer / 4; ++q) {
+      const float4 a = __ldg(reinterpret_cast<const float4*>(rt + v0) + q);
+      xt[4 * q] = a.x, xt[4 * q + 1] = a.y, xt[4 * q + 2] = a.z, xt[4 * q + 3] = a.w;
+      const float4 d = rd ? __ldg(reinterpret_cast<const float4*>(rd + v0) + q) : make_float4(0.f, 0.f, 0.f, 0.f);
+      xd[4 * q] = d.x, xd[4 * q + 1] = d.y, xd[4 * q + 2] = d.z, xd[4 * q + 3] = d.w;
+    }
+  } else {
+#pragma unroll
+    for (int e = 0; e < kDrawPer; ++e) {
+      const bool in = v0 + e < V;
+      xt[e] = in ? __ldg(rt + v0 + e) : -INFINITY;
+      xd[e] = (in && rd) ? __ldg(rd + v0 + e) : 0.f;
+    }
   }
 }
 
@@ -408,20 +434,25 @@ __device__ float block_sum(float x, float* red) {
   return t;  // valid in thread 0
 }
 
+// grid (chunk, scene): chunk c of the draw row holds values [c * kDrawChunk,
+// (c + 1) * kDrawChunk), thread t the kDrawPer consecutive values from
+// c * kDrawChunk + t * kDrawPer, summed in order.
 __global__ void __launch_bounds__(kThreads)
     sample_draw_kernel(const float* __restrict__ zt, const float* __restrict__ zd, int K, int V,
-                       float c2, int chunk, int n_chunks, const float* __restrict__ u,
+                       float c2, int n_chunks, bool vec, const float* __restrict__ u,
                        int32_t* __restrict__ tokens, const DrawInfo* __restrict__ info,
                        float2* __restrict__ sums, uint32_t* __restrict__ ticket) {
   const int c = blockIdx.x, b = blockIdx.y;
   const DrawInfo di = info[b];
   const float* rt = zt + (static_cast<long long>(b) * (K + 1) + di.ell) * V;
   const float* rd = di.ell < K ? zd + (static_cast<long long>(b) * K + di.ell) * V : nullptr;
-  const int lo = c * chunk, hi = min(V, lo + chunk);
+  float xt[kDrawPer], xd[kDrawPer];
+  draw_load(rt, rd, c * kDrawChunk + threadIdx.x * kDrawPer, V, vec, xt, xd);
   float sr = 0.f, sp = 0.f;
-  for (int v = lo + threadIdx.x; v < hi; v += kThreads) {
+#pragma unroll
+  for (int e = 0; e < kDrawPer; ++e) {
     float wr, wt;
-    weights(rt, rd, di, K, c2, v, wr, wt);
+    weights(xt[e], xd[e], di, K, c2, wr, wt);
     sr = __fadd_rn(sr, wr);
     sp = __fadd_rn(sp, wt);
   }
@@ -509,16 +540,19 @@ __global__ void __launch_bounds__(kThreads)
     }
   }
   __syncthreads();
-  // in-chunk scan: each thread owns a run of consecutive elements
-  const int clo = s_chunk * chunk, chi = min(V, clo + chunk);
-  const int per = (chunk + kThreads - 1) / kThreads;
-  const int my_lo = min(chi, clo + threadIdx.x * per), my_hi = min(chi, my_lo + per);
+  // in-chunk scan: thread t owns the same kDrawPer consecutive values as in
+  // the chunk sums above
+  const int my_lo = s_chunk * kDrawChunk + threadIdx.x * kDrawPer;
   const bool use_res = s_use_res != 0;
+  draw_load(rt, rd, my_lo, V, vec, xt, xd);
+  float w[kDrawPer];
   float tsum = 0.f;
-  for (int v = my_lo; v < my_hi; ++v) {
+#pragma unroll
+  for (int e = 0; e < kDrawPer; ++e) {
     float wr, wt;
-    weights(rt, rd, di, K, c2, v, wr, wt);
-    tsum = __fadd_rn(tsum, use_res ? wr : wt);
+    weights(xt[e], xd[e], di, K, c2, wr, wt);
+    w[e] = use_res ? wr : wt;
+    tsum = __fadd_rn(tsum, w[e]);
   }
   // exclusive prefix of the thread sums: warp scan + warp offsets (fixed)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -534,15 +568,14 @@ __global__ void __launch_bounds__(kThreads)
   if (lane == 31) s_wtot[warp] = incl;
   __syncthreads();
   float woff = 0.f;
-  for (int w = 0; w < warp; ++w) woff = __fadd_rn(woff, s_wtot[w]);
+  for (int q = 0; q < warp; ++q) woff = __fadd_rn(woff, s_wtot[q]);
   float run = __fadd_rn(s_base, __fadd_rn(woff, excl));
   int cand = 0x7fffffff, last_pos = -1;
-  for (int v = my_lo; v < my_hi; ++v) {
-    float wr, wt;
-    weights(rt, rd, di, K, c2, v, wr, wt);
-    const float w = use_res ? wr : wt;
-    if (w > 0.f) last_pos = v;
-    run = __fadd_rn(run, w);
+#pragma unroll
+  for (int e = 0; e < kDrawPer; ++e) {
+    const int v = my_lo + e;
+    if (w[e] > 0.f) last_pos = v;
+    run = __fadd_rn(run, w[e]);
     if (cand == 0x7fffffff && run > s_target) cand = v;
   }
   // block min of candidates, block max of the last positive weight
@@ -559,11 +592,11 @@ __global__ void __launch_bounds__(kThreads)
   __syncthreads();
   if (threadIdx.x == 0) {
     int best = 0x7fffffff, lp = -1;
-    for (int w = 0; w < kThreads / 32; ++w) {
-      best = min(best, s_cand[w]);
-      lp = max(lp, s_lastp[w]);
+    for (int q = 0; q < kThreads / 32; ++q) {
+      best = min(best, s_cand[q]);
+      lp = max(lp, s_lastp[q]);
     }
-    const int tok = best != 0x7fffffff ? best : (lp >= 0 ? lp : clo);
+    const int tok = best != 0x7fffffff ? best : (lp >= 0 ? lp : s_chunk * kDrawChunk);
     tokens[static_cast<long long>(b) * (K + 1) + di.ell] = tok;
     ticket[b] = 0;
   }
@@ -586,8 +619,7 @@ Plan plan(int V) {
   p.chunk_scalar = 4096;
   while ((V + p.chunk_scalar - 1) / p.chunk_scalar > kMaxChunks) p.chunk_scalar *= 2;
   p.n_scalar = (V + p.chunk_scalar - 1) / p.chunk_scalar;
-  p.chunk2 = 2048;
-  while ((V + p.chunk2 - 1) / p.chunk2 > kMaxChunks) p.chunk2 *= 2;
+  p.chunk2 = kDrawChunk;
   p.n2 = (V + p.chunk2 - 1) / p.chunk2;
   return p;
 }
@@ -656,7 +688,7 @@ extern "C" sd_status sd_accept_sample(const float* z_target, const float* z_draf
                                       size_t ws_bytes, sd_stream_t stream) {
   if (B < 0 || K < 0 || V <= 0) return SD_ERR_INVALID_ARG;
   if (!(temperature > 0.f) || !isfinite(temperature)) return SD_ERR_INVALID_ARG;
-  if (K > 128 || B > 65535) return SD_ERR_UNSUPPORTED;
+  if (K > 128 || B > 65535 || (V + kDrawChunk - 1) / kDrawChunk > kMaxChunks) return SD_ERR_UNSUPPORTED;
   if (B == 0) return SD_OK;
   if (!z_target || !u || !n_emit || !tokens || (K > 0 && (!z_draft || !draft)))
     return SD_ERR_INVALID_ARG;
@@ -695,8 +727,8 @@ extern "C" sd_status sd_accept_sample(const float* z_target, const float* z_draf
     sample_stats_kernel<false><<<dim3(p.n1, 2 * K + 1, B), kThreads, 0, st>>>(
         z_target, z_draft, K, V, c2, p.chunk1, p.n1, draft, u, n_emit, tokens, part, dlogit, ticket1, info);
   SD_CHECK_LAUNCH();
-  sample_draw_kernel<<<dim3(p.n2, B), kThreads, 0, st>>>(z_target, z_draft, K, V, c2, p.chunk2,
-                                                          p.n2, u, tokens, info, sums, ticket2);
+  sample_draw_kernel<<<dim3(p.n2, B), kThreads, 0, st>>>(z_target, z_draft, K, V, c2, p.n2, p.vec, u, tokens,
+                                                          info, sums, ticket2);
   SD_CHECK_LAUNCH();
   return SD_OK;
 }

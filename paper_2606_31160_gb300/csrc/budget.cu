@@ -5,16 +5,22 @@
 // attention among the non-visual keys (renormalised), divided by the log of
 // their number.
 //
-// A diagnostic beside the verify path, exact rather than fast: one CTA per
-// (query head, scene) takes the rows in groups of 8; for each group it makes
-// two passes over the visible keys on the CUDA cores (fp32 dot products of the
-// bf16 rows): the row maxima, then the weights exp(s - max) summed per segment
-// together with the entropy term sum w (s - max). Block reductions run in a
-// fixed order.
+// A diagnostic beside the verify path. One thread-block cluster per (KV head,
+// scene) splits the visible keys over its S CTAs; the G * R query rows of the
+// KV head (packed row p = i * G + j: new row i, query head j of the group)
+// take their scores from bf16 tensor-core products (mma.sync m16n8k16, fp32
+// accumulation), 16 rows by 8 keys a product, the keys' fragments read
+// straight from the cache. Every thread folds the scores it holds into an
+// online state per row, relative to a running maximum m:
+//   v, t, g = sum of exp(y - m) over the visual, trajectory / prompt-text and
+//             generated keys, n = sum over the non-visual keys of
+//             exp(y - m) (y - m),        y = q . k * scale,
+// the states merge in a fixed order over the lanes and warps, then over the
+// cluster's CTAs through distributed shared memory (rank 0 takes the S
+// partials), and
 //
-//   entropy = (ln l' - T' / l') / ln N'     l' = sum of the non-visual weights,
-//                                           T' = sum over them of w (s - max),
-//                                           N' = number of non-visual keys
+//   entropy = (ln l' - n / l') / ln N'     l' = t + g, N' = number of
+//                                          non-visual keys the row sees
 #include "common.cuh"
 
 #include <math.h>
@@ -25,133 +31,237 @@ namespace {
 
 constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
-constexpr int kGroup = 8;  // rows per group
 constexpr float kLog2e = 1.4426950408889634f;
 
-// scores of key row kr (D bf16, 16-byte aligned) against the group's rows
-template <int D>
-__device__ __forceinline__ void key_scores(const __nv_bfloat16* kr, const float (*qs)[D], float (&acc)[kGroup]) {
-#pragma unroll
-  for (int r = 0; r < kGroup; ++r) acc[r] = 0.f;
-#pragma unroll 4
-  for (int c = 0; c < D / 8; ++c) {
-    const uint4 w = __ldg(reinterpret_cast<const uint4*>(kr) + c);
-    const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
-    float kf[8];
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      kf[2 * j] = sd_bf16_lo(ws[j]);
-      kf[2 * j + 1] = sd_bf16_hi(ws[j]);
+__device__ __forceinline__ float ex2f(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+// Online state of one row (see the header): sums relative to the maximum m.
+struct RowState {
+  float m, v, t, g, n;
+};
+
+__device__ __forceinline__ RowState row_empty() { return RowState{-INFINITY, 0.f, 0.f, 0.f, 0.f}; }
+
+// fold two scores (y[e] of segment seg[e]; -inf: masked) whose block
+// maximum over the row's lanes is bm: one rescale of the state at most
+__device__ __forceinline__ void row_block(RowState& s, const float (&y)[2], const int (&seg)[2], float bm) {
+  if (bm == -INFINITY) return;
+  if (bm > s.m) {
+    if (s.m != -INFINITY) {
+      const float a = ex2f((s.m - bm) * kLog2e);
+      s.n = a * fmaf(s.m - bm, s.t + s.g, s.n);
+      s.v *= a;
+      s.t *= a;
+      s.g *= a;
     }
+    s.m = bm;
+  }
 #pragma unroll
-    for (int r = 0; r < kGroup; ++r)
-#pragma unroll
-      for (int e = 0; e < 8; ++e) acc[r] = fmaf(qs[r][c * 8 + e], kf[e], acc[r]);
+  for (int e = 0; e < 2; ++e) {
+    const float d = y[e] - s.m, w = ex2f(d * kLog2e);  // masked: ex2(-inf) = 0
+    if (seg[e] == 0) {
+      s.v += w;
+    } else {
+      if (seg[e] == 1) s.t += w;
+      else s.g += w;
+      if (w > 0.f) s.n = fmaf(w, d, s.n);
+    }
   }
 }
 
-// block-wide reduction of v[r] (max or sum), fixed order; result in out[r]
-template <bool kMax>
-__device__ __forceinline__ void block_reduce(float (&v)[kGroup], float (*red)[kGroup], float* out) {
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-#pragma unroll
-  for (int r = 0; r < kGroup; ++r)
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      const float x = __shfl_xor_sync(0xffffffffu, v[r], o);
-      v[r] = kMax ? fmaxf(v[r], x) : v[r] + x;
-    }
-  if (lane == 0)
-#pragma unroll
-    for (int r = 0; r < kGroup; ++r) red[warp][r] = v[r];
-  __syncthreads();
-  if (threadIdx.x < kGroup) {
-    float a = red[0][threadIdx.x];
-    for (int w = 1; w < kWarps; ++w) a = kMax ? fmaxf(a, red[w][threadIdx.x]) : a + red[w][threadIdx.x];
-    out[threadIdx.x] = a;
+// a := merge(a, b), both relative to their own maxima
+__device__ __forceinline__ void row_merge(RowState& a, const RowState& b) {
+  if (b.m == -INFINITY) return;
+  if (a.m == -INFINITY) {
+    a = b;
+    return;
   }
-  __syncthreads();
+  const float M = fmaxf(a.m, b.m);
+  const float fa = ex2f((a.m - M) * kLog2e), fb = ex2f((b.m - M) * kLog2e);
+  const float n = fa * fmaf(a.m - M, a.t + a.g, a.n) + fb * fmaf(b.m - M, b.t + b.g, b.n);
+  a.v = fa * a.v + fb * b.v;
+  a.t = fa * a.t + fb * b.t;
+  a.g = fa * a.g + fb * b.g;
+  a.n = n;
+  a.m = M;
 }
+
+__device__ __forceinline__ RowState row_shfl(const RowState& s, int o) {
+  return RowState{__shfl_xor_sync(0xffffffffu, s.m, o), __shfl_xor_sync(0xffffffffu, s.v, o),
+                  __shfl_xor_sync(0xffffffffu, s.t, o), __shfl_xor_sync(0xffffffffu, s.g, o),
+                  __shfl_xor_sync(0xffffffffu, s.n, o)};
+}
+
+__device__ __forceinline__ uint32_t cta_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+// 8 floats (two 16-byte loads) of CTA `rank`'s copy of p
+__device__ __forceinline__ void ld_cluster8(const float* p, uint32_t rank, float (&v)[8]) {
+  uint32_t a;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(a) : "r"(static_cast<uint32_t>(__cvta_generic_to_shared(p))), "r"(rank));
+  asm volatile("ld.shared::cluster.v4.f32 {%0,%1,%2,%3}, [%4];" : "=f"(v[0]), "=f"(v[1]), "=f"(v[2]), "=f"(v[3]) : "r"(a) : "memory");
+  asm volatile("ld.shared::cluster.v4.f32 {%0,%1,%2,%3}, [%4];" : "=f"(v[4]), "=f"(v[5]), "=f"(v[6]), "=f"(v[7]) : "r"(a + 16) : "memory");
+}
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void mma_bf16(float (&c)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+  asm(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+      "{%0,%1,%2,%3};"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+// grid (S, Hkv, B), clusters of S CTAs along x: CTA `rank` of the cluster of
+// (KV head kvh, scene b) takes keys [rank * n / S, (rank + 1) * n / S) of the
+// n = len[b] keys the scene holds, for the M = G * R packed rows in passes of
+// kTiles tiles of 16 rows (lane l of a warp holds rows l / 4 and l / 4 + 8 of
+// a tile, keys 2 (l % 4) and 2 (l % 4) + 1 of every 8-key block); a block's
+// key fragments serve every tile of the pass.
+constexpr int kTiles = 2;
+constexpr int kPassRows = 16 * kTiles;
 
 template <int D>
 __global__ void __launch_bounds__(kThreads)
     budget_kernel(const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* __restrict__ kc,
                   const int32_t* __restrict__ len, const int32_t* __restrict__ n_visual, int R, int Hq,
                   int Hkv, int cap, float scale, float* __restrict__ mass, float* __restrict__ entropy) {
-  __shared__ float qs[kGroup][D];
-  __shared__ float red[kWarps][kGroup];
-  __shared__ float s_max[kGroup], s_lv[kGroup], s_lt[kGroup], s_lg[kGroup], s_tn[kGroup];
-  const int h = blockIdx.x, b = blockIdx.y;
-  const int g = h / (Hq / Hkv);
+  __shared__ RowState red[kWarps][kPassRows];
+  __shared__ __align__(16) float part[kPassRows][8];  // this CTA's state per row of the pass (read by rank 0)
+  __shared__ RowState gath[kPassRows][16];           // rank 0: every CTA's state per row
+  const int kvh = blockIdx.y, b = blockIdx.z;
+  const int S = gridDim.x;
+  const uint32_t rank = cta_rank();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int gq = lane >> 2, tq = lane & 3;
+  const int G = Hq / Hkv, M = G * R;
   const int n_keys = len[b], L = n_keys - R;
   int nv = n_visual[b];
-  if (L < 0 || n_keys > cap) {
-    if (threadIdx.x == 0 && h == 0) sd_set_error(SD_DEVERR_LENGTH);
-    return;
-  }
-  if (nv < 0 || nv > L) {
-    if (threadIdx.x == 0 && h == 0) sd_set_error(SD_DEVERR_LENGTH);
+  // every CTA of a cluster runs the same barriers, so a bad length only
+  // empties the key ranges (and writes nothing)
+  const bool ok = L >= 0 && n_keys <= cap;
+  if (!ok && threadIdx.x == 0 && kvh == 0 && rank == 0) sd_set_error(SD_DEVERR_LENGTH);
+  if (ok && (nv < 0 || nv > L)) {
+    if (threadIdx.x == 0 && kvh == 0 && rank == 0) sd_set_error(SD_DEVERR_LENGTH);
     nv = nv < 0 ? 0 : L;
   }
-  const __nv_bfloat16* kb = kc + (static_cast<long long>(b) * Hkv + g) * cap * D;
-  for (int r0 = 0; r0 < R; r0 += kGroup) {
-    const int nr = min(kGroup, R - r0);
-    for (int idx = threadIdx.x; idx < kGroup * D; idx += kThreads) {
-      const int r = idx / D, d = idx % D;
-      qs[r][d] = r < nr ? __bfloat162float(q[((static_cast<long long>(b) * R + r0 + r) * Hq + h) * D + d]) : 0.f;
-    }
-    __syncthreads();
-    const int last = L + r0 + nr;  // keys visible to the group's last row
-    // pass 1: row maxima of the scaled scores
-    float v[kGroup];
+  const int k_lo = ok ? static_cast<int>(static_cast<long long>(rank) * n_keys / S) : 0;
+  const int k_hi = ok ? static_cast<int>(static_cast<long long>(rank + 1) * n_keys / S) : 0;
+  const __nv_bfloat16* kb = kc + (static_cast<long long>(b) * Hkv + kvh) * cap * D;
+  for (int m0 = 0; m0 < M; m0 += kPassRows) {
+    // query fragments of rows m0 + 16 u + gq and + 8 (zero past M); the keys
+    // each row sees (causal over the new rows); one state per row
+    uint32_t af[kTiles][D / 16][4];
+    int lim[kTiles][2];
+    RowState st[kTiles][2];
 #pragma unroll
-    for (int r = 0; r < kGroup; ++r) v[r] = -INFINITY;
-    for (int k = threadIdx.x; k < last; k += kThreads) {
-      float acc[kGroup];
-      key_scores<D>(kb + static_cast<long long>(k) * D, qs, acc);
+    for (int u = 0; u < kTiles; ++u)
 #pragma unroll
-      for (int r = 0; r < kGroup; ++r)
-        if (r < nr && k <= L + r0 + r) v[r] = fmaxf(v[r], acc[r] * scale);
-    }
-    block_reduce<true>(v, red, s_max);
-    // pass 2: weights per segment and the non-visual entropy term
-    float lv[kGroup], lt[kGroup], lg[kGroup], tn[kGroup];
+      for (int h2 = 0; h2 < 2; ++h2) {
+        const int p = m0 + 16 * u + gq + 8 * h2, i = p / G;
+        const __nv_bfloat16* qr = q + ((static_cast<long long>(b) * R + i) * Hq + kvh * G + (p - i * G)) * D;
 #pragma unroll
-    for (int r = 0; r < kGroup; ++r) lv[r] = lt[r] = lg[r] = tn[r] = 0.f;
-    for (int k = threadIdx.x; k < last; k += kThreads) {
-      float acc[kGroup];
-      key_scores<D>(kb + static_cast<long long>(k) * D, qs, acc);
+        for (int ks = 0; ks < D / 16; ++ks) {
+          const int d0 = ks * 16 + 2 * tq;
+          af[u][ks][h2] = p < M ? *reinterpret_cast<const uint32_t*>(qr + d0) : 0u;
+          af[u][ks][h2 + 2] = p < M ? *reinterpret_cast<const uint32_t*>(qr + d0 + 8) : 0u;
+        }
+        lim[u][h2] = p < M ? L + i : -1;
+        st[u][h2] = row_empty();
+      }
+#pragma unroll 1
+    for (int kb0 = k_lo + 8 * warp; kb0 < k_hi; kb0 += 8 * kWarps) {
+      // this lane's key of the block for the B fragments (clamped into the range)
+      const int kn = min(kb0 + gq, k_hi - 1);
+      const __nv_bfloat16* kr = kb + static_cast<long long>(kn) * D;
+      uint32_t bf[D / 16][2];
 #pragma unroll
-      for (int r = 0; r < kGroup; ++r) {
-        if (r < nr && k <= L + r0 + r) {
-          const float y = acc[r] * scale - s_max[r];
-          const float w = exp2f(y * kLog2e);
-          if (k < nv) {
-            lv[r] += w;
-          } else {
-            if (k < L) lt[r] += w;
-            else lg[r] += w;
-            tn[r] = fmaf(w, y, tn[r]);
+      for (int ks = 0; ks < D / 16; ++ks) {
+        const int d0 = ks * 16 + 2 * tq;
+        bf[ks][0] = __ldg(reinterpret_cast<const uint32_t*>(kr + d0));
+        bf[ks][1] = __ldg(reinterpret_cast<const uint32_t*>(kr + d0 + 8));
+      }
+      int seg[2];
+#pragma unroll
+      for (int e = 0; e < 2; ++e) {
+        const int key = kb0 + 2 * tq + e;
+        seg[e] = key < nv ? 0 : (key < L ? 1 : 2);
+      }
+#pragma unroll
+      for (int u = 0; u < kTiles; ++u) {
+        float c[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int ks = 0; ks < D / 16; ++ks) mma_bf16(c, af[u][ks], bf[ks][0], bf[ks][1]);
+        // scaled, masked scores; the block's maximum per row over the quad of
+        // lanes that holds the row (all four then share the running maximum)
+#pragma unroll
+        for (int h2 = 0; h2 < 2; ++h2) {
+          float y[2];
+#pragma unroll
+          for (int e = 0; e < 2; ++e) {
+            const int key = kb0 + 2 * tq + e;
+            y[e] = (key < k_hi && key <= lim[u][h2]) ? c[2 * h2 + e] * scale : -INFINITY;
           }
+          float bm = fmaxf(y[0], y[1]);
+#pragma unroll
+          for (int o = 1; o < 4; o <<= 1) bm = fmaxf(bm, __shfl_xor_sync(0xffffffffu, bm, o));
+          row_block(st[u][h2], y, seg, bm);
         }
       }
     }
-    block_reduce<false>(lv, red, s_lv);
-    block_reduce<false>(lt, red, s_lt);
-    block_reduce<false>(lg, red, s_lg);
-    block_reduce<false>(tn, red, s_tn);
-    if (threadIdx.x < nr) {
-      const int r = threadIdx.x, i = r0 + r;
-      const float tot = s_lv[r] + s_lt[r] + s_lg[r];
-      const long long o = (static_cast<long long>(b) * R + i) * Hq + h;
-      mass[o * 3 + 0] = s_lv[r] / tot;
-      mass[o * 3 + 1] = s_lt[r] / tot;
-      mass[o * 3 + 2] = s_lg[r] / tot;
-      const float lnv = s_lt[r] + s_lg[r];
-      const int n_rest = (L - nv) + i + 1;
-      entropy[o] = (n_rest > 1 && lnv > 0.f) ? (logf(lnv) - s_tn[r] / lnv) / logf(static_cast<float>(n_rest)) : 0.f;
+    // the four lanes of a row (fixed butterfly), then the warps in order
+#pragma unroll
+    for (int u = 0; u < kTiles; ++u)
+#pragma unroll
+      for (int h2 = 0; h2 < 2; ++h2) {
+#pragma unroll
+        for (int o = 1; o < 4; o <<= 1) row_merge(st[u][h2], row_shfl(st[u][h2], o));
+        if (tq == 0) red[warp][16 * u + gq + 8 * h2] = st[u][h2];
+      }
+    __syncthreads();
+    if (threadIdx.x < kPassRows) {
+      RowState a = red[0][threadIdx.x];
+      for (int w = 1; w < kWarps; ++w) row_merge(a, red[w][threadIdx.x]);
+      part[threadIdx.x][0] = a.m;
+      part[threadIdx.x][1] = a.v;
+      part[threadIdx.x][2] = a.t;
+      part[threadIdx.x][3] = a.g;
+      part[threadIdx.x][4] = a.n;
     }
-    __syncthreads();  // qs is rewritten by the next group
+    cluster_sync_all();  // every CTA's part is written
+    const int nr = min(kPassRows, M - m0);
+    if (rank == 0) {
+      // one thread a (row, CTA): the S partial states travel at once
+      for (int idx = threadIdx.x; idx < nr * S; idx += kThreads) {
+        const int r = idx / S, cc = idx % S;
+        float v[8];
+        ld_cluster8(&part[r][0], cc, v);
+        gath[r][cc] = RowState{v[0], v[1], v[2], v[3], v[4]};
+      }
+      __syncthreads();
+    }
+    if (rank == 0 && threadIdx.x < nr && ok) {
+      const int p = m0 + threadIdx.x, i = p / G, h = kvh * G + (p - i * G);
+      RowState a = row_empty();
+      for (int cc = 0; cc < S; ++cc) row_merge(a, gath[threadIdx.x][cc]);
+      const float tot = a.v + a.t + a.g;
+      const long long o = (static_cast<long long>(b) * R + i) * Hq + h;
+      mass[o * 3 + 0] = a.v / tot;
+      mass[o * 3 + 1] = a.t / tot;
+      mass[o * 3 + 2] = a.g / tot;
+      const float lnv = a.t + a.g;
+      const int n_rest = (L - nv) + i + 1;
+      entropy[o] = (n_rest > 1 && lnv > 0.f) ? (logf(lnv) - a.n / lnv) / logf(static_cast<float>(n_rest)) : 0.f;
+    }
+    cluster_sync_all();  // rank 0 has read every part; red and part may be rewritten
   }
 }
 
@@ -171,13 +281,43 @@ extern "C" sd_status sd_attention_budget(const void* q, const sd_kv_cache* cache
   if (!(scale >= 0.f) || !isfinite(scale)) return SD_ERR_INVALID_ARG;
   const float sc = scale > 0.f ? scale : static_cast<float>(1.0 / sqrt(static_cast<double>(D)));
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-  const dim3 grid(Hq, B);
+  // cluster size: the smallest power of two (up to 16) that leaves each CTA
+  // at most 256 keys of the largest scene (32 keys a warp)
+  int S = 1;
+  while (S < 16 && static_cast<long long>(cap) > 256LL * S) S *= 2;
   const auto* qq = static_cast<const __nv_bfloat16*>(q);
   const auto* kk = static_cast<const __nv_bfloat16*>(cache->k);
-  if (D == 128)
-    budget_kernel<128><<<grid, kThreads, 0, st>>>(qq, kk, cache->len, n_visual, R, Hq, Hkv, cap, sc, mass, entropy);
-  else
-    budget_kernel<64><<<grid, kThreads, 0, st>>>(qq, kk, cache->len, n_visual, R, Hq, Hkv, cap, sc, mass, entropy);
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = S;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.gridDim = dim3(S, Hkv, B);
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.stream = st;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cudaError_t e;
+  // clusters of 16 are non-portable: allowed once per device and kernel
+  static bool allowed[64][2];
+  int dev = 0;
+  if (S > 8 && cudaGetDevice(&dev) == cudaSuccess && dev >= 0 && dev < 64 && !allowed[dev][D == 128]) {
+    if (D == 128) cudaFuncSetAttribute(budget_kernel<128>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    else cudaFuncSetAttribute(budget_kernel<64>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    allowed[dev][D == 128] = true;
+  }
+  if (D == 128) {
+    e = cudaLaunchKernelEx(&cfg, budget_kernel<128>, qq, kk, static_cast<const int32_t*>(cache->len), n_visual, R, Hq,
+                           Hkv, cap, sc, mass, entropy);
+  } else {
+    e = cudaLaunchKernelEx(&cfg, budget_kernel<64>, qq, kk, static_cast<const int32_t*>(cache->len), n_visual, R, Hq,
+                           Hkv, cap, sc, mass, entropy);
+  }
+  if (e != cudaSuccess) {
+    (void)cudaGetLastError();
+    return SD_ERR_CUDA;
+  }
   SD_CHECK_LAUNCH();
   return SD_OK;
 }
