@@ -223,7 +223,9 @@ sd_status sd_set_cluster_size(int cluster_size);
  *   q: [B][R][Hq][D] bf16 (rotated), cache: keys appended (len includes R),
  *   n_visual: int32 [B] device, mass: fp32 [B][R][Hq][3] device,
  *   entropy: fp32 [B][R][Hq] device; scale: 0 selects 1/sqrt(D).
- * Exact rather than fast: two fp32 passes over the keys on the CUDA cores.
+ * One pass over the keys: bf16 tensor-core scores with fp32 accumulation,
+ * fp32 sums with a running maximum per row (within 1e-4 of a float64 reference
+ * on the target layer).
  * D in {64, 128}, Hq % Hkv == 0. A scene with len[b] < R or len[b] >
  * capacity sets SD_DEVERR_LENGTH and is left unwritten; n_visual[b] outside
  * [0, L_b] sets it too and is clamped.
