@@ -1524,6 +1524,8 @@ extern "C" sd_status sd_set_cluster_size(int cluster_size) {
   return SD_ERR_INVALID_ARG;
 }
 
+int sd_internal_forced_cluster() { return g_forced_cluster.load(); }
+
 static TcPlan tc_plan(int B, int R, int Hq, int Hkv, int D, int cap, int max_cs = 16) {
   TcPlan p;
   if (!tc_enabled() || D != kD || Hkv <= 0 || Hq % Hkv || R <= 0) return p;

@@ -55,6 +55,13 @@ extern "C" sd_status sd_verify_layer(void* q, void* k_new, const void* v_new, co
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   auto* ticket = static_cast<uint32_t*>(workspace);
   bool handled = false;
+  // up to 16 packed rows per KV head (the draft's single-row steps): the
+  // small-tile kernel over every SM; larger tiles: the tcgen05 kernel
+  {
+    const sd_status s = sd_internal_verify_layer_dec(q, k_new, v_new, pos, tab, cache, out, R, Hq, scale_log2,
+                                                     ticket, flags & SD_LAYER_PREFIX_EARLY, block, st, &handled);
+    if (handled) return s;
+  }
   const sd_status s = sd_internal_verify_layer_tc(q, k_new, v_new, pos, tab, cache, out, R, Hq,
                                                   scale_log2, ticket, flags & SD_LAYER_PREFIX_EARLY,
                                                   block, st, &handled);
