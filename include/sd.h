@@ -214,6 +214,16 @@ sd_status sd_verify_attention_ex(const void* q, const sd_kv_cache* cache, void* 
 sd_status sd_set_cluster_size(int cluster_size);
 
 /*
+ * Which kernel serves a shape on the CURRENT device: "small-tile",
+ * "tcgen05" or "mma.sync" for sd_verify_attention (layer = 0), and for
+ * sd_verify_layer (layer = 1, or 2 with SD_LAYER_BLOCK_MASK; "three kernels"
+ * when the layer runs as the rotation, append and attention kernels in
+ * sequence); "unsupported" for a shape neither call takes. Host-only, no
+ * device work; a static string.
+ */
+const char* sd_verify_kernel(int B, int R, int Hq, int Hkv, int D, int capacity, int layer);
+
+/*
  * Attention budget of the verify rows (Sec. 4.2 "Empirical confirmation",
  * Table tab:attn-budget), a diagnostic beside the verify path. For scene b,
  * query head h and row i, with p the softmax of q . k * scale over the keys
@@ -274,10 +284,10 @@ size_t sd_verify_layer_workspace(int B, int R, int Hq, int Hkv, int D, int capac
  *   SD_LAYER_BLOCK_MASK: the attention uses the block mask (as
  *   SD_ATTN_BLOCK_MASK of sd_verify_attention_ex).
  * For head_dim 128 this is one kernel: the small-tile kernel for G * R <= 16
- * (the draft's single-row decode steps; block mask included), the tcgen05
- * kernel for 16 < G * R <= 128 and R <= 31 (R <= 16 when G * R <= 32; the
+ * when the layer is block-masked or B * Hkv >= 8, the tcgen05 kernel for the
+ * other shapes with G * R <= 128 and R <= 31 (R <= 16 when G * R <= 32; the
  * block mask only when G * R > 32); other shapes run the three kernels in
- * sequence. A scene whose append would pass the
+ * sequence (sd_verify_kernel names the choice). A scene whose append would pass the
  * capacity sets SD_DEVERR_KV_OVERFLOW and is left untouched.
  */
 sd_status sd_verify_layer(void* q, void* k_new, const void* v_new, const int32_t* pos,

@@ -1551,6 +1551,12 @@ bool sd_internal_tc_serves(int B, int R, int Hq, int Hkv, int D, int cap) {
   return tc_plan(B, R, Hq, Hkv, D, cap).cs > 0;
 }
 
+bool sd_internal_tc_serves_layer(int B, int R, int Hq, int Hkv, int D, int cap) {
+  if (R > 32) return false;
+  const TcPlan plan = tc_plan(B, R, Hq, Hkv, D, cap, 32 - R);
+  return plan.cs > 0 && R <= (plan.rows == 32 ? Cfg<32>::kMaxNew : Cfg<64>::kMaxNew);
+}
+
 template <int kR, int kMode>
 static sd_status launch_tc(const sd_kv_cache* cache, const TcArgs& a, const RopeTable& tab,
                            const TcPlan& plan, bool pdl, cudaStream_t stream) {

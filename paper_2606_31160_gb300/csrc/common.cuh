@@ -43,8 +43,10 @@ cudaError_t sd_take_error_decode(uint32_t* bits);
 sd_status sd_internal_verify_attention_tc(const void* q, const sd_kv_cache* cache, void* out,
                                           int R, int Hq, float scale_log2, int flags, cudaStream_t stream,
                                           bool* handled);
-// Whether the tcgen05 path serves this shape on the current device.
+// Whether the tcgen05 path serves this shape on the current device: the
+// attention, and the fused layer without the block mask.
 bool sd_internal_tc_serves(int B, int R, int Hq, int Hkv, int D, int cap);
+bool sd_internal_tc_serves_layer(int B, int R, int Hq, int Hkv, int D, int cap);
 
 struct RopeTable;
 // The fused verify layer on the tcgen05 path (attention_tc.cu); *handled is
@@ -59,7 +61,7 @@ int sd_internal_forced_cluster();
 
 // The small-tile kernel (decode.cu): head_dim 128 and G * R <= 16 query rows
 // per KV head. Whether it serves a shape on the current device:
-bool sd_internal_decode_serves(int B, int R, int Hq, int Hkv, int D, int cap, bool layer);
+bool sd_internal_decode_serves(int B, int R, int Hq, int Hkv, int D, int cap, bool layer, bool block = false);
 // Verify attention / the fused verify layer on it; *handled is set when the
 // shape is served and the kernel launched.
 sd_status sd_internal_verify_attention_dec(const void* q, const sd_kv_cache* cache, void* out, int R, int Hq,

@@ -619,19 +619,22 @@ __device__ __forceinline__ void decode_body(const CUtensorMap* tm_k, const CUten
     for (int idx = tid; idx < M * (kD / 4); idx += kCT) {
       const int row = idx >> 5;
       const int col = (idx & 31) * 4;
-      float4 ov[kCW];
-#pragma unroll
-      for (int w = 0; w < kCW; ++w) ov[w] = *reinterpret_cast<const float4*>(wpart + w * kPartFloats + row * kLd + col);
-      const float4 f0 = *reinterpret_cast<const float4*>(wf + row * kCW);
-      const float4 f1 = *reinterpret_cast<const float4*>(wf + row * kCW + 4);
-      const float fw[kCW] = {f0.x, f0.y, f0.z, f0.w, f1.x, f1.y, f1.z, f1.w};
       float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
-      for (int w = 0; w < kCW; ++w) {
-        acc.x = fmaf(fw[w], ov[w].x, acc.x);
-        acc.y = fmaf(fw[w], ov[w].y, acc.y);
-        acc.z = fmaf(fw[w], ov[w].z, acc.z);
-        acc.w = fmaf(fw[w], ov[w].w, acc.w);
+      for (int w4 = 0; w4 < kCW; w4 += 4) {
+        float4 ov[4];
+#pragma unroll
+        for (int w = 0; w < 4; ++w)
+          ov[w] = *reinterpret_cast<const float4*>(wpart + (w4 + w) * kPartFloats + row * kLd + col);
+        const float4 fv = *reinterpret_cast<const float4*>(wf + row * kCW + w4);
+        const float fw[4] = {fv.x, fv.y, fv.z, fv.w};
+#pragma unroll
+        for (int w = 0; w < 4; ++w) {
+          acc.x = fmaf(fw[w], ov[w].x, acc.x);
+          acc.y = fmaf(fw[w], ov[w].y, acc.y);
+          acc.z = fmaf(fw[w], ov[w].z, acc.z);
+          acc.w = fmaf(fw[w], ov[w].w, acc.w);
+        }
       }
       *reinterpret_cast<float4*>(part + row * kLd + col) = acc;
     }
@@ -734,8 +737,7 @@ __device__ __forceinline__ void decode_body(const CUtensorMap* tm_k, const CUten
 }
 
 template <bool kLayer>
-// (one CTA per SM: up to 200 registers a thread for the 288 threads)
-__global__ void __maxnreg__(200)
+__global__ void __launch_bounds__(kThreads, 1)
     verify_decode_kernel(const __grid_constant__ CUtensorMap tm_k,
                          const __grid_constant__ CUtensorMap tm_v, const DecArgs a,
                          const RopeTable tab) {
@@ -904,6 +906,15 @@ int pick_size(bool layer, int B, int Hkv, int cap) {
   return 0;
 }
 
+// The fused layer takes this kernel for block-masked layers (the 32-row
+// tcgen05 layer kernel is causal only) and once the launch has at least 8
+// (scene, KV head) clusters; a single scene of the draft's 4 KV heads runs
+// faster on the tcgen05 layer kernel (8.2 against 9.0 us a step, measured),
+// whose 128-key tensor-memory products outrun 16-row mma.sync tiles there.
+bool layer_preferred(int B, int Hkv, int block) {
+  return block != 0 || static_cast<long long>(B) * Hkv >= 8;
+}
+
 bool shape_served(int R, int Hq, int Hkv, int D) {
   if (D != kD || Hkv <= 0 || Hq % Hkv || R <= 0 || R > kMaxNew) return false;
   return (Hq / Hkv) * R <= kRows;
@@ -938,8 +949,9 @@ sd_status launch(const sd_kv_cache* cache, const DecArgs& a, const RopeTable& ta
 
 }  // namespace
 
-bool sd_internal_decode_serves(int B, int R, int Hq, int Hkv, int D, int cap, bool layer) {
+bool sd_internal_decode_serves(int B, int R, int Hq, int Hkv, int D, int cap, bool layer, bool block) {
   if (!shape_served(R, Hq, Hkv, D) || B <= 0 || B > 65535 || Hkv > 65535) return false;
+  if (layer && !layer_preferred(B, Hkv, block)) return false;
   return pick_size(layer, B, Hkv, cap) > 0;
 }
 
@@ -974,7 +986,7 @@ sd_status sd_internal_verify_layer_dec(void* q, void* k_new, const void* v_new, 
                                        cudaStream_t stream, bool* handled) {
   *handled = false;
   const int B = cache->batch, Hkv = cache->n_kv_heads;
-  if (!shape_served(R, Hq, Hkv, cache->head_dim) || B > 65535) return SD_OK;
+  if (!layer_preferred(B, Hkv, block) || !shape_served(R, Hq, Hkv, cache->head_dim) || B > 65535) return SD_OK;
   const int cs = pick_size(true, B, Hkv, cache->capacity);
   if (cs <= 0) return SD_OK;
   DecArgs a = {};

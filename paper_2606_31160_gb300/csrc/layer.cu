@@ -75,3 +75,12 @@ extern "C" sd_status sd_verify_layer(void* q, void* k_new, const void* v_new, co
                                 static_cast<char*>(workspace) + kTicketBytes(B, Hkv),
                                 ws_bytes - kTicketBytes(B, Hkv), stream);
 }
+
+extern "C" const char* sd_verify_kernel(int B, int R, int Hq, int Hkv, int D, int capacity, int layer) {
+  if (B <= 0 || R <= 0 || Hq <= 0 || Hkv <= 0 || capacity <= 0 || Hq % Hkv || (D != 64 && D != 128) ||
+      static_cast<long long>(Hq / Hkv) * R > 128)
+    return "unsupported";
+  if (sd_internal_decode_serves(B, R, Hq, Hkv, D, capacity, layer != 0, layer > 1)) return "small-tile";
+  if (layer) return sd_internal_tc_serves_layer(B, R, Hq, Hkv, D, capacity) ? "tcgen05" : "three kernels";
+  return sd_internal_tc_serves(B, R, Hq, Hkv, D, capacity) ? "tcgen05" : "mma.sync";
+}

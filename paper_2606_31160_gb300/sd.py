@@ -61,6 +61,7 @@ _SIGNATURES = {
     "sd_accept_sample": ([_vp, _vp, _i, _i, _i, _f, _vp, _vp, _vp, _vp, _vp, _sz, _vp], _i),
     "sd_get_device_error": ([_vp, ctypes.POINTER(ctypes.c_uint32)], _i),
     "sd_set_cluster_size": ([_i], _i),
+    "sd_verify_kernel": ([_i, _i, _i, _i, _i, _i, _i], ctypes.c_char_p),
     "sd_attention_budget": ([_vp, ctypes.POINTER(KVCacheStruct), _i, _i, _f, _vp, _vp, _vp, _vp], _i),
 }
 
@@ -370,6 +371,12 @@ def accept_sample(z_target, z_draft, draft, u, temperature, ws=None, n_emit=None
 def set_cluster_size(cluster_size=0):
     """Force the tcgen05 attention cluster size (1, 2, 4, 6, 8, 16); 0 = automatic."""
     _check(lib().sd_set_cluster_size(int(cluster_size)), "sd_set_cluster_size")
+
+
+def verify_kernel(B, R, Hq, Hkv, D, capacity, layer=False):
+    """Name of the kernel that serves this shape on the current device
+    (sd_verify_kernel): "small-tile", "tcgen05", "mma.sync" or "three kernels"."""
+    return lib().sd_verify_kernel(B, R, Hq, Hkv, D, capacity, 1 if layer else 0).decode()
 
 
 def get_device_error():

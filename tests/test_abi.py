@@ -106,3 +106,13 @@ def test_unknown_mask_flags_are_rejected_before_launch(lib):
     assert lib.sd_verify_layer(ctypes.c_void_p(16), ctypes.c_void_p(16), ctypes.c_void_p(16), ctypes.c_void_p(16),
                                (ctypes.c_int32 * 3)(16, 24, 24), 0, 1e6, ctypes.byref(cache), ctypes.c_void_p(16),
                                8, 32, 0.0, null, 0, 4, null) == 1
+
+
+def test_kernel_query_rejects_unsupported_shapes(lib):
+    # sd_verify_kernel is host arithmetic: shapes no entry point takes are
+    # "unsupported" without touching a device
+    from paper_2606_31160_gb300 import sd
+    assert sd.verify_kernel(1, 8, 30, 8, 128, 4104) == "unsupported"     # Hq % Hkv
+    assert sd.verify_kernel(1, 8, 32, 8, 96, 4104) == "unsupported"      # head_dim
+    assert sd.verify_kernel(1, 40, 32, 8, 128, 4104) == "unsupported"    # G * R > 128
+    assert sd.verify_kernel(0, 8, 32, 8, 128, 4104, True) == "unsupported"

@@ -190,3 +190,20 @@ def test_layer_small_tiles_overflow_sets_error_and_leaves_scene():
     assert cache.len.item() == case.cap
     assert torch.all(out == 5.0)
     assert bool(((cache.k == k0) | (cache.k.isnan() & k0.isnan())).all())
+
+
+def test_small_tiles_are_served_by_the_small_tile_kernel():
+    # the shapes above must reach the small-tile kernel itself (a shape it
+    # silently declined would still pass through the tcgen05 kernel)
+    for B, Hq, Hkv, K, prefix in SHAPES:
+        cap = max(prefix) + K + 9
+        assert sd.verify_kernel(B, K + 1, Hq, Hkv, 128, cap) == "small-tile"
+        assert sd.lib().sd_verify_kernel(B, K + 1, Hq, Hkv, 128, cap, 2) == b"small-tile"   # block mask
+        # the fused layer: from 8 (scene, KV head) clusters on; one scene of
+        # the draft's 4 KV heads stays on the tcgen05 layer kernel
+        want = "small-tile" if B * Hkv >= 8 else "tcgen05"
+        assert sd.verify_kernel(B, K + 1, Hq, Hkv, 128, cap, True) == want
+    assert sd.verify_kernel(1, 8, 32, 8, 128, 4104) == "tcgen05"        # 32 rows
+    assert sd.verify_kernel(1, 8, 32, 8, 128, 4104, True) == "tcgen05"
+    assert sd.verify_kernel(1, 5, 4, 1, 64, 300) == "mma.sync"          # head_dim 64
+    assert sd.verify_kernel(1, 5, 4, 1, 64, 300, True) == "three kernels"
