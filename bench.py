@@ -702,6 +702,14 @@ def main():
         sd.kv_append(st.caches[l], st.k[l], st.v[l])
     ms_attn_launch = time_graph(g_attn, reps) / LAYERS
     ms_attn_plain = time_graph(g_attn_plain, reps) / LAYERS
+    # the attention-budget diagnostic (Table tab:attn-budget) on the same 36
+    # appended caches: visual keys = the 4 cameras' 896 patches each
+    nvis = torch.full((1,), 4 * 896, dtype=torch.int32, device=device)
+    mass = torch.empty((1, R, HQ, 3), dtype=torch.float32, device=device)
+    ent = torch.empty((1, R, HQ), dtype=torch.float32, device=device)
+    g_budget = capture(lambda: [sd.attention_budget(st.q[l], st.caches[l], nvis, mass=mass, entropy=ent)
+                                for l in range(LAYERS)])
+    ms_budget = time_graph(g_budget, reps) / LAYERS
     st.lens.copy_(st.lens0)
     torch.cuda.synchronize()
     # ---- the small kernels of the path, per call: M-RoPE of one layer's rows,
@@ -785,6 +793,7 @@ def main():
         "layer_us": round(ms_layer_launch * 1e3, 3),
         "attention_us": round(ms_attn_launch * 1e3, 3),
         "attention_us_no_early_prefix": round(ms_attn_plain * 1e3, 3),
+        "budget_us": round(ms_budget * 1e3, 3),
         "unfused_verify_step_us": round(ms_unfused * 1e3, 3),
         "rope_us": round(ms_rope * 1e3, 3),
         "kv_append_us": round(ms_append * 1e3, 3),

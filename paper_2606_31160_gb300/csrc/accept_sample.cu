@@ -21,7 +21,9 @@
 //           when the rows are aligned); each CTA writes the chunk sums of the
 //           residual weights and of the target weights; the last CTA of a
 //           scene finds the chunk where the running sum passes u_K * S and
-//           re-scans the same per-thread runs inside it.
+//           re-scans the same per-thread runs inside it. A programmatic
+//           dependent launch: its CTAs are resident once every statistics CTA
+//           runs, and wait for the statistics to complete before they read.
 // All reductions run in a fixed order (deterministic), the weight formula
 // uses non-contractible intrinsics so both passes of the draw evaluate
 // identical values, and every spin-free ticket is re-armed after use.
@@ -87,32 +89,47 @@ __device__ __noinline__ void accept_tail(const float* __restrict__ zt, const flo
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int kT = nthreads;
   __shared__ float row_m[2 * 128 + 1], row_s[2 * 128 + 1];
-  for (int r = warp; r < rows; r += kT / 32) {
-    float rm = -INFINITY, rs = 0.f;
-    const float2* pr = part + (static_cast<long long>(b) * rows + r) * n_chunks;
-    for (int k = lane; k < n_chunks; k += 32) {
-      const float2 e = __ldcg(pr + k);
-      merge_ms(rm, rs, e.x, e.y, c2);
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      const float m2 = __shfl_xor_sync(0xffffffffu, rm, o);
-      const float s2 = __shfl_xor_sync(0xffffffffu, rs, o);
-      merge_ms(rm, rs, m2, s2, c2);
-    }
-    if (lane == 0) {
-      row_m[r] = rm;
-      row_s[r] = rs;
-    }
-  }
-  __syncthreads();
-  // the K draft tokens' two logits, recorded by the CTAs holding them
-  __shared__ float s_zt[128], s_zd[128];
+  // every load of the tail is issued before any result is used (one memory
+  // round trip): the K draft tokens' two logits, recorded by the CTAs holding
+  // them, the scene's K acceptance uniforms, and the rows' chunk partials,
+  // two rows a warp at a time
+  __shared__ float s_zt[128], s_zd[128], s_u[128];
   for (int j = threadIdx.x; j < K; j += kT) {
     const int x = s_x[j];
     const bool ok = x >= 0 && x < V;
     s_zt[j] = ok ? __ldcg(dlogit + static_cast<long long>(b) * rows + j) : 0.f;
     s_zd[j] = ok ? __ldcg(dlogit + static_cast<long long>(b) * rows + K + 1 + j) : 0.f;
+    s_u[j] = u[static_cast<long long>(b) * (K + 1) + j];
+  }
+  const int nw = kT / 32;
+  for (int r0 = warp; r0 < rows; r0 += 2 * nw) {
+    const int r1 = r0 + nw;
+    float rm[2] = {-INFINITY, -INFINITY}, rs[2] = {0.f, 0.f};
+    const float2* p0 = part + (static_cast<long long>(b) * rows + r0) * n_chunks;
+    const float2* p1 = part + (static_cast<long long>(b) * rows + (r1 < rows ? r1 : r0)) * n_chunks;
+    for (int k = lane; k < n_chunks; k += 32) {
+      const float2 e0 = __ldcg(p0 + k);
+      const float2 e1 = __ldcg(p1 + k);
+      merge_ms(rm[0], rs[0], e0.x, e0.y, c2);
+      merge_ms(rm[1], rs[1], e1.x, e1.y, c2);
+    }
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        const float m2 = __shfl_xor_sync(0xffffffffu, rm[h], o);
+        const float s2 = __shfl_xor_sync(0xffffffffu, rs[h], o);
+        merge_ms(rm[h], rs[h], m2, s2, c2);
+      }
+    }
+    if (lane == 0) {
+      row_m[r0] = rm[0];
+      row_s[r0] = rs[0];
+      if (r1 < rows) {
+        row_m[r1] = rm[1];
+        row_s[r1] = rs[1];
+      }
+    }
   }
   __syncthreads();
   if (threadIdx.x == 0) {
@@ -127,7 +144,7 @@ __device__ __noinline__ void accept_tail(const float* __restrict__ zt, const flo
       }
       const float p = __fdiv_rn(wexp(s_zt[j], row_m[j], c2), row_s[j]);
       const float q = __fdiv_rn(wexp(s_zd[j], row_m[K + 1 + j], c2), row_s[K + 1 + j]);
-      if (!(__fmul_rn(u[static_cast<long long>(b) * (K + 1) + j], q) <= p)) {
+      if (!(__fmul_rn(s_u[j], q) <= p)) {
         ell = j;
         break;
       }
@@ -163,6 +180,7 @@ __global__ void __launch_bounds__(kVec ? kVecThreads : kThreads)
                         DrawInfo* __restrict__ info) {
   constexpr int kT = kVec ? kVecThreads : kThreads;
   const int c = blockIdx.x, rr = blockIdx.y, b = blockIdx.z;
+  if (threadIdx.x == 0) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const int rows = 2 * K + 1;
   const float* row = row_ptr(zt, zd, b, rr, K, V);
   const int lo = c * chunk, hi = min(V, lo + chunk);
@@ -274,6 +292,7 @@ __global__ void __launch_bounds__(kStreamThreads)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const float* row = row_ptr(zt, zd, b, rr, K, V);
   const int lo = c * seg, hi = min(V, lo + seg);
+  if (threadIdx.x == 0) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const int n_st = hi > lo ? (hi - lo + kStageFloats - 1) / kStageFloats : 0;
   if (threadIdx.x == 0) {
     for (int i = 0; i < kStreamStages; ++i) {
@@ -443,6 +462,9 @@ __global__ void __launch_bounds__(kThreads)
                        int32_t* __restrict__ tokens, const DrawInfo* __restrict__ info,
                        float2* __restrict__ sums, uint32_t* __restrict__ ticket) {
   const int c = blockIdx.x, b = blockIdx.y;
+  // a programmatic dependent launch: resident while the statistics finish,
+  // reading nothing they write before they have completed
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   const DrawInfo di = info[b];
   const float* rt = zt + (static_cast<long long>(b) * (K + 1) + di.ell) * V;
   const float* rd = di.ell < K ? zd + (static_cast<long long>(b) * K + di.ell) * V : nullptr;
@@ -727,8 +749,22 @@ extern "C" sd_status sd_accept_sample(const float* z_target, const float* z_draf
     sample_stats_kernel<false><<<dim3(p.n1, 2 * K + 1, B), kThreads, 0, st>>>(
         z_target, z_draft, K, V, c2, p.chunk1, p.n1, draft, u, n_emit, tokens, part, dlogit, ticket1, info);
   SD_CHECK_LAUNCH();
-  sample_draw_kernel<<<dim3(p.n2, B), kThreads, 0, st>>>(z_target, z_draft, K, V, c2, p.n2, p.vec, u, tokens,
-                                                          info, sums, ticket2);
-  SD_CHECK_LAUNCH();
+  // the draw is a programmatic dependent launch (it waits for the
+  // statistics before its first read of their results)
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.gridDim = dim3(p.n2, B, 1);
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.stream = st;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  const bool vec = p.vec;
+  if (cudaLaunchKernelEx(&cfg, sample_draw_kernel, z_target, z_draft, K, V, c2, p.n2, vec, u, static_cast<int32_t*>(tokens),
+                         static_cast<const DrawInfo*>(info), sums, ticket2) != cudaSuccess) {
+    (void)cudaGetLastError();
+    return SD_ERR_CUDA;
+  }
   return SD_OK;
 }

@@ -129,8 +129,10 @@ __device__ __forceinline__ void mma_bf16(float (&c)[4], const uint32_t (&a)[4], 
 constexpr int kTiles = 2;
 constexpr int kPassRows = 16 * kTiles;
 
+// two CTAs an SM (at most 128 registers a thread), so that clusters of 16
+// need only 8 SMs of a GPC and every cluster of a launch fits in one wave
 template <int D>
-__global__ void __launch_bounds__(kThreads)
+__global__ void __launch_bounds__(kThreads, 2)
     budget_kernel(const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* __restrict__ kc,
                   const int32_t* __restrict__ len, const int32_t* __restrict__ n_visual, int R, int Hq,
                   int Hkv, int cap, float scale, float* __restrict__ mass, float* __restrict__ entropy) {
@@ -140,6 +142,10 @@ __global__ void __launch_bounds__(kThreads)
   const int kvh = blockIdx.y, b = blockIdx.z;
   const int S = gridDim.x;
   const uint32_t rank = cta_rank();
+  // a programmatic dependent launch: resident while the kernel before it
+  // runs, reading nothing before it has completed
+  if (threadIdx.x == 0) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int gq = lane >> 2, tq = lane & 3;
   const int G = Hq / Hkv, M = G * R;
@@ -239,19 +245,26 @@ __global__ void __launch_bounds__(kThreads)
     cluster_sync_all();  // every CTA's part is written
     const int nr = min(kPassRows, M - m0);
     if (rank == 0) {
-      // one thread a (row, CTA): the S partial states travel at once
-      for (int idx = threadIdx.x; idx < nr * S; idx += kThreads) {
+      // one lane a (row, CTA): the S partial states travel at once and merge
+      // over the row's S lanes (S a power of two, so a row's lanes are an
+      // aligned group of one warp) in a fixed butterfly
+      for (int base0 = 0; base0 < kPassRows * S; base0 += kThreads) {  // block-uniform
+        const int idx = base0 + threadIdx.x;
         const int r = idx / S, cc = idx % S;
-        float v[8];
-        ld_cluster8(&part[r][0], cc, v);
-        gath[r][cc] = RowState{v[0], v[1], v[2], v[3], v[4]};
+        RowState a = row_empty();
+        if (r < nr) {
+          float v[8];
+          ld_cluster8(&part[r][0], cc, v);
+          a = RowState{v[0], v[1], v[2], v[3], v[4]};
+        }
+        for (int o = 1; o < S; o <<= 1) row_merge(a, row_shfl(a, o));
+        if (cc == 0 && r < kPassRows) gath[r][0] = a;
       }
       __syncthreads();
     }
     if (rank == 0 && threadIdx.x < nr && ok) {
       const int p = m0 + threadIdx.x, i = p / G, h = kvh * G + (p - i * G);
-      RowState a = row_empty();
-      for (int cc = 0; cc < S; ++cc) row_merge(a, gath[threadIdx.x][cc]);
+      const RowState a = gath[threadIdx.x][0];
       const float tot = a.v + a.t + a.g;
       const long long o = (static_cast<long long>(b) * R + i) * Hq + h;
       mass[o * 3 + 0] = a.v / tot;
@@ -288,16 +301,18 @@ extern "C" sd_status sd_attention_budget(const void* q, const sd_kv_cache* cache
   const auto* qq = static_cast<const __nv_bfloat16*>(q);
   const auto* kk = static_cast<const __nv_bfloat16*>(cache->k);
   cudaLaunchConfig_t cfg = {};
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = S;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.gridDim = dim3(S, Hkv, B);
   cfg.blockDim = dim3(kThreads, 1, 1);
   cfg.stream = st;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   cudaError_t e;
   // clusters of 16 are non-portable: allowed once per device and kernel
   static bool allowed[64][2];
