@@ -622,7 +622,7 @@ def main():
     ap.add_argument("--floor", action="store_true",
                     help="measure the platform floors of the chained layers (empty dependent launches, "
                          "TMA streams of one layer's bytes) and print one JSON line per point; no bench line")
-    ap.add_argument("--only", choices=["attention", "layer", "accept", "step", "sample"], default=None,
+    ap.add_argument("--only", choices=["attention", "layer", "accept", "step", "sample", "tiny"], default=None,
                     help="profiling mode: run one kernel family eagerly `steps` times on the "
                          "target-layer workload (sample: the stochastic-acceptance workload) "
                          "for ncu captures; prints no bench line")
@@ -974,6 +974,23 @@ def profile_only(args):
         ws = sd.workspace(sd.sample_workspace_bytes(w["B"], w["K"], w["V"]), dev)
         for _ in range(args.steps):
             sd.accept_sample(zt, zd, dr, u, w["temperature"], ws=ws)
+        torch.cuda.synchronize()
+        print(json.dumps({"profile_only": args.only, "launches": args.steps,
+                          "device_error": sd.get_device_error()}))
+        return
+    if args.only == "tiny":
+        # the tiny verify step (4 q / 1 KV x 64, L = 256, K = 4): M-RoPE, append
+        # and the mma.sync attention kernel (head_dim 64), accept, rollback
+        dev = torch.device("cuda", 0)
+        case = workloads.tiny()
+        q, k, v, pos = (x.to(dev) for x in (case.q, case.k_new, case.v_new, case.pos))
+        lens = torch.from_numpy(case.prefix.astype(np.int32)).to(dev)
+        cache = sd.KVCache(case.k_cache.to(dev), case.v_cache.to(dev), lens)
+        logits, draft = case.extra["logits"].to(dev), case.extra["draft"].to(dev)
+        for _ in range(args.steps):
+            lens.copy_(torch.from_numpy(case.prefix.astype(np.int32)).to(dev))
+            sd.verify_layer(q, k, v, pos, case.sections, cache, case.interleaved, case.base)
+            n_emit, tokens, _ = sd.accept_greedy(logits, draft)
         torch.cuda.synchronize()
         print(json.dumps({"profile_only": args.only, "launches": args.steps,
                           "device_error": sd.get_device_error()}))
