@@ -303,17 +303,16 @@ __global__ void __launch_bounds__(kStreamThreads)
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     s_timeout = 0;
   }
-  for (int j = threadIdx.x; j < K; j += kStreamThreads) s_x[j] = __ldg(draft + static_cast<long long>(b) * K + j);
   __syncthreads();
+  // the drafts (for the scene's last CTA; read after the barriers below), by
+  // the consumers: the producer's first copies do not wait for them
+  if (warp < kStreamConsumers / 32)
+    for (int j = threadIdx.x; j < K; j += kStreamConsumers) s_x[j] = __ldg(draft + static_cast<long long>(b) * K + j);
   float m = -INFINITY, s = 0.f;
   if (warp == kStreamConsumers / 32) {
-    // ---- producer: thread 0 of warp 8; also records the draft token's logit
+    // ---- producer: thread 0 of warp 8; the first copies go out before it
+    //      records the draft token's logit (a load it then waits for)
     if (lane == 0) {
-      if (rr != K) {
-        const int j = rr < K ? rr : rr - K - 1;
-        const int x = s_x[j];
-        if (x >= lo && x < hi) dlogit[static_cast<long long>(b) * rows + rr] = __ldg(row + x);
-      }
       for (int t = 0; t < n_st; ++t) {
         const int st = t % kStreamStages;
         if (t >= kStreamStages &&
@@ -330,6 +329,11 @@ __global__ void __launch_bounds__(kStreamThreads)
                          static_cast<uint32_t>(__cvta_generic_to_shared(&stage[st][0]))),
                      "l"(row + p0), "r"(bytes), "r"(fb)
                      : "memory");
+      }
+      if (rr != K) {
+        const int j = rr < K ? rr : rr - K - 1;
+        const int x = __ldg(draft + static_cast<long long>(b) * K + j);
+        if (x >= lo && x < hi) dlogit[static_cast<long long>(b) * rows + rr] = __ldg(row + x);
       }
     }
   } else {
