@@ -132,36 +132,49 @@ __device__ __noinline__ void accept_tail(const float* __restrict__ zt, const flo
     }
   }
   __syncthreads();
-  if (threadIdx.x == 0) {
+  if (warp == 0) {
+    // the K acceptance tests side by side (lane j of a 32-draft group), the
+    // first stop by ballot: l = the first j whose token is out of range or
+    // whose test fails, as a sequential scan would find it
     int ell = K;
-    bool range_ok = true;
-    for (int j = 0; j < K; ++j) {
-      const int x = s_x[j];
-      if (x < 0 || x >= V) {
-        range_ok = false;
-        ell = j;
-        break;
+    bool range_bad = false;
+    for (int j0 = 0; j0 < K; j0 += 32) {  // warp-uniform
+      const int j = j0 + lane;
+      bool stop = false, bad = false;
+      if (j < K) {
+        const int x = s_x[j];
+        bad = x < 0 || x >= V;
+        if (bad) {
+          stop = true;
+        } else {
+          const float p = __fdiv_rn(wexp(s_zt[j], row_m[j], c2), row_s[j]);
+          const float q = __fdiv_rn(wexp(s_zd[j], row_m[K + 1 + j], c2), row_s[K + 1 + j]);
+          stop = !(__fmul_rn(s_u[j], q) <= p);
+        }
       }
-      const float p = __fdiv_rn(wexp(s_zt[j], row_m[j], c2), row_s[j]);
-      const float q = __fdiv_rn(wexp(s_zd[j], row_m[K + 1 + j], c2), row_s[K + 1 + j]);
-      if (!(__fmul_rn(s_u[j], q) <= p)) {
-        ell = j;
+      const unsigned hit = __ballot_sync(0xffffffffu, stop);
+      if (hit) {
+        const int first = __ffs(hit) - 1;
+        ell = j0 + first;
+        range_bad = __shfl_sync(0xffffffffu, bad, first);
         break;
       }
     }
-    if (!range_ok) sd_set_error(SD_DEVERR_TOKEN_RANGE);
-    DrawInfo di;
-    di.ell = ell;
-    di.mt = row_m[ell];
-    di.inv_zt = __fdiv_rn(1.f, row_s[ell]);
-    di.md = ell < K ? row_m[K + 1 + ell] : 0.f;
-    di.inv_zd = ell < K ? __fdiv_rn(1.f, row_s[K + 1 + ell]) : 0.f;
-    di.pad[0] = di.pad[1] = di.pad[2] = 0.f;
-    info[b] = di;
+    if (lane == 0) {
+      if (range_bad) sd_set_error(SD_DEVERR_TOKEN_RANGE);
+      DrawInfo di;
+      di.ell = ell;
+      di.mt = row_m[ell];
+      di.inv_zt = __fdiv_rn(1.f, row_s[ell]);
+      di.md = ell < K ? row_m[K + 1 + ell] : 0.f;
+      di.inv_zd = ell < K ? __fdiv_rn(1.f, row_s[K + 1 + ell]) : 0.f;
+      di.pad[0] = di.pad[1] = di.pad[2] = 0.f;
+      info[b] = di;
+      n_emit[b] = ell + 1;
+      ticket[b] = 0;
+    }
     int32_t* tk = tokens + static_cast<long long>(b) * (K + 1);
-    for (int j = 0; j <= K; ++j) tk[j] = j < ell ? s_x[j] : -1;
-    n_emit[b] = ell + 1;
-    ticket[b] = 0;
+    for (int j = lane; j <= K; j += 32) tk[j] = j < ell ? s_x[j] : -1;
   }
 }
 
