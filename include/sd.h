@@ -161,12 +161,8 @@ size_t sd_verify_attention_workspace(int B, int R, int Hq, int Hkv, int D, int c
  * SD_DEVERR_LENGTH and its output is left unwritten. The first call per
  * device and shape should come before any stream capture (it sets kernel
  * attributes and queries the occupancy).
- * Kernel choice is by shape: head_dim 128 with G*R <= 16 (single-row decode
- * steps and short verify blocks) takes the small-tile kernel (one thread-block
- * cluster of up to 16 CTAs per KV head over every SM, mma.sync tiles of 16
- * packed rows, partial states merged in distributed shared memory; no
- * workspace), head_dim 128 with 16 < G*R <= 128 the tcgen05 kernel, every
- * other shape the mma.sync kernel. A test-only override exists:
+ * Kernel choice is by shape: head_dim 128 with G*R <= 128 takes the tcgen05
+ * kernel, every other shape the mma.sync kernel (sd_verify_kernel names it). A test-only override exists:
  * the environment variable SD_ATTENTION_KERNEL=mma, read once per process,
  * sends every shape to the mma.sync kernel so that tests can compare the two
  * kernels on the same inputs; production callers leave it unset.
@@ -199,8 +195,8 @@ sd_status sd_verify_attention_ex(const void* q, const sd_kv_cache* cache, void* 
                                  size_t ws_bytes, sd_stream_t stream);
 
 /*
- * Cluster size of the tcgen05 and small-tile verify-attention kernels
- * (sd_verify_attention and sd_verify_layer, head_dim 128, G*R <= 128): one
+ * Cluster size of the tcgen05 verify-attention kernels and the small-tile
+ * layer kernel (sd_verify_attention and sd_verify_layer, head_dim 128): one
  * thread-block cluster of `cluster_size` CTAs per (scene, KV head) splits that
  * head's keys evenly and merges the partial softmax states in distributed
  * shared memory (the split-L form of Eq. verify). 0 (the default) lets every
@@ -283,11 +279,13 @@ size_t sd_verify_layer_workspace(int B, int R, int Hq, int Hkv, int D, int capac
  *   k_new and v_new are read only after the predecessor has completed.
  *   SD_LAYER_BLOCK_MASK: the attention uses the block mask (as
  *   SD_ATTN_BLOCK_MASK of sd_verify_attention_ex).
- * For head_dim 128 this is one kernel: the small-tile kernel for G * R <= 16
- * when the layer is block-masked or B * Hkv >= 8, the tcgen05 kernel for the
- * other shapes with G * R <= 128 and R <= 31 (R <= 16 when G * R <= 32; the
- * block mask only when G * R > 32); other shapes run the three kernels in
- * sequence (sd_verify_kernel names the choice). A scene whose append would pass the
+ * For head_dim 128 this is one kernel: the tcgen05 kernel for G * R <= 128
+ * and R <= 31 (R <= 16 when G * R <= 32), except that its 32-row tile is
+ * causal only, so block-masked layers with G * R <= 16 take the small-tile
+ * kernel (one thread-block cluster of up to 16 CTAs per KV head, mma.sync
+ * tiles of 16 packed rows) and those with 16 < G * R <= 32 the three kernels;
+ * other shapes run the three kernels in sequence (sd_verify_kernel names the
+ * choice). A scene whose append would pass the
  * capacity sets SD_DEVERR_KV_OVERFLOW and is left untouched.
  */
 sd_status sd_verify_layer(void* q, void* k_new, const void* v_new, const int32_t* pos,

@@ -782,7 +782,6 @@ static sd_status check_shape(int B, int R, int Hq, int Hkv, int D, int cap) {
 
 extern "C" size_t sd_verify_attention_workspace(int B, int R, int Hq, int Hkv, int D, int capacity) {
   if (check_shape(B, R, Hq, Hkv, D, capacity) != SD_OK || B == 0) return 0;
-  if (sd_internal_decode_serves(B, R, Hq, Hkv, D, capacity, false)) return 0;
   if (sd_internal_tc_serves(B, R, Hq, Hkv, D, capacity)) return 0;
   Plan p;
   if (!make_plan(B, R, Hq, Hkv, D, capacity, &p)) return 0;
@@ -814,9 +813,7 @@ extern "C" sd_status sd_verify_attention_ex(const void* q, const sd_kv_cache* ca
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   {
     bool handled = false;
-    sd_status s = sd_internal_verify_attention_dec(q, cache, out, R, Hq, scale_log2, flags, st, &handled);
-    if (handled) return s;
-    s = sd_internal_verify_attention_tc(q, cache, out, R, Hq, scale_log2, flags, st, &handled);
+    const sd_status s = sd_internal_verify_attention_tc(q, cache, out, R, Hq, scale_log2, flags, st, &handled);
     if (handled) return s;
   }
   Plan p;

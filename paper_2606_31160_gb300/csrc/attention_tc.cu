@@ -1551,9 +1551,10 @@ bool sd_internal_tc_serves(int B, int R, int Hq, int Hkv, int D, int cap) {
   return tc_plan(B, R, Hq, Hkv, D, cap).cs > 0;
 }
 
-bool sd_internal_tc_serves_layer(int B, int R, int Hq, int Hkv, int D, int cap) {
+bool sd_internal_tc_serves_layer(int B, int R, int Hq, int Hkv, int D, int cap, bool block) {
   if (R > 32) return false;
   const TcPlan plan = tc_plan(B, R, Hq, Hkv, D, cap, 32 - R);
+  if (block && plan.rows == 32) return false;  // the 32-row fused kernel is causal only
   return plan.cs > 0 && R <= (plan.rows == 32 ? Cfg<32>::kMaxNew : Cfg<64>::kMaxNew);
 }
 

@@ -46,7 +46,7 @@ sd_status sd_internal_verify_attention_tc(const void* q, const sd_kv_cache* cach
 // Whether the tcgen05 path serves this shape on the current device: the
 // attention, and the fused layer without the block mask.
 bool sd_internal_tc_serves(int B, int R, int Hq, int Hkv, int D, int cap);
-bool sd_internal_tc_serves_layer(int B, int R, int Hq, int Hkv, int D, int cap);
+bool sd_internal_tc_serves_layer(int B, int R, int Hq, int Hkv, int D, int cap, bool block);
 
 struct RopeTable;
 // The fused verify layer on the tcgen05 path (attention_tc.cu); *handled is
@@ -59,13 +59,10 @@ sd_status sd_internal_verify_layer_tc(void* q, void* k_new, const void* v_new, c
 // Cluster size forced by sd_set_cluster_size (0: chosen per call).
 int sd_internal_forced_cluster();
 
-// The small-tile kernel (decode.cu): head_dim 128 and G * R <= 16 query rows
-// per KV head. Whether it serves a shape on the current device:
-bool sd_internal_decode_serves(int B, int R, int Hq, int Hkv, int D, int cap, bool layer, bool block = false);
-// Verify attention / the fused verify layer on it; *handled is set when the
-// shape is served and the kernel launched.
-sd_status sd_internal_verify_attention_dec(const void* q, const sd_kv_cache* cache, void* out, int R, int Hq,
-                                           float scale_log2, int flags, cudaStream_t stream, bool* handled);
+// The small-tile layer kernel (decode.cu): head_dim 128 and G * R <= 16 query
+// rows per KV head, block-masked layers. Whether it serves a shape on the
+// current device, and the layer on it (*handled is set when it launched):
+bool sd_internal_decode_serves(int B, int R, int Hq, int Hkv, int D, int cap, bool block);
 sd_status sd_internal_verify_layer_dec(void* q, void* k_new, const void* v_new, const int32_t* pos,
                                        const RopeTable& tab, const sd_kv_cache* cache, void* out, int R,
                                        int Hq, float scale_log2, uint32_t* ticket, int early, int block,

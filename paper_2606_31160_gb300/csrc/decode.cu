@@ -1,8 +1,11 @@
-// K3 for small packed row tiles: verify attention (Eq. verify, Sec. 3.2) and
-// the fused verify layer (M-RoPE of Sec. 3.3 / Sec. 4.2 + the KV append of
-// Eq. commit + the attention) when the G * R query rows that share a KV head
-// fit one 16-row tile, as in the draft's single-row decode steps (Eq.
-// propose: R = 1, G = 4) and short verify blocks.
+// The fused verify layer (M-RoPE of Sec. 3.3 / Sec. 4.2 + the KV append of
+// Eq. commit + the verify attention of Eq. verify, Sec. 3.2) on small packed
+// row tiles: the G * R query rows that share a KV head fit one 16-row tile,
+// as in the draft's single-row decode steps (Eq. propose: R = 1, G = 4) and
+// short verify blocks. The library sends it the block-masked short layers
+// (the tcgen05 layer kernel's 32-row tile is causal only); the causal ones
+// run faster on the tcgen05 kernel's 128-key tensor-memory products (see the
+// routing note at layer_preferred below).
 //
 // Such a tile carries too few rows to pay for a 128-key tensor-memory product
 // per key tile, and one (scene, KV head) holds too few keys to keep more than
@@ -250,14 +253,12 @@ __device__ __forceinline__ uint4 rotate_chunk(uint4 w, const float2* cs) {
 }
 
 // --------------------------------------------------------------------------
-// Kernel body. kLayer: the fused verify layer (len[b] is the prefix length,
-// the new rows come from q / k_new / v_new); otherwise attention over a cache
-// that already holds the R new rows (len[b] counts them), q already rotated.
-// Grid: (cluster size, Hkv, B), one cluster per (scene, KV head).
+// Kernel body: len[b] is the prefix length, the new rows come from q /
+// k_new / v_new. Grid: (cluster size, Hkv, B), one cluster per (scene, KV
+// head).
 //
 // `issued`: prefix blocks the producer already issued before the dependency wait.
 // --------------------------------------------------------------------------
-template <bool kLayer>
 __device__ __forceinline__ void decode_body(const CUtensorMap* tm_k, const CUtensorMap* tm_v,
                                             const DecArgs& a, const RopeTable& tab, uint8_t* smem,
                                             int issued) {
@@ -293,7 +294,7 @@ __device__ __forceinline__ void decode_body(const CUtensorMap* tm_k, const CUten
   // entries, loaded whole (the axis is chosen once they are in)
   int pv[kMaxNew * 64 / kCT][3];
   if (warp < kCW) {
-    if (kLayer) {
+    {
 #pragma unroll
       for (int e = 0; e < kMaxNew * 64 / kCT; ++e) {
         const int idx = tid + kCT * e;
@@ -309,7 +310,7 @@ __device__ __forceinline__ void decode_body(const CUtensorMap* tm_k, const CUten
         qraw = *reinterpret_cast<const uint4*>(a.q + ((static_cast<long long>(b) * R + i) * a.Hq + h * G + gq) *
                                                          kD + my_c * 8);
       }
-      if (kLayer && last_rank && my_p < R) {
+      if (last_rank && my_p < R) {
         const long long row = (static_cast<long long>(b) * R + my_p) * a.Hkv + h;
         kraw = *reinterpret_cast<const uint4*>(a.k_new + row * kD + my_c * 8);
         vraw = *reinterpret_cast<const uint4*>(a.v_new + row * kD + my_c * 8);
@@ -319,19 +320,14 @@ __device__ __forceinline__ void decode_body(const CUtensorMap* tm_k, const CUten
 
   int L_b, n_keys;  // prefix length; keys the rows see at most
   bool valid;
-  if (kLayer) {
+  {
     L_b = len_in;
     n_keys = len_in + R;
     valid = len_in >= 0 && len_in + R <= a.cap;
     if (!valid && tid == 0 && rank == 0 && h == 0) sd_set_error(SD_DEVERR_KV_OVERFLOW);
-  } else {
-    L_b = len_in - R;
-    n_keys = len_in;
-    valid = len_in >= R && len_in <= a.cap;
-    if (!valid && tid == 0 && rank == 0 && h == 0) sd_set_error(SD_DEVERR_LENGTH);
   }
   if (!valid) return;  // the whole cluster agrees (same len[b]); nothing was written
-  if (kLayer && tid == 0) {
+  if (tid == 0) {
     // the last CTA of the scene to read len[b] advances it (after every read)
     const uint32_t n_ctas = static_cast<uint32_t>(a.Hkv) * static_cast<uint32_t>(C);
     if (atom_add_acq_rel(a.ticket + b, 1u) == n_ctas - 1) {
@@ -340,13 +336,13 @@ __device__ __forceinline__ void decode_body(const CUtensorMap* tm_k, const CUten
     }
   }
 
-  // ---- this CTA's run of 32-key blocks: the prefix (layer) or every key
-  const int loop_keys = kLayer ? L_b : n_keys;
+  // ---- this CTA's run of 32-key blocks of the prefix
+  const int loop_keys = L_b;
   const int nblk = (loop_keys + kBlk - 1) / kBlk;
   const int blk_begin = static_cast<int>((static_cast<long long>(rank) * nblk) / C);
   const int blk_end = static_cast<int>((static_cast<long long>(rank + 1) * nblk) / C);
   const int n_run = blk_end - blk_begin;
-  const bool has_new = kLayer && last_rank;
+  const bool has_new = last_rank;
   const int n_items = n_run + (has_new ? 1 : 0);  // the new-key block is the last item
 
   if (warp == kCW) {
@@ -368,7 +364,7 @@ __device__ __forceinline__ void decode_body(const CUtensorMap* tm_k, const CUten
     __syncwarp();
   } else {
     // ------------------------------------------------------------ consumers
-    if (kLayer) {
+    {
       // (cos, sin) of every (new row, pair): the rotation kernel's arithmetic
 #pragma unroll
       for (int e = 0; e < kMaxNew * 64 / kCT; ++e) {
@@ -381,8 +377,8 @@ __device__ __forceinline__ void decode_body(const CUtensorMap* tm_k, const CUten
       named_bar_sync(1, kCT);
     }
     // the packed query row chunk -> shared memory (swizzled like the K boxes),
-    // rotated in the layer; padding rows are zero
-    if (kLayer && my_p < M) qraw = rotate_chunk(qraw, cs_tab + (my_p / G) * 64 + my_c * 4);
+    // rotated; padding rows are zero
+    if (my_p < M) qraw = rotate_chunk(qraw, cs_tab + (my_p / G) * 64 + my_c * 4);
     asm volatile("st.shared.v4.u32 [%0], {%1,%2,%3,%4};" ::"r"(qs + (my_c >> 3) * kQHalf + swz(my_p, my_c & 7)),
                  "r"(qraw.x), "r"(qraw.y), "r"(qraw.z), "r"(qraw.w)
                  : "memory");
@@ -433,17 +429,12 @@ __device__ __forceinline__ void decode_body(const CUtensorMap* tm_k, const CUten
     for (int hh = 0; hh < 2; ++hh) {
       const int p = g8 + 8 * hh;
       const int i = p < M ? p / G : R - 1;
-      if (kLayer) {
-        lim[hh] = L_b - 1;
-        lim_new[hh] = a.block ? R - 1 : i;
-      } else {
-        lim[hh] = a.block ? n_keys - 1 : min(L_b + i, n_keys - 1);
-        lim_new[hh] = -1;
-      }
+      lim[hh] = L_b - 1;
+      lim_new[hh] = a.block ? R - 1 : i;
     }
     // smallest limit over the rows; last key read (values past it are zeroed)
-    const int mask_from = kLayer ? L_b - 1 : (a.block ? n_keys - 1 : L_b);
-    const int last_key = kLayer ? L_b - 1 : n_keys - 1;
+    const int mask_from = L_b - 1;
+    const int last_key = L_b - 1;
 
     float o[16][4];
 #pragma unroll
@@ -665,7 +656,7 @@ __device__ __forceinline__ void decode_body(const CUtensorMap* tm_k, const CUten
   if (warp < kCW) {
     // the layer's rotated query rows go back to q now that every rank has
     // read the raw ones (all ranks passed the cluster barrier above)
-    if (kLayer && rank == 0) {
+    if (rank == 0) {
       for (int idx = tid; idx < M * 16; idx += kCT) {
         const int p = idx >> 4, c = idx & 15;
         const int i = p / G, gq = p - i * G;
@@ -736,7 +727,6 @@ __device__ __forceinline__ void decode_body(const CUtensorMap* tm_k, const CUten
   cluster_wait();
 }
 
-template <bool kLayer>
 __global__ void __launch_bounds__(kThreads, 1)
     verify_decode_kernel(const __grid_constant__ CUtensorMap tm_k,
                          const __grid_constant__ CUtensorMap tm_v, const DecArgs a,
@@ -767,11 +757,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int C = static_cast<int>(gridDim.x), rank = static_cast<int>(cluster_rank());
     const int h = blockIdx.y, b = blockIdx.z;
     const int len_in = a.len[b];
-    const int L_b = kLayer ? len_in : len_in - a.R;
-    const int n_keys = kLayer ? len_in + a.R : len_in;
-    const bool valid = kLayer ? (len_in >= 0 && len_in + a.R <= a.cap) : (len_in >= a.R && len_in <= a.cap);
+    const int L_b = len_in;
+    const bool valid = len_in >= 0 && len_in + a.R <= a.cap;
     if (valid) {
-      const int nblk = ((kLayer ? L_b : n_keys) + kBlk - 1) / kBlk;
+      const int nblk = (L_b + kBlk - 1) / kBlk;
       const int blk_begin = static_cast<int>((static_cast<long long>(rank) * nblk) / C);
       const int blk_end = static_cast<int>((static_cast<long long>(rank + 1) * nblk) / C);
       issued = min(blk_end - blk_begin, kSlots);
@@ -788,7 +777,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   }
   if (!a.early) griddep_wait();
-  decode_body<kLayer>(&tm_k, &tm_v, a, tab, smem, issued);
+  decode_body(&tm_k, &tm_v, a, tab, smem, issued);
 }
 
 // --------------------------------------------------------------------------
@@ -834,12 +823,11 @@ constexpr int kNumSizes = 5;
 // Per device: attributes set, and how many clusters of each size fit at once.
 struct DevState {
   bool ok = false;
-  int active[2][kNumSizes] = {};  // [kLayer][size]
+  int active[kNumSizes] = {};  // co-resident clusters of each size
 };
 
-template <bool kLayer>
 bool setup_kernel(int* active) {
-  auto kern = verify_decode_kernel<kLayer>;
+  auto kern = verify_decode_kernel;
   if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes) != cudaSuccess ||
       cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess) {
     (void)cudaGetLastError();
@@ -879,7 +867,7 @@ DevState* state() {
   std::lock_guard<std::mutex> lock(mu);
   if (!done[dev]) {
     done[dev] = true;
-    st[dev].ok = setup_kernel<false>(st[dev].active[0]) && setup_kernel<true>(st[dev].active[1]);
+    st[dev].ok = setup_kernel(st[dev].active);
   }
   return &st[dev];
 }
@@ -888,17 +876,17 @@ DevState* state() {
 // and fits, else the largest size whose clusters for every (scene, KV head)
 // fit on the device in one wave and leave each CTA at least two 32-key blocks
 // of the capacity; 0 when the kernel does not serve.
-int pick_size(bool layer, int B, int Hkv, int cap) {
+int pick_size(int B, int Hkv, int cap) {
   DevState* s = state();
   if (!s || !s->ok) return 0;
   const long long units = static_cast<long long>(B) * Hkv;
   const long long nblk = (cap + kBlk - 1) / kBlk;
   const int forced = sd_internal_forced_cluster();
   for (int i = 0; i < kNumSizes && forced > 0; ++i)
-    if (kSizes[i] == forced && s->active[layer ? 1 : 0][i] > 0) return forced;
+    if (kSizes[i] == forced && s->active[i] > 0) return forced;
   for (int i = 0; i < kNumSizes; ++i) {
     const int cs = kSizes[i];
-    const int act = s->active[layer ? 1 : 0][i];
+    const int act = s->active[i];
     if (act <= 0) continue;
     if (cs > 1 && nblk < 2LL * cs) continue;
     if (units <= act || cs == 1) return cs;
@@ -906,23 +894,22 @@ int pick_size(bool layer, int B, int Hkv, int cap) {
   return 0;
 }
 
-// The fused layer takes this kernel for block-masked layers (the 32-row
-// tcgen05 layer kernel is causal only) and once the launch has at least 8
-// (scene, KV head) clusters; a single scene of the draft's 4 KV heads runs
-// faster on the tcgen05 layer kernel (8.2 against 9.0 us a step, measured),
-// whose 128-key tensor-memory products outrun 16-row mma.sync tiles there.
-bool layer_preferred(int B, int Hkv, int block) {
-  return block != 0 || static_cast<long long>(B) * Hkv >= 8;
-}
+// The library sends this kernel the block-masked layers only (the tcgen05
+// layer kernel's 32-row tile is causal only, so they would otherwise run as
+// three kernels). Causal layers and every attention call run faster on the
+// tcgen05 kernel, measured on one box: the draft step (one scene, 4 KV heads,
+// one row) 8.0 against 9.0 us, and every K = 1 / K = 2 point of the batched
+// sweep (e.g. B = 1, L = 8192: 0.38 against 0.31 of the measured copy; B = 8,
+// L = 2048: 0.59 against 0.56), where 128-key tensor-memory products outrun
+// 16-row mma.sync tiles (~1.7k cycles a 32-key block a warp).
+bool layer_preferred(int block) { return block != 0; }
 
 bool shape_served(int R, int Hq, int Hkv, int D) {
   if (D != kD || Hkv <= 0 || Hq % Hkv || R <= 0 || R > kMaxNew) return false;
   return (Hq / Hkv) * R <= kRows;
 }
 
-template <bool kLayer>
-sd_status launch(const sd_kv_cache* cache, const DecArgs& a, const RopeTable& tab, int cs,
-                 cudaStream_t stream) {
+sd_status launch(const sd_kv_cache* cache, const DecArgs& a, const RopeTable& tab, int cs, cudaStream_t stream) {
   const int B = cache->batch, Hkv = cache->n_kv_heads, cap = cache->capacity;
   CUtensorMap tk, tv;
   if (!make_map(&tk, cache->k, cap, B * Hkv) || !make_map(&tv, cache->v, cap, B * Hkv)) return SD_ERR_CUDA;
@@ -940,7 +927,7 @@ sd_status launch(const sd_kv_cache* cache, const DecArgs& a, const RopeTable& ta
   cfg.stream = stream;
   cfg.attrs = attr;
   cfg.numAttrs = 2;
-  if (cudaLaunchKernelEx(&cfg, verify_decode_kernel<kLayer>, tk, tv, a, tab) != cudaSuccess) {
+  if (cudaLaunchKernelEx(&cfg, verify_decode_kernel, tk, tv, a, tab) != cudaSuccess) {
     (void)cudaGetLastError();
     return SD_ERR_CUDA;
   }
@@ -949,35 +936,9 @@ sd_status launch(const sd_kv_cache* cache, const DecArgs& a, const RopeTable& ta
 
 }  // namespace
 
-bool sd_internal_decode_serves(int B, int R, int Hq, int Hkv, int D, int cap, bool layer, bool block) {
-  if (!shape_served(R, Hq, Hkv, D) || B <= 0 || B > 65535 || Hkv > 65535) return false;
-  if (layer && !layer_preferred(B, Hkv, block)) return false;
-  return pick_size(layer, B, Hkv, cap) > 0;
-}
-
-sd_status sd_internal_verify_attention_dec(const void* q, const sd_kv_cache* cache, void* out, int R, int Hq,
-                                           float scale_log2, int flags, cudaStream_t stream, bool* handled) {
-  *handled = false;
-  const int B = cache->batch, Hkv = cache->n_kv_heads;
-  if (!shape_served(R, Hq, Hkv, cache->head_dim) || B > 65535) return SD_OK;
-  const int cs = pick_size(false, B, Hkv, cache->capacity);
-  if (cs <= 0) return SD_OK;
-  DecArgs a = {};
-  a.q = static_cast<__nv_bfloat16*>(const_cast<void*>(q));
-  a.out = static_cast<__nv_bfloat16*>(out);
-  a.len = cache->len;
-  a.R = R;
-  a.Hq = Hq;
-  a.Hkv = Hkv;
-  a.G = Hq / Hkv;
-  a.M = a.G * R;
-  a.cap = cache->capacity;
-  a.early = (flags & SD_ATTN_PREFIX_EARLY) ? 1 : 0;
-  a.block = (flags & SD_ATTN_BLOCK_MASK) ? 1 : 0;
-  a.scale_log2 = scale_log2;
-  RopeTable tab = {};
-  *handled = true;
-  return launch<false>(cache, a, tab, cs, stream);
+bool sd_internal_decode_serves(int B, int R, int Hq, int Hkv, int D, int cap, bool block) {
+  if (!layer_preferred(block) || !shape_served(R, Hq, Hkv, D) || B <= 0 || B > 65535 || Hkv > 65535) return false;
+  return pick_size(B, Hkv, cap) > 0;
 }
 
 sd_status sd_internal_verify_layer_dec(void* q, void* k_new, const void* v_new, const int32_t* pos,
@@ -986,8 +947,8 @@ sd_status sd_internal_verify_layer_dec(void* q, void* k_new, const void* v_new, 
                                        cudaStream_t stream, bool* handled) {
   *handled = false;
   const int B = cache->batch, Hkv = cache->n_kv_heads;
-  if (!layer_preferred(B, Hkv, block) || !shape_served(R, Hq, Hkv, cache->head_dim) || B > 65535) return SD_OK;
-  const int cs = pick_size(true, B, Hkv, cache->capacity);
+  if (!layer_preferred(block) || !shape_served(R, Hq, Hkv, cache->head_dim) || B > 65535) return SD_OK;
+  const int cs = pick_size(B, Hkv, cache->capacity);
   if (cs <= 0) return SD_OK;
   DecArgs a = {};
   a.q = static_cast<__nv_bfloat16*>(q);
@@ -1009,5 +970,5 @@ sd_status sd_internal_verify_layer_dec(void* q, void* k_new, const void* v_new, 
   a.block = block ? 1 : 0;
   a.scale_log2 = scale_log2;
   *handled = true;
-  return launch<true>(cache, a, tab, cs, stream);
+  return launch(cache, a, tab, cs, stream);
 }

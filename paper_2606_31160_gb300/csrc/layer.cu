@@ -55,8 +55,9 @@ extern "C" sd_status sd_verify_layer(void* q, void* k_new, const void* v_new, co
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   auto* ticket = static_cast<uint32_t*>(workspace);
   bool handled = false;
-  // up to 16 packed rows per KV head (the draft's single-row steps): the
-  // small-tile kernel over every SM; larger tiles: the tcgen05 kernel
+  // block-masked layers of up to 16 packed rows per KV head: the small-tile
+  // kernel (the tcgen05 kernel's 32-row layer tile is causal only); the
+  // others: the tcgen05 kernel
   {
     const sd_status s = sd_internal_verify_layer_dec(q, k_new, v_new, pos, tab, cache, out, R, Hq, scale_log2,
                                                      ticket, flags & SD_LAYER_PREFIX_EARLY, block, st, &handled);
@@ -80,7 +81,7 @@ extern "C" const char* sd_verify_kernel(int B, int R, int Hq, int Hkv, int D, in
   if (B <= 0 || R <= 0 || Hq <= 0 || Hkv <= 0 || capacity <= 0 || Hq % Hkv || (D != 64 && D != 128) ||
       static_cast<long long>(Hq / Hkv) * R > 128)
     return "unsupported";
-  if (sd_internal_decode_serves(B, R, Hq, Hkv, D, capacity, layer != 0, layer > 1)) return "small-tile";
-  if (layer) return sd_internal_tc_serves_layer(B, R, Hq, Hkv, D, capacity) ? "tcgen05" : "three kernels";
+  if (layer != 0 && sd_internal_decode_serves(B, R, Hq, Hkv, D, capacity, layer > 1)) return "small-tile";
+  if (layer) return sd_internal_tc_serves_layer(B, R, Hq, Hkv, D, capacity, layer > 1) ? "tcgen05" : "three kernels";
   return sd_internal_tc_serves(B, R, Hq, Hkv, D, capacity) ? "tcgen05" : "mma.sync";
 }

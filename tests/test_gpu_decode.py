@@ -1,8 +1,10 @@
-"""The small-tile kernel (up to 16 packed query rows per KV head: the draft's
-single-row decode steps and short verify blocks) against the float64 oracle:
-verify attention and the fused verify layer, ragged scenes, stale NaN rows,
-every cluster size the launch picks, the block mask, chained dependent
-launches and the draft's decode loop on one cache."""
+"""The small-tile layer kernel: fused verify layers with the block mask of the
+block-diffusion drafts (every new row sees the prefix and all R new rows) and
+up to 16 packed query rows per KV head, against the float64 oracle and against
+the separate rotation, append and attention calls: ragged scenes, stale NaN
+rows, an empty prefix and prefixes shorter than one 32-key block, every
+cluster size the launch picks, interleaved M-RoPE, chained dependent launches,
+sequential steps on one cache, and the overflow error."""
 import numpy as np
 import pytest
 import torch
@@ -27,24 +29,17 @@ def _case(B, Hq, Hkv, K, prefix, layer, cap_pad=8, tail=float("nan"), sections=(
                                  layer=layer, tail_fill=tail)
 
 
-def _appended(case):
-    """Cache with the raw new rows appended on the host (attention-only tests:
-    rotation is not under test, so q and the new keys are used as drawn)."""
-    k, v = case.k_cache.clone(), case.v_cache.clone()
-    for b, p in enumerate(case.prefix):
-        k[b, :, p:p + case.R] = case.k_new[b].transpose(0, 1)
-        v[b, :, p:p + case.R] = case.v_new[b].transpose(0, 1)
-    lens = torch.from_numpy((case.prefix + case.R).astype(np.int32)).cuda()
-    return sd.KVCache(k.cuda(), v.cuda(), lens)
+def _oracle_block(q, cache):
+    return oracle.verify_attention(to64(q), to64(cache.k), to64(cache.v), cache.len.cpu().numpy(), block=True)
 
 
-def _oracle_attention(q, cache, block=False):
-    return oracle.verify_attention(to64(q), to64(cache.k), to64(cache.v), cache.len.cpu().numpy(), block=block)
+def _same(x, y):  # stale cache rows hold NaN on both sides
+    return bool(((x == y) | (x.isnan() & y.isnan())).all())
 
 
-# (B, Hq, Hkv, K, prefix): draft decode (G*R = 4), K = 1..3 of the 8B target
-# (8..16 rows), one KV head per query head with 16 rows, ragged scenes with an
-# empty prefix and prefixes shorter than one 32-key block
+# (B, Hq, Hkv, K, prefix): the draft's shape (G*R = 4), K = 1..3 of the 8B
+# target (8..16 rows), one KV head per query head with 16 rows, ragged scenes
+# with an empty prefix and prefixes shorter than one 32-key block
 SHAPES = [
     (1, 16, 4, 0, [4096]),
     (2, 32, 8, 1, [4096, 3001]),
@@ -54,71 +49,60 @@ SHAPES = [
 ]
 
 
-@pytest.mark.parametrize("B,Hq,Hkv,K,prefix", SHAPES)
-def test_attention_small_tiles_match_oracle(B, Hq, Hkv, K, prefix):
-    case = _case(B, Hq, Hkv, K, prefix, layer=700 + K)
-    cache = _appended(case)
-    q = case.q.cuda()
-    out = sd.verify_attention(q, cache)
-    ref = _oracle_attention(q, cache)
-    assert np.isfinite(to64(out)).all() and attn_within(to64(out), ref), np.abs(to64(out) - ref).max()
-    assert sd.get_device_error() == 0
-
-
-@pytest.mark.parametrize("B,Hq,Hkv,K,prefix", SHAPES[1:4])
-def test_attention_small_tiles_block_mask(B, Hq, Hkv, K, prefix):
-    case = _case(B, Hq, Hkv, K, prefix, layer=720 + K)
-    cache = _appended(case)
-    q = case.q.cuda()
-    out = sd.verify_attention(q, cache, block=True)
-    ref = _oracle_attention(q, cache, block=True)
-    assert attn_within(to64(out), ref), np.abs(to64(out) - ref).max()
-    assert sd.get_device_error() == 0
-
-
-@pytest.mark.parametrize("B,Hkv", [(1, 4), (2, 8), (8, 4), (40, 8)])
-def test_attention_every_cluster_size(B, Hkv):
-    # the launch sizes its clusters from B * Hkv (16, 8, 4 ... 1 CTAs per head):
-    # each size merges the same states through distributed shared memory
-    prefix = [2048 - 13 * b for b in range(B)]
-    case = _case(B, 4 * Hkv, Hkv, 1, prefix, layer=740 + B, tail=0.0)
-    cache = _appended(case)
-    q = case.q.cuda()
-    out = sd.verify_attention(q, cache)
-    ref = _oracle_attention(q, cache)
-    assert attn_within(to64(out), ref), np.abs(to64(out) - ref).max()
-    assert sd.get_device_error() == 0
+def test_block_masked_short_layers_take_the_small_tile_kernel():
+    # block-masked layers of <= 16 packed rows take this kernel (the tcgen05
+    # layer kernel's 32-row tile is causal only); causal layers and attention
+    # calls of the same shapes take the tcgen05 kernel
+    for B, Hq, Hkv, K, prefix in SHAPES:
+        cap = max(prefix) + K + 9
+        assert sd.lib().sd_verify_kernel(B, K + 1, Hq, Hkv, 128, cap, 2) == b"small-tile"
+        assert sd.verify_kernel(B, K + 1, Hq, Hkv, 128, cap, True) == "tcgen05"
+        assert sd.verify_kernel(B, K + 1, Hq, Hkv, 128, cap) == "tcgen05"
+    assert sd.lib().sd_verify_kernel(1, 8, 32, 8, 128, 4104, 2) == b"three kernels"   # 32 rows, causal tile
+    assert sd.lib().sd_verify_kernel(1, 17, 32, 8, 128, 4113, 2) == b"tcgen05"        # 68 rows: 64-row tile
+    assert sd.verify_kernel(1, 5, 4, 1, 64, 300, True) == "three kernels"              # head_dim 64
 
 
 @pytest.mark.parametrize("B,Hq,Hkv,K,prefix", SHAPES)
-def test_layer_small_tiles_match_oracle_and_separate_calls(B, Hq, Hkv, K, prefix):
+def test_block_masked_layer_matches_oracle_and_separate_calls(B, Hq, Hkv, K, prefix):
     case = _case(B, Hq, Hkv, K, prefix, layer=760 + K)
-    # separate calls: rotation kernel, append kernel, attention
+    # separate calls: rotation kernel, append kernel, block-masked attention
     qa, ka, va, pa, ca = gpu_case(case)
     sd.rope_apply(qa, ka, pa, case.sections, 0, case.base)
     sd.kv_append(ca, ka, va)
-    oa = sd.verify_attention(qa, ca)
+    oa = sd.verify_attention(qa, ca, block=True)
     # the fused layer
     qb, kb, vb, pb, cb = gpu_case(case)
-    ob = sd.verify_layer(qb, kb, vb, pb, case.sections, cb, 0, case.base)
+    ob = sd.verify_layer(qb, kb, vb, pb, case.sections, cb, 0, case.base, block=True)
     torch.cuda.synchronize()
-
-    def same(x, y):  # stale cache rows hold NaN on both sides
-        return bool(((x == y) | (x.isnan() & y.isnan())).all())
-
     assert torch.equal(qa, qb) and torch.equal(ka, kb)          # the rotation kernel's bits
-    assert same(ca.k, cb.k) and same(ca.v, cb.v) and torch.equal(ca.len, cb.len)
+    assert _same(ca.k, cb.k) and _same(ca.v, cb.v) and torch.equal(ca.len, cb.len)
     assert cb.len.cpu().tolist() == [p + K + 1 for p in prefix]
     pos = case.pos.numpy()[:, :, None, :]
     ref_q = oracle.mrope_apply(to64(case.q), pos, case.sections, 0, case.base)
     assert np.all(np.abs(to64(qb) - ref_q) <= rope_bound(ref_q, pair_magnitude(to64(case.q))))
-    ref_o = _oracle_attention(qb, cb)
+    ref_o = _oracle_block(qb, cb)
     assert np.isfinite(to64(ob)).all() and attn_within(to64(ob), ref_o), np.abs(to64(ob) - ref_o).max()
     assert (ob.float() - oa.float()).abs().max().item() <= 2 * ATTN_ATOL
     assert sd.get_device_error() == 0
 
 
-def test_layer_small_tiles_block_mask_and_interleaved():
+@pytest.mark.parametrize("B,Hkv,L", [(1, 4, 2048), (2, 8, 2048), (8, 4, 2048), (24, 4, 1000), (48, 4, 700)])
+def test_block_masked_layer_every_cluster_size(B, Hkv, L):
+    # the launch sizes its clusters from B * Hkv (16, 4, 4, 1 CTAs per head;
+    # the last case runs past one wave): each size merges the same states
+    # through distributed shared memory
+    prefix = [L - 13 * b for b in range(B)]
+    case = _case(B, 4 * Hkv, Hkv, 1, prefix, layer=740 + B, tail=0.0)
+    assert sd.lib().sd_verify_kernel(B, 2, 4 * Hkv, Hkv, 128, case.cap, 2) == b"small-tile"
+    q, k, v, p, cache = gpu_case(case)
+    out = sd.verify_layer(q, k, v, p, case.sections, cache, 0, case.base, block=True)
+    ref = _oracle_block(q, cache)
+    assert attn_within(to64(out), ref), np.abs(to64(out) - ref).max()
+    assert sd.get_device_error() == 0
+
+
+def test_block_masked_layer_interleaved_mrope():
     case = _case(2, 32, 8, 2, [900, 4096], layer=780)
     case.interleaved = 1
     rng = np.random.default_rng(781)
@@ -130,19 +114,19 @@ def test_layer_small_tiles_block_mask_and_interleaved():
     ref_k = oracle.mrope_apply(to64(case.k_new), pos, case.sections, 1, case.base)
     assert np.all(np.abs(to64(q) - ref_q) <= rope_bound(ref_q, pair_magnitude(to64(case.q))))
     assert np.all(np.abs(to64(k) - ref_k) <= rope_bound(ref_k, pair_magnitude(to64(case.k_new))))
-    ref_o = _oracle_attention(q, cache, block=True)
+    ref_o = _oracle_block(q, cache)
     assert attn_within(to64(out), ref_o), np.abs(to64(out) - ref_o).max()
     assert sd.get_device_error() == 0
 
 
-def test_layer_small_tiles_chained_early_prefix():
-    # back-to-back layers of a batched decode: every layer after the first
-    # streams its prefix before the previous layer ends; same bits as plain
-    cases = [_case(3, 16, 4, 0, [4096, 2500, 17], layer=800 + l) for l in range(5)]
+def test_block_masked_layers_chained_early_prefix():
+    # back-to-back block-masked layers: every layer after the first streams its
+    # prefix before the previous layer ends; same bits as plain launches
+    cases = [_case(3, 16, 4, 2, [4096, 2500, 17], layer=800 + l) for l in range(5)]
     runs = []
     for early in (False, True):
         state = [gpu_case(c) for c in cases]
-        outs = [sd.verify_layer(q, k, v, p, c.sections, cache, 0, c.base, early=early and l > 0)
+        outs = [sd.verify_layer(q, k, v, p, c.sections, cache, 0, c.base, early=early and l > 0, block=True)
                 for l, (c, (q, k, v, p, cache)) in enumerate(zip(cases, state))]
         torch.cuda.synchronize()
         runs.append((outs, state))
@@ -151,59 +135,47 @@ def test_layer_small_tiles_chained_early_prefix():
         assert torch.equal(oa[l], ob[l]) and torch.equal(sa[l][0], sb[l][0])
         assert torch.equal(sa[l][4].len, sb[l][4].len)
     q, _, _, _, cache = sb[3]
-    ref = _oracle_attention(q, cache)
-    assert attn_within(to64(ob[3]), ref)
+    assert attn_within(to64(ob[3]), _oracle_block(q, cache))
     assert sd.get_device_error() == 0
 
 
-def test_draft_decode_loop_on_one_cache():
-    # the draft's propose loop: single-row steps on one cache, each appending
-    # the row the next step attends to (plain launches: each step waits for
-    # the previous one), then the rollback
+def test_block_masked_steps_on_one_cache():
+    # sequential steps on one cache (plain launches: each step's append is
+    # the next step's prefix), three-row blocks of a 16 q / 4 KV head layer
     w = workloads.draft_flat()
-    L, steps = w["L"], w["steps"]
-    cache = sd.KVCache(w["k_cache"].cuda(), w["v_cache"].cuda(), torch.tensor([L], dtype=torch.int32).cuda())
-    qs = [w["q"][s].cuda() for s in range(steps)]
+    L = w["L"]
+    rng = np.random.default_rng(830)
+    steps, R = 2, 3
+    k0 = torch.zeros((1, 4, L + steps * R, 128), dtype=torch.bfloat16)
+    v0 = torch.zeros_like(k0)
+    k0[:, :, :L] = w["k_cache"][:, :, :L]
+    v0[:, :, :L] = w["v_cache"][:, :, :L]
+    cache = sd.KVCache(k0.cuda(), v0.cuda(), torch.tensor([L], dtype=torch.int32).cuda())
+    qs = [workloads.to_bf16(rng.standard_normal((1, R, 16, 128))).cuda() for _ in range(steps)]
+    ks = [workloads.to_bf16(rng.standard_normal((1, R, 4, 128))).cuda() for _ in range(steps)]
+    vs = [workloads.to_bf16(rng.standard_normal((1, R, 4, 128))).cuda() for _ in range(steps)]
     outs = []
     for s in range(steps):
-        pos = torch.full((1, 1, 3), L + s, dtype=torch.int32, device="cuda")
-        outs.append(sd.verify_layer(qs[s], w["k_new"][s].cuda(), w["v_new"][s].cuda(), pos, (16, 24, 24), cache,
-                                    0, w["base"]))
+        pos = torch.from_numpy(workloads.text_positions(L + R * s, R)[None]).cuda()
+        outs.append(sd.verify_layer(qs[s], ks[s], vs[s], pos, (16, 24, 24), cache, 0, w["base"], block=True))
     torch.cuda.synchronize()
-    assert cache.len.item() == L + steps
+    assert cache.len.item() == L + steps * R
     k64, v64 = to64(cache.k), to64(cache.v)
     for s in range(steps):
-        ref = oracle.verify_attention(to64(qs[s]), k64, v64, np.array([L + s + 1]))
-        assert np.abs(to64(outs[s]) - ref).max() <= ATTN_ATOL
+        ref = oracle.verify_attention(to64(qs[s]), k64, v64, np.array([L + R * (s + 1)]), block=True)
+        assert attn_within(to64(outs[s]), ref)
     assert sd.get_device_error() == 0
 
 
-def test_layer_small_tiles_overflow_sets_error_and_leaves_scene():
+def test_block_masked_layer_overflow_sets_error_and_leaves_scene():
     case = _case(1, 16, 4, 0, [300], layer=820)
     q, k, v, p, cache = gpu_case(case)
     cache.len.fill_(case.cap)            # one more row does not fit
     out = torch.full_like(q, 5.0)
     k0 = cache.k.clone()
     sd.get_device_error()
-    sd.verify_layer(q, k, v, p, case.sections, cache, 0, 1e6, out=out)
+    sd.verify_layer(q, k, v, p, case.sections, cache, 0, 1e6, out=out, block=True)
     assert sd.get_device_error() & sd.SD_DEVERR_KV_OVERFLOW
     assert cache.len.item() == case.cap
     assert torch.all(out == 5.0)
-    assert bool(((cache.k == k0) | (cache.k.isnan() & k0.isnan())).all())
-
-
-def test_small_tiles_are_served_by_the_small_tile_kernel():
-    # the shapes above must reach the small-tile kernel itself (a shape it
-    # silently declined would still pass through the tcgen05 kernel)
-    for B, Hq, Hkv, K, prefix in SHAPES:
-        cap = max(prefix) + K + 9
-        assert sd.verify_kernel(B, K + 1, Hq, Hkv, 128, cap) == "small-tile"
-        assert sd.lib().sd_verify_kernel(B, K + 1, Hq, Hkv, 128, cap, 2) == b"small-tile"   # block mask
-        # the fused layer: from 8 (scene, KV head) clusters on; one scene of
-        # the draft's 4 KV heads stays on the tcgen05 layer kernel
-        want = "small-tile" if B * Hkv >= 8 else "tcgen05"
-        assert sd.verify_kernel(B, K + 1, Hq, Hkv, 128, cap, True) == want
-    assert sd.verify_kernel(1, 8, 32, 8, 128, 4104) == "tcgen05"        # 32 rows
-    assert sd.verify_kernel(1, 8, 32, 8, 128, 4104, True) == "tcgen05"
-    assert sd.verify_kernel(1, 5, 4, 1, 64, 300) == "mma.sync"          # head_dim 64
-    assert sd.verify_kernel(1, 5, 4, 1, 64, 300, True) == "three kernels"
+    assert _same(cache.k, k0)
