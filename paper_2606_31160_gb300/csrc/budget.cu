@@ -23,7 +23,10 @@
 //                                          non-visual keys the row sees
 #include "common.cuh"
 
+#include <cuda.h>  // CUtensorMap and its enums (header only; no libcuda link)
+
 #include <math.h>
+#include <mutex>
 
 SD_DEFINE_ERROR_ACCESSOR(sd_take_error_budget)
 
@@ -128,12 +131,13 @@ __device__ __forceinline__ void mma_bf16(float (&c)[4], const uint32_t (&a)[4], 
 // key fragments serve every tile of the pass.
 constexpr int kTiles = 2;
 constexpr int kPassRows = 16 * kTiles;
+constexpr int kChunkKeys = 320;  // keys a CTA stages at once (10 boxes of 32)
 
 // two CTAs an SM (at most 128 registers a thread), so that clusters of 16
 // need only 8 SMs of a GPC and every cluster of a launch fits in one wave
 template <int D>
 __global__ void __launch_bounds__(kThreads, 2)
-    budget_kernel(const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* __restrict__ kc,
+    budget_kernel(const __grid_constant__ CUtensorMap tm_k, const __nv_bfloat16* __restrict__ q,
                   const int32_t* __restrict__ len, const int32_t* __restrict__ n_visual, int R, int Hq,
                   int Hkv, int cap, float scale, float* __restrict__ mass, float* __restrict__ entropy) {
   __shared__ RowState red[kWarps][kPassRows];
@@ -161,7 +165,21 @@ __global__ void __launch_bounds__(kThreads, 2)
   }
   const int k_lo = ok ? static_cast<int>(static_cast<long long>(rank) * n_keys / S) : 0;
   const int k_hi = ok ? static_cast<int>(static_cast<long long>(rank + 1) * n_keys / S) : 0;
-  const __nv_bfloat16* kb = kc + (static_cast<long long>(b) * Hkv + kvh) * cap * D;
+  // the CTA's keys are staged in shared memory a chunk of up to kChunkKeys at
+  // a time (one TMA round trip a chunk): 32-key boxes of 64 columns with the
+  // 128-byte swizzle, one region per 64-column half
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t kbuf = (static_cast<uint32_t>(__cvta_generic_to_shared(smem_raw)) + 1023u) & ~1023u;
+  __shared__ __align__(8) uint64_t chunk_bar;
+  const uint32_t bar = static_cast<uint32_t>(__cvta_generic_to_shared(&chunk_bar));
+  if (threadIdx.x == 0) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(bar) : "memory");
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  __syncthreads();
+  const int n_chunks = (k_hi - k_lo + kChunkKeys - 1) / kChunkKeys;
+  int loaded = -1;
+  uint32_t phase = 0;
   for (int m0 = 0; m0 < M; m0 += kPassRows) {
     // query fragments of rows m0 + 16 u + gq and + 8 (zero past M); the keys
     // each row sees (causal over the new rows); one state per row
@@ -184,16 +202,51 @@ __global__ void __launch_bounds__(kThreads, 2)
         st[u][h2] = row_empty();
       }
 #pragma unroll 1
-    for (int kb0 = k_lo + 8 * warp; kb0 < k_hi; kb0 += 8 * kWarps) {
-      // this lane's key of the block for the B fragments (clamped into the range)
-      const int kn = min(kb0 + gq, k_hi - 1);
-      const __nv_bfloat16* kr = kb + static_cast<long long>(kn) * D;
+    for (int ci = 0; ci < n_chunks; ++ci) {  // block-uniform
+      const int c0 = k_lo + ci * kChunkKeys, nk = min(kChunkKeys, k_hi - c0);
+      if (loaded != ci) {
+        __syncthreads();  // every warp is done with the chunk in place
+        if (threadIdx.x == 0) {
+          const int nbox = (nk + 31) / 32;
+          asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar),
+                       "r"(static_cast<uint32_t>(nbox * 32 * 128 * (D / 64)))
+                       : "memory");
+          for (int bx = 0; bx < nbox; ++bx)
+#pragma unroll
+            for (int hf = 0; hf < D / 64; ++hf)
+              asm volatile(
+                  "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+                  " [%0], [%1, {%3, %4, %5}], [%2];" ::"r"(kbuf + hf * kChunkKeys * 128 + bx * 32 * 128),
+                  "l"(reinterpret_cast<uint64_t>(&tm_k)), "r"(bar), "r"(hf * 64), "r"(c0 + bx * 32),
+                  "r"(b * Hkv + kvh)
+                  : "memory");
+        }
+        // bounded wait on the chunk's copies
+        uint32_t done = 0;
+        for (uint32_t it = 0; it < (1u << 22) && !done; ++it)
+          asm volatile(
+              "{\n\t.reg .pred p;\n\tmbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+              "selp.u32 %0, 1, 0, p;\n\t}"
+              : "=r"(done)
+              : "r"(bar), "r"(phase)
+              : "memory");
+        if (!done && threadIdx.x == 0) sd_set_error(SD_DEVERR_TIMEOUT);
+        phase ^= 1u;
+        loaded = ci;
+      }
+#pragma unroll 1
+    for (int kb = 8 * warp; kb < nk; kb += 8 * kWarps) {
+      const int kb0 = c0 + kb;  // the block's first key
+      // B fragments of the block's 8 keys from the staged rows: ldmatrix of
+      // (8 keys x 8 d) matrices, two k16 steps a load
       uint32_t bf[D / 16][2];
 #pragma unroll
-      for (int ks = 0; ks < D / 16; ++ks) {
-        const int d0 = ks * 16 + 2 * tq;
-        bf[ks][0] = __ldg(reinterpret_cast<const uint32_t*>(kr + d0));
-        bf[ks][1] = __ldg(reinterpret_cast<const uint32_t*>(kr + d0 + 8));
+      for (int ks = 0; ks < D / 16; ks += 2) {
+        const int row = kb + (lane & 7), chunk = 2 * ks + (lane >> 3);
+        const uint32_t addr = kbuf + (chunk >> 3) * kChunkKeys * 128 + row * 128 + (((chunk & 7) ^ (row & 7)) << 4);
+        asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+                     : "=r"(bf[ks][0]), "=r"(bf[ks][1]), "=r"(bf[ks + 1][0]), "=r"(bf[ks + 1][1])
+                     : "r"(addr));
       }
       int seg[2];
 #pragma unroll
@@ -222,6 +275,7 @@ __global__ void __launch_bounds__(kThreads, 2)
           row_block(st[u][h2], y, seg, bm);
         }
       }
+    }
     }
     // the four lanes of a row (fixed butterfly), then the warps in order
 #pragma unroll
@@ -278,6 +332,42 @@ __global__ void __launch_bounds__(kThreads, 2)
   }
 }
 
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult qres;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &qres) == cudaSuccess &&
+        qres == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  });
+  return fn;
+}
+
+// [B*Hkv][cap][D] bf16 keys as a 3-D tensor; boxes of 64 columns x 32 rows,
+// 128-byte swizzle (the layout the kernel's ldmatrix reads)
+bool make_key_map(CUtensorMap* map, void* base, int D, int cap, int planes) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[3] = {static_cast<cuuint64_t>(D), static_cast<cuuint64_t>(cap), static_cast<cuuint64_t>(planes)};
+  cuuint64_t strides[2] = {static_cast<cuuint64_t>(D) * 2, static_cast<cuuint64_t>(cap) * static_cast<cuuint64_t>(D) * 2};
+  cuuint32_t box[3] = {64, 32, 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, base, dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+            CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int D>
+constexpr int smem_bytes() { return kChunkKeys * 128 * (D / 64) + 1024; }
+
 }  // namespace
 
 extern "C" sd_status sd_attention_budget(const void* q, const sd_kv_cache* cache, int R, int Hq, float scale,
@@ -299,7 +389,8 @@ extern "C" sd_status sd_attention_budget(const void* q, const sd_kv_cache* cache
   int S = 1;
   while (S < 16 && static_cast<long long>(cap) > 256LL * S) S *= 2;
   const auto* qq = static_cast<const __nv_bfloat16*>(q);
-  const auto* kk = static_cast<const __nv_bfloat16*>(cache->k);
+  CUtensorMap tk;
+  if (!make_key_map(&tk, cache->k, D, cap, B * Hkv)) return SD_ERR_CUDA;
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -310,23 +401,31 @@ extern "C" sd_status sd_attention_budget(const void* q, const sd_kv_cache* cache
   attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.gridDim = dim3(S, Hkv, B);
   cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.dynamicSmemBytes = D == 128 ? smem_bytes<128>() : smem_bytes<64>();
   cfg.stream = st;
   cfg.attrs = attr;
   cfg.numAttrs = 2;
   cudaError_t e;
-  // clusters of 16 are non-portable: allowed once per device and kernel
+  // clusters of 16 are non-portable and the staging buffer passes 48 KB:
+  // both allowed once per device and kernel
   static bool allowed[64][2];
   int dev = 0;
-  if (S > 8 && cudaGetDevice(&dev) == cudaSuccess && dev >= 0 && dev < 64 && !allowed[dev][D == 128]) {
-    if (D == 128) cudaFuncSetAttribute(budget_kernel<128>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-    else cudaFuncSetAttribute(budget_kernel<64>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  if (cudaGetDevice(&dev) == cudaSuccess && dev >= 0 && dev < 64 && !allowed[dev][D == 128]) {
+    if (D == 128) {
+      cudaFuncSetAttribute(budget_kernel<128>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+      cudaFuncSetAttribute(budget_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes<128>());
+    } else {
+      cudaFuncSetAttribute(budget_kernel<64>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+      cudaFuncSetAttribute(budget_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes<64>());
+    }
+    (void)cudaGetLastError();
     allowed[dev][D == 128] = true;
   }
   if (D == 128) {
-    e = cudaLaunchKernelEx(&cfg, budget_kernel<128>, qq, kk, static_cast<const int32_t*>(cache->len), n_visual, R, Hq,
+    e = cudaLaunchKernelEx(&cfg, budget_kernel<128>, tk, qq, static_cast<const int32_t*>(cache->len), n_visual, R, Hq,
                            Hkv, cap, sc, mass, entropy);
   } else {
-    e = cudaLaunchKernelEx(&cfg, budget_kernel<64>, qq, kk, static_cast<const int32_t*>(cache->len), n_visual, R, Hq,
+    e = cudaLaunchKernelEx(&cfg, budget_kernel<64>, tk, qq, static_cast<const int32_t*>(cache->len), n_visual, R, Hq,
                            Hkv, cap, sc, mass, entropy);
   }
   if (e != cudaSuccess) {

@@ -41,6 +41,8 @@ def test_target_layer_budget():
     (3, 5, 4, 1, 64, [1, 17, 300], [0, 9, 300]),     # no visual keys / all visual
     (2, 17, 32, 8, 128, [2000, 513], [1750, 448]),   # K = 16: three row groups
     (1, 1, 16, 4, 128, [4096], [3584]),              # draft-shaped single row
+    (1, 8, 32, 8, 128, [8000], [7000]),              # two staged chunks of keys a CTA
+    (1, 17, 32, 8, 128, [6000], [5000]),             # two chunks, reloaded for each of three row groups
 ])
 def test_random_shapes(B, R, Hq, Hkv, D, prefix, nvis):
     rng = np.random.default_rng(B * 10 + R)
