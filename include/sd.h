@@ -195,23 +195,22 @@ sd_status sd_verify_attention_ex(const void* q, const sd_kv_cache* cache, void* 
                                  size_t ws_bytes, sd_stream_t stream);
 
 /*
- * Cluster size of the tcgen05 verify-attention kernels and the small-tile
- * layer kernel (sd_verify_attention and sd_verify_layer, head_dim 128): one
+ * Cluster size of the tcgen05 verify-attention kernels (sd_verify_attention
+ * and sd_verify_layer, head_dim 128): one
  * thread-block cluster of `cluster_size` CTAs per (scene, KV head) splits that
  * head's keys evenly and merges the partial softmax states in distributed
  * shared memory (the split-L form of Eq. verify). 0 (the default) lets every
  * call choose from the occupancy of each size and the capacity; 1, 2, 4, 6, 8
  * or 16 forces that size for later calls on every device (a size of which no
- * cluster fits on the device, or which the kernel does not build -- 6 on the
- * small-tile kernel -- falls back to the automatic choice). Process-wide, host-only, no
+ * cluster fits on the device falls back to the automatic choice). Process-wide, host-only, no
  * device work; results are the same for every size up to fp32 rounding order.
  * Returns SD_ERR_INVALID_ARG for any other value.
  */
 sd_status sd_set_cluster_size(int cluster_size);
 
 /*
- * Which kernel serves a shape on the CURRENT device: "small-tile",
- * "tcgen05" or "mma.sync" for sd_verify_attention (layer = 0), and for
+ * Which kernel serves a shape on the CURRENT device: "tcgen05" or
+ * "mma.sync" for sd_verify_attention (layer = 0), and for
  * sd_verify_layer (layer = 1, or 2 with SD_LAYER_BLOCK_MASK; "three kernels"
  * when the layer runs as the rotation, append and attention kernels in
  * sequence); "unsupported" for a shape neither call takes. Host-only, no
@@ -280,10 +279,8 @@ size_t sd_verify_layer_workspace(int B, int R, int Hq, int Hkv, int D, int capac
  *   SD_LAYER_BLOCK_MASK: the attention uses the block mask (as
  *   SD_ATTN_BLOCK_MASK of sd_verify_attention_ex).
  * For head_dim 128 this is one kernel: the tcgen05 kernel for G * R <= 128
- * and R <= 31 (R <= 16 when G * R <= 32), except that its 32-row tile is
- * causal only, so block-masked layers with G * R <= 16 take the small-tile
- * kernel (one thread-block cluster of up to 16 CTAs per KV head, mma.sync
- * tiles of 16 packed rows) and those with 16 < G * R <= 32 the three kernels;
+ * and R <= 31 (R <= 16 when a causal layer has G * R <= 32: its 32-row tile
+ * is causal only, so block-masked layers always take the 64-row tile);
  * other shapes run the three kernels in sequence (sd_verify_kernel names the
  * choice). A scene whose append would pass the
  * capacity sets SD_DEVERR_KV_OVERFLOW and is left untouched.

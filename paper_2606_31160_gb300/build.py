@@ -31,7 +31,7 @@ ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC,-O2",
               "--expt-relaxed-constexpr", "-I" + INCLUDE] + ARCH
 SOURCES = ["api.cu", "rope.cu", "kv.cu", "attention.cu", "attention_tc.cu", "layer.cu",
-           "accept_greedy.cu", "accept_sample.cu", "budget.cu", "decode.cu"]
+           "accept_greedy.cu", "accept_sample.cu", "budget.cu"]
 
 
 def nvcc_path():

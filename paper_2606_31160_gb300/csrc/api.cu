@@ -27,8 +27,7 @@ extern "C" sd_status sd_get_device_error(sd_stream_t stream, uint32_t* bits) {
   cudaError_t (*take[])(uint32_t*) = {sd_take_error_rope, sd_take_error_kv,
                                       sd_take_error_attention, sd_take_error_attention_tc,
                                       sd_take_error_greedy,
-                                      sd_take_error_sample, sd_take_error_budget,
-                                      sd_take_error_decode};
+                                      sd_take_error_sample, sd_take_error_budget};
   for (auto fn : take) {
     if (fn(bits) != cudaSuccess) {
       (void)cudaGetLastError();

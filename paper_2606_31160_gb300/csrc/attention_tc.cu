@@ -459,8 +459,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   // prefix (and len) before the dependency wait; the block mask
   const bool early = kMode == 1 || (kMode == 2 && (a.early & 1) != 0);
   // (the fused layer's 32-row tile takes no block mask: its callers are the
-  // target's causal verify steps; the host sends block-masked 32-row layers
-  // through the separate kernels)
+  // target's causal verify steps; the host sends block-masked layers of up to
+  // 32 packed rows to the 64-row tile)
   const bool block = kMode == 0 ? a.early != 0 : ((kMode == 2 || kR == 64) && (a.early & 2) != 0);
   constexpr int kS = C::kStages;
   constexpr int kRpt = C::kRpt;
@@ -1524,16 +1524,17 @@ extern "C" sd_status sd_set_cluster_size(int cluster_size) {
   return SD_ERR_INVALID_ARG;
 }
 
-int sd_internal_forced_cluster() { return g_forced_cluster.load(); }
-
-static TcPlan tc_plan(int B, int R, int Hq, int Hkv, int D, int cap, int max_cs = 16) {
+// rows64: the 64-row tile even for G * R <= 32 (the block-masked fused layer:
+// the 32-row fused kernel is compiled causal only, and an N = 64 product
+// costs about what an N = 32 one does)
+static TcPlan tc_plan(int B, int R, int Hq, int Hkv, int D, int cap, int max_cs = 16, bool rows64 = false) {
   TcPlan p;
   if (!tc_enabled() || D != kD || Hkv <= 0 || Hq % Hkv || R <= 0) return p;
   const int M = (Hq / Hkv) * R;
   if (M > 2 * 64) return p;
   DevState* s = state();
   if (!s || !s->ok) return p;
-  p.rows = M <= 32 ? 32 : 64;
+  p.rows = M <= 32 && !rows64 ? 32 : 64;
   p.mblocks = (M + p.rows - 1) / p.rows;
   const int* active = s->active[p.rows == 32 ? 0 : 1];
   // sizes above max_cs are not used (the fused merge holds csize partials and
@@ -1553,8 +1554,7 @@ bool sd_internal_tc_serves(int B, int R, int Hq, int Hkv, int D, int cap) {
 
 bool sd_internal_tc_serves_layer(int B, int R, int Hq, int Hkv, int D, int cap, bool block) {
   if (R > 32) return false;
-  const TcPlan plan = tc_plan(B, R, Hq, Hkv, D, cap, 32 - R);
-  if (block && plan.rows == 32) return false;  // the 32-row fused kernel is causal only
+  const TcPlan plan = tc_plan(B, R, Hq, Hkv, D, cap, 32 - R, block);
   return plan.cs > 0 && R <= (plan.rows == 32 ? Cfg<32>::kMaxNew : Cfg<64>::kMaxNew);
 }
 
@@ -1648,10 +1648,10 @@ sd_status sd_internal_verify_layer_tc(void* q, void* k_new, const void* v_new, c
   // the new rows are held in shared memory (16 with the 32-row tile, 32 with
   // the 64-row tile) and merged in the lanes of one warp with the partials
   if (R > 32) return SD_OK;
-  const TcPlan plan = tc_plan(B, R, Hq, Hkv, cache->head_dim, cache->capacity, 32 - R);
+  // block-masked layers take the 64-row tile (the 32-row fused kernel is causal only)
+  const TcPlan plan = tc_plan(B, R, Hq, Hkv, cache->head_dim, cache->capacity, 32 - R, block != 0);
   if (plan.cs <= 0) return SD_OK;
   if (R > (plan.rows == 32 ? Cfg<32>::kMaxNew : Cfg<64>::kMaxNew)) return SD_OK;
-  if (block && plan.rows == 32) return SD_OK;  // the 32-row fused kernel is causal only
   TcArgs a = {};
   a.q = static_cast<const __nv_bfloat16*>(q);
   a.out = static_cast<__nv_bfloat16*>(out);

@@ -36,7 +36,6 @@ cudaError_t sd_take_error_attention_tc(uint32_t* bits);
 cudaError_t sd_take_error_greedy(uint32_t* bits);
 cudaError_t sd_take_error_sample(uint32_t* bits);
 cudaError_t sd_take_error_budget(uint32_t* bits);
-cudaError_t sd_take_error_decode(uint32_t* bits);
 
 // Verify attention on the tcgen05 path (attention_tc.cu). Sets *handled when
 // the shape is one it serves (head_dim 128, G * R <= 32) and it launched.
@@ -55,18 +54,6 @@ sd_status sd_internal_verify_layer_tc(void* q, void* k_new, const void* v_new, c
                                       const RopeTable& tab, const sd_kv_cache* cache, void* out,
                                       int R, int Hq, float scale_log2, uint32_t* ticket, int early,
                                       int block, cudaStream_t stream, bool* handled);
-
-// Cluster size forced by sd_set_cluster_size (0: chosen per call).
-int sd_internal_forced_cluster();
-
-// The small-tile layer kernel (decode.cu): head_dim 128 and G * R <= 16 query
-// rows per KV head, block-masked layers. Whether it serves a shape on the
-// current device, and the layer on it (*handled is set when it launched):
-bool sd_internal_decode_serves(int B, int R, int Hq, int Hkv, int D, int cap, bool block);
-sd_status sd_internal_verify_layer_dec(void* q, void* k_new, const void* v_new, const int32_t* pos,
-                                       const RopeTable& tab, const sd_kv_cache* cache, void* out, int R,
-                                       int Hq, float scale_log2, uint32_t* ticket, int early, int block,
-                                       cudaStream_t stream, bool* handled);
 
 // ---------------------------------------------------------------------------
 // Host helpers

@@ -2,7 +2,7 @@
 // Sec. 4.2), the KV append (Eq. commit) and the verify attention (Eq. verify,
 // Sec. 3.2) of one attention layer as one call.
 //
-// On the tcgen05 path (head_dim 128, G * R <= 128, R <= 16) it is one kernel launch that
+// On the tcgen05 path (head_dim 128, G * R <= 128, R <= 31) it is one kernel launch that
 // may overlap the previous layer: the cached prefix of a layer does not
 // depend on the layer before it, so with SD_LAYER_PREFIX_EARLY the kernel is
 // a programmatic dependent launch that starts streaming that prefix while the
@@ -55,14 +55,6 @@ extern "C" sd_status sd_verify_layer(void* q, void* k_new, const void* v_new, co
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   auto* ticket = static_cast<uint32_t*>(workspace);
   bool handled = false;
-  // block-masked layers of up to 16 packed rows per KV head: the small-tile
-  // kernel (the tcgen05 kernel's 32-row layer tile is causal only); the
-  // others: the tcgen05 kernel
-  {
-    const sd_status s = sd_internal_verify_layer_dec(q, k_new, v_new, pos, tab, cache, out, R, Hq, scale_log2,
-                                                     ticket, flags & SD_LAYER_PREFIX_EARLY, block, st, &handled);
-    if (handled) return s;
-  }
   const sd_status s = sd_internal_verify_layer_tc(q, k_new, v_new, pos, tab, cache, out, R, Hq,
                                                   scale_log2, ticket, flags & SD_LAYER_PREFIX_EARLY,
                                                   block, st, &handled);
@@ -81,7 +73,6 @@ extern "C" const char* sd_verify_kernel(int B, int R, int Hq, int Hkv, int D, in
   if (B <= 0 || R <= 0 || Hq <= 0 || Hkv <= 0 || capacity <= 0 || Hq % Hkv || (D != 64 && D != 128) ||
       static_cast<long long>(Hq / Hkv) * R > 128)
     return "unsupported";
-  if (layer != 0 && sd_internal_decode_serves(B, R, Hq, Hkv, D, capacity, layer > 1)) return "small-tile";
   if (layer) return sd_internal_tc_serves_layer(B, R, Hq, Hkv, D, capacity, layer > 1) ? "tcgen05" : "three kernels";
   return sd_internal_tc_serves(B, R, Hq, Hkv, D, capacity) ? "tcgen05" : "mma.sync";
 }

@@ -375,7 +375,7 @@ def set_cluster_size(cluster_size=0):
 
 def verify_kernel(B, R, Hq, Hkv, D, capacity, layer=False):
     """Name of the kernel that serves this shape on the current device
-    (sd_verify_kernel): "small-tile", "tcgen05", "mma.sync" or "three kernels"."""
+    (sd_verify_kernel): "tcgen05", "mma.sync" or "three kernels"."""
     return lib().sd_verify_kernel(B, R, Hq, Hkv, D, capacity, 1 if layer else 0).decode()
 
 

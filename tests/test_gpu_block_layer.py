@@ -1,9 +1,10 @@
-"""The small-tile layer kernel: fused verify layers with the block mask of the
-block-diffusion drafts (every new row sees the prefix and all R new rows) and
-up to 16 packed query rows per KV head, against the float64 oracle and against
-the separate rotation, append and attention calls: ragged scenes, stale NaN
-rows, an empty prefix and prefixes shorter than one 32-key block, every
-cluster size the launch picks, interleaved M-RoPE, chained dependent launches,
+"""Short block-masked fused layers on the tcgen05 kernel's 64-row tile: verify
+layers with the block mask of the block-diffusion drafts (Sec. 5: every new
+row sees the prefix and all R new rows) and up to 32 packed query rows per KV
+head, which the causal-only 32-row tile does not take, against the float64
+oracle and against the separate rotation, append and attention calls: ragged
+scenes, stale NaN rows, an empty prefix and prefixes shorter than one key
+tile, every cluster size, interleaved M-RoPE, chained dependent launches,
 sequential steps on one cache, and the overflow error."""
 import numpy as np
 import pytest
@@ -21,10 +22,10 @@ def _lib():
     ensure_lib()
 
 
-def _case(B, Hq, Hkv, K, prefix, layer, cap_pad=8, tail=float("nan"), sections=(16, 24, 24)):
+def _case(B, Hq, Hkv, K, prefix, layer, cap_pad=8, tail=float("nan"), sections=(16, 24, 24), D=128):
     R = K + 1
     qpos = np.stack([workloads.text_positions(int(p) + 1, R) for p in prefix])
-    return workloads.verify_case(workloads.SWEEP, B=B, Hq=Hq, Hkv=Hkv, D=128, prefix=prefix, K=K,
+    return workloads.verify_case(workloads.SWEEP, B=B, Hq=Hq, Hkv=Hkv, D=D, prefix=prefix, K=K,
                                  sections=sections, base=1e6, query_pos=qpos, cap=max(prefix) + R + cap_pad,
                                  layer=layer, tail_fill=tail)
 
@@ -37,35 +38,37 @@ def _same(x, y):  # stale cache rows hold NaN on both sides
     return bool(((x == y) | (x.isnan() & y.isnan())).all())
 
 
-# (B, Hq, Hkv, K, prefix): the draft's shape (G*R = 4), K = 1..3 of the 8B
-# target (8..16 rows), one KV head per query head with 16 rows, ragged scenes
-# with an empty prefix and prefixes shorter than one 32-key block
+# (B, Hq, Hkv, K, prefix): the draft's shape (G*R = 4), K = 1..3 and 7 of the
+# 8B target (8..32 rows), one KV head per query head with 16 rows, ragged
+# scenes with an empty prefix and prefixes shorter than one key tile
 SHAPES = [
     (1, 16, 4, 0, [4096]),
     (2, 32, 8, 1, [4096, 3001]),
     (3, 32, 8, 3, [0, 31, 1000]),
+    (1, 32, 8, 7, [2500]),
     (2, 8, 8, 15, [77, 2048]),
     (4, 4, 1, 2, [1, 33, 64, 500]),
 ]
 
 
-def test_block_masked_short_layers_take_the_small_tile_kernel():
-    # block-masked layers of <= 16 packed rows take this kernel (the tcgen05
-    # layer kernel's 32-row tile is causal only); causal layers and attention
-    # calls of the same shapes take the tcgen05 kernel
+def test_block_masked_short_layers_take_the_tcgen05_kernel():
+    # block-masked layers of <= 32 packed rows run as one tcgen05 launch (on
+    # the 64-row tile), as causal layers and attention calls of the same shapes
     for B, Hq, Hkv, K, prefix in SHAPES:
         cap = max(prefix) + K + 9
-        assert sd.lib().sd_verify_kernel(B, K + 1, Hq, Hkv, 128, cap, 2) == b"small-tile"
+        assert sd.lib().sd_verify_kernel(B, K + 1, Hq, Hkv, 128, cap, 2) == b"tcgen05"
         assert sd.verify_kernel(B, K + 1, Hq, Hkv, 128, cap, True) == "tcgen05"
         assert sd.verify_kernel(B, K + 1, Hq, Hkv, 128, cap) == "tcgen05"
-    assert sd.lib().sd_verify_kernel(1, 8, 32, 8, 128, 4104, 2) == b"three kernels"   # 32 rows, causal tile
-    assert sd.lib().sd_verify_kernel(1, 17, 32, 8, 128, 4113, 2) == b"tcgen05"        # 68 rows: 64-row tile
+    assert sd.lib().sd_verify_kernel(1, 17, 32, 8, 128, 4113, 2) == b"tcgen05"        # 68 rows: two m-blocks
     assert sd.verify_kernel(1, 5, 4, 1, 64, 300, True) == "three kernels"              # head_dim 64
 
 
-@pytest.mark.parametrize("B,Hq,Hkv,K,prefix", SHAPES)
-def test_block_masked_layer_matches_oracle_and_separate_calls(B, Hq, Hkv, K, prefix):
-    case = _case(B, Hq, Hkv, K, prefix, layer=760 + K)
+@pytest.mark.parametrize("B,Hq,Hkv,K,prefix,D", [s + (128,) for s in SHAPES] + [(2, 8, 2, 3, [300, 5], 64)])
+def test_block_masked_layer_matches_oracle_and_separate_calls(B, Hq, Hkv, K, prefix, D):
+    # head_dim 64 runs the layer as the three kernels
+    sections = (16, 24, 24) if D == 128 else (8, 12, 12)
+    case = _case(B, Hq, Hkv, K, prefix, layer=760 + K, sections=sections, D=D)
+    assert sd.verify_kernel(B, K + 1, Hq, Hkv, D, case.cap, True) == ("tcgen05" if D == 128 else "three kernels")
     # separate calls: rotation kernel, append kernel, block-masked attention
     qa, ka, va, pa, ca = gpu_case(case)
     sd.rope_apply(qa, ka, pa, case.sections, 0, case.base)
@@ -87,16 +90,21 @@ def test_block_masked_layer_matches_oracle_and_separate_calls(B, Hq, Hkv, K, pre
     assert sd.get_device_error() == 0
 
 
-@pytest.mark.parametrize("B,Hkv,L", [(1, 4, 2048), (2, 8, 2048), (8, 4, 2048), (24, 4, 1000), (48, 4, 700)])
-def test_block_masked_layer_every_cluster_size(B, Hkv, L):
-    # the launch sizes its clusters from B * Hkv (16, 4, 4, 1 CTAs per head;
-    # the last case runs past one wave): each size merges the same states
-    # through distributed shared memory
+@pytest.mark.parametrize("cluster", [0, 1, 2, 4, 6, 8, 16])
+@pytest.mark.parametrize("B,Hkv,L", [(1, 4, 2048), (3, 8, 1000)])
+def test_block_masked_layer_every_cluster_size(cluster, B, Hkv, L):
+    # each cluster size (0: the launch's own choice) splits a head's keys and
+    # merges the same states through distributed shared memory
     prefix = [L - 13 * b for b in range(B)]
-    case = _case(B, 4 * Hkv, Hkv, 1, prefix, layer=740 + B, tail=0.0)
-    assert sd.lib().sd_verify_kernel(B, 2, 4 * Hkv, Hkv, 128, case.cap, 2) == b"small-tile"
+    case = _case(B, 4 * Hkv, Hkv, 1, prefix, layer=740 + B + cluster, tail=0.0)
+    assert sd.lib().sd_verify_kernel(B, 2, 4 * Hkv, Hkv, 128, case.cap, 2) == b"tcgen05"
     q, k, v, p, cache = gpu_case(case)
-    out = sd.verify_layer(q, k, v, p, case.sections, cache, 0, case.base, block=True)
+    sd.set_cluster_size(cluster)
+    try:
+        out = sd.verify_layer(q, k, v, p, case.sections, cache, 0, case.base, block=True)
+        torch.cuda.synchronize()
+    finally:
+        sd.set_cluster_size(0)
     ref = _oracle_block(q, cache)
     assert attn_within(to64(out), ref), np.abs(to64(out) - ref).max()
     assert sd.get_device_error() == 0
