@@ -1047,6 +1047,19 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int sw = kR == 32 ? (kl >> 1) & 3 : kl & 7;
 #pragma unroll
         for (int j0 = 0; j0 < kRpt; j0 += 16) {
+          // 16 rows past the tile's existing rows (warp-uniform): no scores to
+          // read and no P to write; their P columns stay stale and reach only
+          // O columns that are never read. The buffer release and the PV wait
+          // stay, so every barrier phase still completes in order.
+          if (row0 + j0 >= rows_in) {
+            if (j0 + 16 >= kRpt) {
+              tc_fence_before();
+              __syncwarp();
+              if (lane == 0) mbar_arrive(SFREE(T));
+            }
+            if (T >= 2 && j0 == 0) mbar_wait(PVDONE(T - 2), ring_parity(T - 2));
+            continue;
+          }
           uint32_t r[16];
           tmem_ld16(tmem_s + kR * (T % kSB) + row0 + j0 + lane_off, r);
           if (j0 + 16 >= kRpt) {
