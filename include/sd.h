@@ -187,6 +187,9 @@ sd_status sd_verify_attention(const void* q, const sd_kv_cache* cache, void* out
  * G * R > 32) the call is then a programmatic dependent launch that reads len
  * and streams the whole cache while its predecessor still runs, and reads q
  * only after the predecessor has completed; other shapes ignore the flag.
+ * Without the flag those shapes are programmatic dependent launches too, but
+ * the kernel waits for its predecessor to complete before its first global
+ * access, so only its launch and set-up overlap it.
  * Other bits: SD_ERR_INVALID_ARG. Everything else as sd_verify_attention
  * (which is this call with flags 0).
  */
@@ -276,6 +279,10 @@ size_t sd_verify_layer_workspace(int B, int R, int Hq, int Hkv, int D, int capac
  *   pass). The call is then a programmatic dependent launch that reads len and
  *   pos and streams the cached prefix while its predecessor still runs; q,
  *   k_new and v_new are read only after the predecessor has completed.
+ *   Without the flag the tcgen05 kernel is still a programmatic dependent
+ *   launch, but it waits for its predecessor to complete before its first
+ *   global access (only its launch and set-up overlap), so such calls may
+ *   share a workspace.
  *   SD_LAYER_BLOCK_MASK: the attention uses the block mask (as
  *   SD_ATTN_BLOCK_MASK of sd_verify_attention_ex).
  * For head_dim 128 this is one kernel: the tcgen05 kernel for G * R <= 128

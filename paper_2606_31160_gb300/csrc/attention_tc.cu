@@ -535,7 +535,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                  : "memory");
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
-  if (kNew && !early) griddep_wait();  // len, pos and the prefix may come from the previous kernel
+  // len, pos, the rows and the prefix may come from the previous kernel: a
+  // launch without the early prefix waits here, before any global access
+  if (kNew && !early) griddep_wait();
   int* s_len = reinterpret_cast<int*>(smem + C::kOffMisc + 12);
   if (threadIdx.x == 0) {
     *s_len = a.len[b];  // the scene's length advances at the producer's end
@@ -1645,7 +1647,10 @@ sd_status sd_internal_verify_attention_tc(const void* q, const sd_kv_cache* cach
   *handled = true;
   if (mode == 2) {
     a.early = (early ? 1 : 0) | (block ? 2 : 0);
-    return launch_plan<2>(cache, a, tab, plan, early, stream);
+    // a programmatic dependent launch either way: without the flag the kernel
+    // waits before its first global access, so only its launch and set-up
+    // (barriers, tensor memory) overlap the kernel before it
+    return launch_plan<2>(cache, a, tab, plan, true, stream);
   }
   a.early = block ? 1 : 0;  // the all-keys kernel's block mask
   return launch_plan<0>(cache, a, tab, plan, false, stream);
@@ -1689,5 +1694,7 @@ sd_status sd_internal_verify_layer_tc(void* q, void* k_new, const void* v_new, c
   a.scale_log2 = scale_log2;
   *handled = true;
   if (early) return launch_plan<1>(cache, a, tab, plan, true, stream);
-  return launch_plan<3>(cache, a, tab, plan, false, stream);
+  // dependent as well: the wait comes before any global access (the draft's
+  // single-row steps, each reading the length the step before advanced)
+  return launch_plan<3>(cache, a, tab, plan, true, stream);
 }
