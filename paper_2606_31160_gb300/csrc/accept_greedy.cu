@@ -127,6 +127,7 @@ __global__ void __launch_bounds__(kThreads) greedy_kernel(const T* __restrict__ 
                                                           float2* __restrict__ part,
                                                           uint32_t* __restrict__ ticket) {
   const int c = blockIdx.x, r = blockIdx.y, b = blockIdx.z;
+  sd_pdl_enter();  // a plain launch: no wait; a programmatic successor may become resident
   const T* row = logits + (static_cast<long long>(b) * R + r) * V;
   const bool vec_ok = ((static_cast<long long>(V) * sizeof(T)) % 16 == 0) &&
                       ((reinterpret_cast<uintptr_t>(logits) & 15) == 0);
@@ -207,6 +208,7 @@ __global__ void __launch_bounds__(kCThreads, 1)
   const int rank = blockIdx.x, csize = gridDim.x, r = blockIdx.y, b = blockIdx.z;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int K = R - 1;
+  sd_pdl_enter();  // a plain launch: no wait; a programmatic successor may become resident
   if (rank == 0)  // read early: only the scene's last row uses them
     for (int j = threadIdx.x; j < K; j += kCThreads) s_draft[j] = __ldg(draft + static_cast<long long>(b) * K + j);
   const T* row = logits + (static_cast<long long>(b) * R + r) * V;

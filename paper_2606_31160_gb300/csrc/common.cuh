@@ -73,6 +73,25 @@ static inline int sd_num_sms() {
   return cached[dev];
 }
 
+// Programmatic dependent launch of a kernel that begins with sd_pdl_enter():
+// it may become resident while the previous kernel on the stream finishes,
+// but reaches no global memory before that kernel has completed.
+template <typename... P, typename... A>
+static inline cudaError_t sd_launch_pdl(void (*kernel)(P...), dim3 grid, dim3 block, size_t smem,
+                                        cudaStream_t stream, A... args) {
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
+
 #define SD_CHECK_LAUNCH()                                   \
   do {                                                      \
     if (cudaPeekAtLastError() != cudaSuccess) {             \
@@ -84,6 +103,15 @@ static inline int sd_num_sms() {
 // ---------------------------------------------------------------------------
 // Device helpers
 // ---------------------------------------------------------------------------
+// First statement of a kernel launched by sd_launch_pdl: wait until the
+// previous kernel on the stream has completed (its writes visible), then let
+// the next kernel launch. Waiting first keeps a successor's pre-wait phase
+// from overlapping anything but this kernel.
+__device__ __forceinline__ void sd_pdl_enter() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 __device__ __forceinline__ float sd_bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float sd_bf16_hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
 

@@ -20,6 +20,7 @@ __global__ void __launch_bounds__(512) kv_append_kernel(uint4* __restrict__ kc, 
                                                         const uint4* __restrict__ kn,
                                                         const uint4* __restrict__ vn, int R, int hkv,
                                                         int cap, int vec_per_row) {
+  sd_pdl_enter();
   const int b = blockIdx.x;
   __shared__ int s_len;
   if (threadIdx.x == 0) {
@@ -48,6 +49,7 @@ __global__ void __launch_bounds__(512) kv_append_kernel(uint4* __restrict__ kc, 
 
 __global__ void kv_rollback_kernel(int32_t* __restrict__ len, int count, int B,
                                    const int32_t* __restrict__ committed, int n_appended) {
+  sd_pdl_enter();
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= count) return;
   const int c = committed[i % B];
@@ -73,10 +75,13 @@ extern "C" sd_status sd_kv_append(const sd_kv_cache* cache, const void* k_new, c
   if (!sd_aligned16(cache->k) || !sd_aligned16(cache->v) || !sd_aligned16(k_new) ||
       !sd_aligned16(v_new))
     return SD_ERR_INVALID_ARG;
-  kv_append_kernel<<<B, 512, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
-      static_cast<uint4*>(cache->k), static_cast<uint4*>(cache->v), cache->len,
-      static_cast<const uint4*>(k_new), static_cast<const uint4*>(v_new), R, hkv, cap, D / 8);
-  SD_CHECK_LAUNCH();
+  if (sd_launch_pdl(kv_append_kernel, dim3(B), dim3(512), 0, reinterpret_cast<cudaStream_t>(stream),
+                    static_cast<uint4*>(cache->k), static_cast<uint4*>(cache->v), cache->len,
+                    static_cast<const uint4*>(k_new), static_cast<const uint4*>(v_new), R, hkv, cap,
+                    D / 8) != cudaSuccess) {
+    (void)cudaGetLastError();
+    return SD_ERR_CUDA;
+  }
   return SD_OK;
 }
 
@@ -87,8 +92,11 @@ extern "C" sd_status sd_kv_rollback(int32_t* len, int count, int B, const int32_
   if (count == 0) return SD_OK;
   if (!len || !committed) return SD_ERR_INVALID_ARG;
   const int threads = 128;
-  kv_rollback_kernel<<<(count + threads - 1) / threads, threads, 0,
-                       reinterpret_cast<cudaStream_t>(stream)>>>(len, count, B, committed, n_appended);
-  SD_CHECK_LAUNCH();
+  if (sd_launch_pdl(kv_rollback_kernel, dim3((count + threads - 1) / threads), dim3(threads), 0,
+                    reinterpret_cast<cudaStream_t>(stream), len, count, B, committed,
+                    n_appended) != cudaSuccess) {
+    (void)cudaGetLastError();
+    return SD_ERR_CUDA;
+  }
   return SD_OK;
 }

@@ -28,6 +28,7 @@ __global__ void __launch_bounds__(256) rope_kernel(__nv_bfloat16* __restrict__ q
                                                    int rows, int hq, int hkv,
                                                    const int32_t* __restrict__ pos,
                                                    RopeTable tab) {
+  sd_pdl_enter();
   constexpr int kVecPerHead = D / 8;
   const int heads = hq + hkv;
   const long long total = (long long)rows * heads * kVecPerHead;
@@ -77,14 +78,13 @@ sd_status launch(void* q, void* k, int B, int R, int Hq, int Hkv, int D, const i
   if (blocks > cap) blocks = cap;
   auto* qp = static_cast<__nv_bfloat16*>(q);
   auto* kp = static_cast<__nv_bfloat16*>(k);
-  if (D == 64) {
-    if (flat) rope_kernel<64, true><<<(int)blocks, threads, 0, stream>>>(qp, kp, (int)rows, Hq, Hkv, pos, tab);
-    else rope_kernel<64, false><<<(int)blocks, threads, 0, stream>>>(qp, kp, (int)rows, Hq, Hkv, pos, tab);
-  } else {
-    if (flat) rope_kernel<128, true><<<(int)blocks, threads, 0, stream>>>(qp, kp, (int)rows, Hq, Hkv, pos, tab);
-    else rope_kernel<128, false><<<(int)blocks, threads, 0, stream>>>(qp, kp, (int)rows, Hq, Hkv, pos, tab);
+  auto* kern = D == 64 ? (flat ? rope_kernel<64, true> : rope_kernel<64, false>)
+                       : (flat ? rope_kernel<128, true> : rope_kernel<128, false>);
+  if (sd_launch_pdl(kern, dim3((unsigned)blocks), dim3(threads), 0, stream, qp, kp, (int)rows, Hq, Hkv,
+                    pos, tab) != cudaSuccess) {
+    (void)cudaGetLastError();
+    return SD_ERR_CUDA;
   }
-  SD_CHECK_LAUNCH();
   return SD_OK;
 }
 
