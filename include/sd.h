@@ -17,6 +17,11 @@
  *     allocates device memory and never synchronises, except
  *     sd_get_device_error(), which synchronises the stream it is given.
  *   - Every call is asynchronous on `stream` (NULL = legacy default stream).
+ *     The rotation, append and rollback kernels (and the tcgen05 attention and
+ *     layer kernels) are programmatic dependent launches: they may become
+ *     resident while the kernel before them on the stream finishes, but touch
+ *     no memory before it has completed (the early-prefix flags below are the
+ *     one exception, and say what they promise). Stream order is kept.
  *   - Problems visible on the host (bad sizes, NULL pointers, unsupported
  *     shapes, short workspace) return a status before anything is launched.
  *     Problems only visible on the device (a length past the capacity, a
