@@ -148,8 +148,7 @@ __global__ void __launch_bounds__(kThreads, 2)
   const uint32_t rank = cta_rank();
   // a programmatic dependent launch: resident while the kernel before it
   // runs, reading nothing before it has completed
-  if (threadIdx.x == 0) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-  asm volatile("griddepcontrol.wait;" ::: "memory");
+  sd_pdl_enter();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int gq = lane >> 2, tq = lane & 3;
   const int G = Hq / Hkv, M = G * R;
