@@ -1320,16 +1320,33 @@ __global__ void __launch_bounds__(kThreads, 1)
         mloc = rref;
         nx = ny = nl = 0.f;
         const float* sn = s_new + r * a.R;
+        if constexpr (kR == 64) {
+          // unrolled: the shared-memory loads of several keys issue together
+          // (a rolled loop waits on each in turn, ~0.03 us a row and key: up
+          // to 64 rows x 17 keys of a K = 16 block on one CTA)
+#pragma unroll 4
+          for (int n = 0; n < n_new; ++n) mloc = fmaxf(mloc, sn[n]);
+          const float msub = mloc == -INFINITY ? 0.f : mloc;
+#pragma unroll 4
+          for (int n = 0; n < n_new; ++n) {
+            const float w = ex2(sn[n] - msub);
+            const uint32_t v2 = *reinterpret_cast<const uint32_t*>(smem + C::kOffNewV + n * kNewRow + d * 2);
+            nl += w;
+            nx = fmaf(w, sd_bf16_lo(v2), nx);
+            ny = fmaf(w, sd_bf16_hi(v2), ny);
+          }
+        } else {
 #pragma unroll 1
-        for (int n = 0; n < n_new; ++n) mloc = fmaxf(mloc, sn[n]);
-        const float msub = mloc == -INFINITY ? 0.f : mloc;
+          for (int n = 0; n < n_new; ++n) mloc = fmaxf(mloc, sn[n]);
+          const float msub = mloc == -INFINITY ? 0.f : mloc;
 #pragma unroll 1
-        for (int n = 0; n < n_new; ++n) {
-          const float w = ex2(sn[n] - msub);
-          const uint32_t v2 = *reinterpret_cast<const uint32_t*>(smem + C::kOffNewV + n * kNewRow + d * 2);
-          nl += w;
-          nx = fmaf(w, sd_bf16_lo(v2), nx);
-          ny = fmaf(w, sd_bf16_hi(v2), ny);
+          for (int n = 0; n < n_new; ++n) {
+            const float w = ex2(sn[n] - msub);
+            const uint32_t v2 = *reinterpret_cast<const uint32_t*>(smem + C::kOffNewV + n * kNewRow + d * 2);
+            nl += w;
+            nx = fmaf(w, sd_bf16_lo(v2), nx);
+            ny = fmaf(w, sd_bf16_hi(v2), ny);
+          }
         }
       }
       const float* part = recv + r * kRowF;  // rank c's partial at part + c * rpc * kRowF
