@@ -116,3 +116,56 @@ def test_kernel_query_rejects_unsupported_shapes(lib):
     assert sd.verify_kernel(1, 8, 32, 8, 96, 4104) == "unsupported"      # head_dim
     assert sd.verify_kernel(1, 40, 32, 8, 128, 4104) == "unsupported"    # G * R > 128
     assert sd.verify_kernel(0, 8, 32, 8, 128, 4104, True) == "unsupported"
+
+
+def _layer(lib, cache, q=16, out=16, R=8, Hq=32, interleaved=0, base=1e6, scale=0.0, ws=16, ws_bytes=1 << 30,
+           flags=0, sections=(16, 24, 24)):
+    sec = (ctypes.c_int32 * 3)(*sections)
+    return lib.sd_verify_layer(ctypes.c_void_p(q), ctypes.c_void_p(16), ctypes.c_void_p(16), ctypes.c_void_p(16),
+                               sec, interleaved, base, cache, ctypes.c_void_p(out), R, Hq, scale,
+                               ctypes.c_void_p(ws), ws_bytes, flags, ctypes.c_void_p(0))
+
+
+def test_layer_host_checks_return_before_launch(lib):
+    # sd_verify_layer validates everything it can on the host, in this order:
+    # shape, head dim, flags, pointers and alignment, scale and base, the
+    # workspace, then the rotation sections; nothing reaches a device
+    ok = sd.KVCacheStruct(16, 16, 16, 1, 8, 4200, 128)
+    assert _layer(lib, None) == 1                                               # no cache
+    assert _layer(lib, ctypes.byref(ok), R=0) == 1                              # no new rows
+    assert _layer(lib, ctypes.byref(ok), Hq=30) == 1                            # Hq % Hkv
+    assert _layer(lib, ctypes.byref(sd.KVCacheStruct(16, 16, 16, 1, 8, 4200, 96))) == 2   # head dim
+    assert _layer(lib, ctypes.byref(ok), interleaved=2) == 1
+    assert _layer(lib, ctypes.byref(ok), flags=8) == 1                          # unknown flag bit
+    assert _layer(lib, ctypes.byref(sd.KVCacheStruct(0, 0, 0, 0, 8, 4200, 128)), q=0, out=0) == 0  # no scenes
+    assert _layer(lib, ctypes.byref(ok), q=0) == 1                              # NULL q
+    assert _layer(lib, ctypes.byref(ok), out=24) == 1                           # misaligned out
+    assert _layer(lib, ctypes.byref(sd.KVCacheStruct(40, 16, 16, 1, 8, 4200, 128))) == 1  # misaligned cache
+    assert _layer(lib, ctypes.byref(ok), scale=-1.0) == 1
+    assert _layer(lib, ctypes.byref(ok), scale=float("nan")) == 1
+    assert _layer(lib, ctypes.byref(ok), base=1.0) == 1
+    assert _layer(lib, ctypes.byref(ok), base=float("inf")) == 1
+    need = lib.sd_verify_layer_workspace(1, 8, 32, 8, 128, 4200)
+    assert need >= 256                                                          # the tickets at least
+    assert _layer(lib, ctypes.byref(ok), ws=0) == 3
+    assert _layer(lib, ctypes.byref(ok), ws_bytes=need - 1) == 3
+    assert _layer(lib, ctypes.byref(ok), ws=24) == 3                            # misaligned workspace
+    assert _layer(lib, ctypes.byref(ok), sections=(16, 24, 23)) == 1            # sections must sum to D / 2
+    assert lib.sd_verify_layer_workspace(0, 8, 32, 8, 128, 4200) == 0
+
+
+def test_budget_host_checks_return_before_launch(lib):
+    def budget(cache, R=8, Hq=32, scale=0.0, q=16, mass=16):
+        return lib.sd_attention_budget(ctypes.c_void_p(q), cache, R, Hq, scale, ctypes.c_void_p(16),
+                                       ctypes.c_void_p(mass), ctypes.c_void_p(16), ctypes.c_void_p(0))
+    ok = sd.KVCacheStruct(16, 16, 16, 1, 8, 4200, 128)
+    assert budget(None) == 1
+    assert budget(ctypes.byref(ok), R=0) == 1
+    assert budget(ctypes.byref(ok), Hq=12) == 1                                 # Hq % Hkv
+    assert budget(ctypes.byref(sd.KVCacheStruct(16, 16, 16, 1, 8, 4200, 80))) == 2
+    assert budget(ctypes.byref(sd.KVCacheStruct(16, 16, 16, 70000, 8, 4200, 128))) == 2   # grid z limit
+    assert budget(ctypes.byref(sd.KVCacheStruct(0, 0, 0, 0, 8, 4200, 128)), q=0, mass=0) == 0
+    assert budget(ctypes.byref(ok), mass=0) == 1
+    assert budget(ctypes.byref(sd.KVCacheStruct(8, 16, 16, 1, 8, 4200, 128))) == 1        # misaligned keys
+    assert budget(ctypes.byref(ok), scale=-0.5) == 1
+    assert budget(ctypes.byref(ok), scale=float("inf")) == 1
